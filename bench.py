@@ -1,0 +1,439 @@
+"""Benchmark of the batched embedding Get + gradient apply through the store.
+
+One step = Get(keys) into a device buffer, then apply_grad(keys, grads) (one
+Adagrad step per distinct key on its summed gradient), on the DLRM-shaped
+store: 26 tables x 4,000,000 rows x dim 128 fp32 (rows + Adagrad state resident
+in HBM, about 107 GB), 65,536 samples x 26 Zipf(1.2) lookups per step
+(1,703,936 lookups).  Inputs are seeded and synthetic, generated before timing
+and resident in HBM; each step's gradients (872 MB) and Get output (872 MB)
+exceed the 129 MB L2, so no flush is needed between steps.
+
+Prints one JSON line.  `value` is lookups (rows) per second of the whole job;
+`e2e` is the same metric through the host-buffer C-ABI calls with the copies
+inside the timed region; `roofline` is the dominant kernel's algorithmic bytes
+per launch over its CUDA-event duration against the measured HBM copy peak;
+`cpu_baseline` is the oracle (single thread, host cores) on a bounded sample.
+
+--impl reference times the oracle itself on the host, as the reference arm.
+"""
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+METRIC = "embedding rows/s (Get + grad-apply) and achieved HBM GB/s vs ~8 TB/s peak"
+UNIT = "rows/s"
+NOMINAL_HBM_GBS = 8000.0
+SEQ_SEGMENT_MAX = 32
+CHUNK = 64
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+# --- clocks during the timed region ---------------------------------------------
+class ClockSampler:
+    """Samples SM clock and clock-event reasons with nvidia-smi (-lms) and, where
+    the driver's NVML library loads, a fast NVML poll (short timed regions)."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.samples = []  # (sm_mhz, max_mhz, reasons_mask)
+        self._stop = threading.Event()
+        self._smi = None
+        self._thread = None
+        self._nvml = None
+        self._handle = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() == 0:
+                h = ctypes.c_void_p()
+                if nv.nvmlDeviceGetHandleByIndex_v2(gpu_index, ctypes.byref(h)) == 0:
+                    self._nvml, self._handle = nv, h
+        except OSError:
+            pass
+
+    def _poll(self):
+        nv, h = self._nvml, self._handle
+        clk, mx, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
+        get_reasons = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            getattr(nv, "nvmlDeviceGetCurrentClocksThrottleReasons")
+        while not self._stop.is_set():
+            if nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0 and \
+                    nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0 and \
+                    get_reasons(h, ctypes.byref(rs)) == 0:
+                self.samples.append((clk.value, mx.value, rs.value))
+            time.sleep(0.002)
+
+    def start(self):
+        os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+        try:
+            self._smi_path = os.path.join(ROOT, "gpurun_out", "clocks.csv")
+            self._smi = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.idx}",
+                 "--query-gpu=index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=open(self._smi_path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self._smi = None
+        if self._nvml is not None:
+            self._thread = threading.Thread(target=self._poll, daemon=True)
+            self._thread.start()
+
+    def stop(self):
+        self._stop.set()
+        if self._thread:
+            self._thread.join()
+        if self._smi:
+            self._smi.terminate()
+            self._smi.wait()
+            try:
+                for ln in open(self._smi_path):
+                    f = [x.strip() for x in ln.split(",")]
+                    if len(f) >= 5 and f[1].isdigit():
+                        mask = int(f[4], 16) if f[4].startswith("0x") else 0
+                        self.samples.append((int(f[1]), int(f[2]), mask))
+            except OSError:
+                pass
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        mask = 0
+        for _, _, r in self.samples:
+            mask |= r
+        return {"sm_mhz": statistics.median(s[0] for s in self.samples),
+                "sm_max_mhz": max(s[1] for s in self.samples),
+                "reasons": [v for k, v in sorted(self.REASONS.items()) if mask & k],
+                "samples": len(self.samples)}
+
+
+# --- workload statistics (algorithmic bytes) ----------------------------------------
+def batch_stats(keys: np.ndarray, d: int) -> dict:
+    """Exact per-kernel algorithmic bytes of one step on this batch."""
+    _, counts = np.unique(keys, return_counts=True)
+    B, U = len(keys), len(counts)
+    long_ = counts > SEQ_SEGMENT_MAX
+    Bl, Ul = int(counts[long_].sum()), int(long_.sum())
+    Bs, Us = B - Bl, U - Ul
+    items = int(np.ceil(counts[long_] / CHUNK).sum())
+    row = 4 * d
+    return {
+        "B": B, "U": U, "Bs": Bs, "Us": Us, "Bl": Bl, "Ul": Ul, "items": items,
+        # Get: keys + output per lookup; index sector + row per distinct key
+        "get_gather": B * (8 + row) + U * (32 + row),
+        # reduce: gradient rows + sorted position per lookup; row and state read
+        # and written once plus the segment bounds and row id per distinct key
+        "reduce_short": Bs * (row + 4) + Us * (4 * row + 12),
+        "reduce_long": Bl * (row + 4) + Ul * (4 * row + 12) + items * 2 * row,
+        # whole step (the survey's accounting: keys twice, output + grads, index
+        # sector + Get row read + row/state RMW per distinct key)
+        "step": B * (16 + 2 * row) + U * (32 + 5 * row),
+    }
+
+
+def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
+    if kid == 1:
+        return stats["get_gather"]
+    if kid == 4:
+        return stats["reduce_short"]
+    if kid == 5:
+        return stats["reduce_long"]
+    if kid == 3:
+        return stats["B"] * 16.0  # per pass: (row id, position) read and written
+    if kid == 2:
+        return stats["B"] * 12.0 + stats["U"] * 32.0
+    if kid == 6:
+        return stats["B"] * 4.0 + stats["U"] * 4.0
+    return 0.0
+
+
+KERNEL_NAMES = {1: "k_get (probe + row gather)", 2: "k_probe", 3: "k_sort_scatter",
+                4: "k_reduce_short (segment sum + Adagrad)", 5: "k_reduce_long (chunked sum + Adagrad)",
+                6: "segments"}
+KERNEL_SOURCES = {1: "mlkv_index.cu", 2: "mlkv_index.cu", 3: "mlkv_sort.cu", 4: "mlkv_apply.cu",
+                  5: "mlkv_apply.cu", 6: "mlkv_sort.cu"}
+
+
+def traffic_for(kid: int):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current source of that kernel (source hash match), else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f).get(str(kid))
+    except (OSError, ValueError):
+        return None
+    if not rec:
+        return None
+    src = os.path.join(ROOT, "paper_2504_01506_gb300", "csrc", KERNEL_SOURCES[kid])
+    h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    return rec.get("bytes_per_launch") if rec.get("source_sha") == h else None
+
+
+# --- distributed plumbing (replicas) --------------------------------------------------
+def dist_setup(n_gpus: int):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+
+        backend = "nccl" if os.environ.get("MLKV_BENCH_BACKEND", "nccl") == "nccl" else "gloo"
+        dist.init_process_group(backend=backend)
+        return dist, rank, local, world
+    return None, 0, 0, 1
+
+
+def barrier(dist, torch):
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+
+
+def max_over_ranks(dist, torch, x: float) -> float:
+    if dist is None:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# --- the oracle arms -------------------------------------------------------------------
+def oracle_steps(cfg, steps: int, sample: int, warmup: int = 0):
+    """Times the oracle (one host thread) on `steps` Get + apply steps, each on
+    the first `sample` lookups of that step's batch.  Returns (lookups/s, seconds)."""
+    import oracle
+
+    ref = oracle.Table(cfg.dim, lr=cfg.lr, eps=cfg.eps, state_init=cfg.state_init, init_lo=cfg.init_lo,
+                       init_hi=cfg.init_hi, seed=cfg.seed, precision=32)
+    batches = [(cfg.batch_keys(s)[:sample], cfg.grads(s, sample)) for s in range(warmup + steps)]
+    for k, g in batches[:warmup]:
+        ref.get(k)
+        ref.apply_grad(k, g)
+    t0 = time.perf_counter()
+    for k, g in batches[warmup:]:
+        ref.get(k)
+        ref.apply_grad(k, g)
+    dt = time.perf_counter() - t0
+    ref.close()
+    return steps * sample / dt, dt
+
+
+def run_reference(args, cfg):
+    dist, rank, _, world = None, int(os.environ.get("RANK", "0")), 0, int(os.environ.get("WORLD_SIZE", "1"))
+    if rank != 0:
+        return 0
+    sample = max(1, cfg.batch // 8)
+    value, dt = oracle_steps(cfg, args.steps, sample, args.warmup)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic", "config": workload_config(cfg),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"first {sample} of {cfg.batch} lookups of each step (Get + apply)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(cfg) -> dict:
+    c = {"workload": f"{cfg.name}: {cfg.n_keys:,} rows x dim {cfg.dim} fp32 (+ Adagrad state) in HBM, "
+                     f"{cfg.batch:,} lookups/step",
+         "rows": cfg.n_keys, "dim": cfg.dim, "batch_lookups": cfg.batch, "lr": cfg.lr,
+         "l2": "inputs larger than L2 every step (gradients and Get output 4*dim B per lookup)"}
+    if isinstance(cfg, W.configs.DlrmConfig):
+        c.update({"tables": cfg.tables, "zipf_alpha": cfg.alpha})
+    return c
+
+
+# --- our arm ----------------------------------------------------------------------------
+def run_ours(args, cfg):
+    import torch
+
+    from paper_2504_01506_gb300 import EmbeddingStore, _lib
+
+    dist, rank, local, world = dist_setup(args.gpus)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    hbm_peak, peak_kind = peaks()
+
+    store = EmbeddingStore(dim=cfg.dim, capacity=cfg.n_keys, max_batch=cfg.batch, lr=cfg.lr, eps=cfg.eps,
+                           state_init=cfg.state_init, init_lo=cfg.init_lo, init_hi=cfg.init_hi,
+                           seed=cfg.seed, device=dev)
+    # preload every key of the table (untimed), in preload order
+    chunk = cfg.batch
+    for s in range(0, cfg.n_keys, chunk):
+        store.insert(torch.from_numpy(cfg.preload_keys(s, s + chunk)).to(dev))
+    assert store.sync() == 0, "preload failed"
+
+    pool = max(1, min(args.pool, args.steps + args.warmup))
+    keys_h = [cfg.batch_keys(s) for s in range(pool)]
+    keys_d = [torch.from_numpy(k).to(dev) for k in keys_h]
+    gen = torch.Generator(device=dev)
+    grads_d = []
+    for s in range(pool):
+        gen.manual_seed(cfg.seed * 1000 + s)
+        grads_d.append(torch.randn((cfg.batch, cfg.dim), generator=gen, device=dev) * cfg.grad_sigma)
+    out = torch.empty((cfg.batch, cfg.dim), dtype=torch.float32, device=dev)
+    stats = [batch_stats(k, cfg.dim) for k in keys_h]
+    passes = (int(cfg.n_keys).bit_length() + 7) // 8
+
+    def step(i):
+        j = i % pool
+        store.get(keys_d[j], out=out)
+        store.apply_grad(keys_d[j], grads_d[j])
+
+    # pick the dominant kernel: one step per kernel class, timed with events
+    kernel_ms = {}
+    for kid in (1, 2, 3, 4, 5, 6):
+        store.time_kernel(kid)
+        step(0)
+        ms, n = store.kernel_time()
+        kernel_ms[kid] = ms
+    store.time_kernel(0)
+    dominant = max(kernel_ms, key=kernel_ms.get)
+    for i in range(args.warmup):
+        step(i)
+    assert store.sync() == 0
+
+    stream = torch.cuda.current_stream(dev)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    store.time_kernel(dominant)
+    launches0 = store.launch_count()
+    barrier(dist, torch)
+    clocks.start()
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(args.warmup + i)
+    ev1.record(stream)
+    barrier(dist, torch)
+    clocks.stop()
+    launches = store.launch_count() - launches0
+    dom_ms, dom_n = store.kernel_time()
+    store.time_kernel(0)
+    assert store.sync() == 0, "device status set during the timed region"
+    elapsed_ms = ev0.elapsed_time(ev1)
+    elapsed_ms = max_over_ranks(dist, torch, elapsed_ms)
+    lookups = cfg.batch * args.steps * world
+    value = lookups / (elapsed_ms / 1e3)
+    step_bytes = np.mean([s["step"] for s in stats])
+    achieved_step = step_bytes * args.steps / (elapsed_ms / 1e3) / 1e9
+
+    # roofline of the dominant kernel over the timed region
+    steps_idx = [(args.warmup + i) % pool for i in range(args.steps)]
+    per_launch_bytes = np.mean([kernel_bytes(stats[j], dominant, passes) for j in steps_idx])
+    if dominant in (3, 6):  # several launches per step
+        per_launch_bytes = per_launch_bytes  # per launch of that kernel
+    avg_ms = dom_ms / max(dom_n, 1)
+    achieved = per_launch_bytes / (avg_ms / 1e3) / 1e9
+    roofline = {"bound": "hbm", "kernel": KERNEL_NAMES[dominant], "achieved": achieved, "peak": hbm_peak,
+                "unit": "GB/s", "frac": achieved / hbm_peak, "peak_kind": peak_kind,
+                "traffic": traffic_for(dominant), "bytes_per_launch": per_launch_bytes,
+                "avg_launch_ms": avg_ms, "launches": dom_n,
+                "share_of_step": dom_ms / elapsed_ms if elapsed_ms else None}
+
+    # end to end through the host-buffer calls (copies inside the timed region)
+    e2e = None
+    if not args.no_e2e:
+        e2e_pool = min(pool, 2)
+        hk = [torch.from_numpy(keys_h[j]).pin_memory() for j in range(e2e_pool)]
+        hg = [grads_d[j].cpu().pin_memory() for j in range(e2e_pool)]
+        hout = torch.empty((cfg.batch, cfg.dim), dtype=torch.float32).pin_memory()
+        e2e_steps = max(1, min(args.steps, 20))
+        for i in range(2):
+            store.get_host(hk[i % e2e_pool], hout)
+            store.apply_grad_host(hk[i % e2e_pool], hg[i % e2e_pool])
+        barrier(dist, torch)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(e2e_steps):
+            store.get_host(hk[i % e2e_pool], hout)
+            store.apply_grad_host(hk[i % e2e_pool], hg[i % e2e_pool])
+        e1.record(stream)
+        barrier(dist, torch)
+        e_ms = max_over_ranks(dist, torch, e0.elapsed_time(e1))
+        assert store.sync() == 0
+        h2d = cfg.batch * 8 * 2 + cfg.batch * cfg.dim * 4
+        d2h = cfg.batch * cfg.dim * 4
+        e2e = {"value": cfg.batch * e2e_steps * world / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+               "link_gbs": (h2d + d2h) * e2e_steps / (e_ms / 1e3) / 1e9}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        sample = max(1, cfg.batch // 8)
+        steps = max(1, args.cpu_steps)
+        v, dt = oracle_steps(cfg, steps, sample)
+        cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"{steps} steps x first {sample} of {cfg.batch} lookups (Get + apply), "
+                         f"{dt:.1f} s on one host thread"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": dict(workload_config(cfg), parallelism=f"replicas{world}", distinct_batches=pool),
+            "achieved_gbs": achieved_step, "hbm_frac_measured": achieved_step / hbm_peak,
+            "hbm_frac_nominal": achieved_step / NOMINAL_HBM_GBS,
+            "distinct_per_step": float(np.mean([s["U"] for s in stats])),
+            "roofline": roofline, "kernel_ms_one_step": {KERNEL_NAMES[k]: v for k, v in kernel_ms.items()},
+            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clocks.summary(),
+        }
+        print(json.dumps(line), flush=True)
+    store.close()
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="dlrm", choices=sorted(W.ALL))
+    ap.add_argument("--pool", type=int, default=8, help="distinct pre-generated batches, cycled")
+    ap.add_argument("--cpu-steps", type=int, default=6)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    cfg = W.ALL[args.config]()
+    if args.impl == "reference":
+        return run_reference(args, cfg)
+    return run_ours(args, cfg)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

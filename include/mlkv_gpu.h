@@ -1,0 +1,210 @@
+/*
+ * mlkv_gpu.h -- C ABI of the GB300 batched embedding key-value store.
+ *
+ * One table = an open-addressing hash index (64-bit key -> dense row id) plus
+ * fp32 rows and fp32 Adagrad state, all resident in HBM.  The calls follow the
+ * storage interface of MLKV (arXiv 2504.01506):
+ *   Section 3.1  Open(model_id, dim, staleness_bound), Get(keys) -> values,
+ *                Put(keys, values) (upsert), Lookahead(keys, dest);
+ *   Section 3.2  step 8 and Figure 2: the gradient update is a per-key
+ *                read-modify-write of the stored vectors (Put or Rmw of
+ *                values + emb_optimizer(gradients)).
+ * The optimizer is element-wise Adagrad, one step per distinct key on the sum
+ * of that key's gradients in the batch (the gradient of the embedding map E of
+ * Section 2.1):
+ *       G[r] += g*g ;  w[r] -= lr * g / (sqrt(G[r]) + eps)
+ *
+ * Conventions shared by every call
+ *   - Pointers named d_* are DEVICE pointers owned by the caller; pointers
+ *     named h_* are HOST pointers owned by the caller (pinned memory makes
+ *     the copies asynchronous; pageable memory works but the copy blocks).
+ *     Buffers must stay valid until the stream has executed the call.
+ *   - Keys are int64 reinterpreted as uint64.  The key -1 (all bits set) is
+ *     reserved for empty index slots: a kernel that meets it records
+ *     MLKV_ERR_INVALID and treats that lookup as absent (NaN output, no
+ *     update, never inserted).
+ *   - Row-major layouts: values, gradients and outputs are [n][dim] fp32.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *     default stream).  All calls of one table share its scratch memory, so
+ *     issue them on one stream, or order them with events.  A table may be
+ *     used from one host thread at a time.
+ *   - Errors a host check finds are returned at once and nothing is enqueued.
+ *     Errors a kernel finds (MLKV_ERR_FULL, MLKV_ERR_PROBE_LIMIT,
+ *     MLKV_ERR_NOT_FOUND, MLKV_ERR_INVALID for the reserved key) are sticky:
+ *     they are recorded in the table's status word, returned by mlkv_sync and
+ *     by later calls once the GPU has reached the failing call, and cleared by
+ *     mlkv_clear_status.
+ *   - n == 0 is a no-op that returns MLKV_OK (after the argument checks).
+ *   - No call allocates device memory except mlkv_open (the table, its index,
+ *     its scratch sized for max_batch) and the first *_host call (staging
+ *     sized for max_batch).  Every wait inside a kernel is bounded.
+ */
+#ifndef MLKV_GPU_H
+#define MLKV_GPU_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+#define MLKV_OK 0
+#define MLKV_ERR_INVALID 1     /* bad argument: null pointer, n < 0, n > max_batch, reserved key */
+#define MLKV_ERR_UNSUPPORTED 2 /* a configuration this build does not provide */
+#define MLKV_ERR_CUDA 3        /* a CUDA runtime call failed; mlkv_last_error has the text */
+#define MLKV_ERR_NOMEM 4       /* device or pinned allocation failed */
+#define MLKV_ERR_FULL 5        /* more distinct keys than `capacity` */
+#define MLKV_ERR_PROBE_LIMIT 6 /* an index probe exceeded the probe bound */
+#define MLKV_ERR_NOT_FOUND 7   /* absent key and insert_on_miss == 0 */
+
+/* Largest dimension the row kernels take (8 vectors per lane of a warp). */
+#define MLKV_MAX_DIM 1024  /* dim > 256 needs dim % 4 == 0 */
+
+/* Segments (runs of one key in a gradient batch) of at most this many
+ * occurrences are summed by one warp in occurrence order, so their Adagrad
+ * step is the same op sequence as a sequential fp32 statement of it.  Longer
+ * segments are summed in fixed chunks, combined in chunk order: deterministic
+ * run to run, not the sequential rounding. */
+#define MLKV_SEQ_SEGMENT_MAX 32
+
+/* Flags of mlkv_config.flags. */
+#define MLKV_IDENTITY_HASH 2u  /* index slot = key mod 2^k (tests of long probe chains only) */
+
+/* Longest probe sequence of the index; a longer one records MLKV_ERR_PROBE_LIMIT. */
+#define MLKV_PROBE_LIMIT 1024
+
+/*
+ * Open of MLKV Section 3.1: Open(model_id, dim, staleness_bound).  model_id
+ * maps to the returned handle; one handle per table.
+ */
+typedef struct mlkv_config {
+    int32_t dim;             /* embedding dimension d, 1..MLKV_MAX_DIM */
+    int32_t insert_on_miss;  /* 1: Get / apply_grad of an absent key insert it with the init row */
+    int64_t capacity;        /* maximum number of distinct keys (rows), >= 1, < 2^31 */
+    int64_t max_batch;       /* maximum n of one call, >= 1, < 2^31 */
+    float lr;                /* Adagrad learning rate */
+    float eps;               /* Adagrad epsilon, added to sqrt(G) */
+    float state_init;        /* Adagrad state of a new row */
+    float init_lo, init_hi;  /* a new row is drawn U[init_lo, init_hi) by the counter-based init */
+    uint64_t seed;           /* seed of the counter-based init */
+    int64_t staleness_bound; /* MLKV's consistency bound; 0 (bulk-synchronous) is the only one accepted */
+    int64_t hbm_cache_rows;  /* 0: the whole table is resident in HBM; > 0 is not accepted yet */
+    uint32_t flags;          /* 0 or MLKV_IDENTITY_HASH */
+    uint32_t reserved;       /* 0 */
+} mlkv_config;
+
+typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
+
+/* Row initialisation of a new key k, element j (any implementation reproduces it):
+ *   x = splitmix64(seed ^ splitmix64(k ^ (j * 0x9E3779B97F4A7C15)))
+ *   v = init_lo + ((x >> 40) * 2^-24) * (init_hi - init_lo)   (fp32, each op rounded)
+ * where splitmix64(z) is the output of a SplitMix64 generator (Steele, Lea &
+ * Flood 2014) whose state is z.  State starts at state_init. */
+
+/* Creates a table on the current CUDA device.  Allocates rows + state
+ * (capacity x 2 x dim fp32, rows padded to 32 bytes), the index (a power of
+ * two >= 2 x capacity slots of 16 bytes) and scratch for max_batch.
+ * Returns MLKV_ERR_INVALID (bad field), MLKV_ERR_UNSUPPORTED
+ * (staleness_bound != 0, hbm_cache_rows != 0), MLKV_ERR_NOMEM or
+ * MLKV_ERR_CUDA.  On success *out owns everything; free it with mlkv_close. */
+int mlkv_open(const mlkv_config* cfg, mlkv_table** out);
+
+/* Waits for the table's work, frees all its memory.  Null is a no-op. */
+int mlkv_close(mlkv_table* t);
+
+/* Get of MLKV Section 3.1: d_out[i][:] = row of d_keys[i] for i < n.
+ * Absent keys: inserted (init row, state_init; row ids handed out in
+ * first-occurrence order) when insert_on_miss, otherwise d_out[i][:] = NaN and
+ * MLKV_ERR_NOT_FOUND is recorded.  d_out is fp32 [n][dim], 16-byte aligned
+ * when dim % 4 == 0. */
+int mlkv_get(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_out, void* stream);
+
+/* Put of MLKV Section 3.1 (upsert): row of d_keys[i] = d_vals[i][:]; a new key
+ * is inserted with state_init; a present key keeps its state.  Duplicate keys:
+ * the last occurrence wins. */
+int mlkv_put(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_vals, void* stream);
+
+/* Inserts the absent keys among d_keys with the init row (preloading a key
+ * set); present keys are left alone.  Row ids follow first occurrence. */
+int mlkv_insert(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream);
+
+/* The Rmw of MLKV Section 3.2 step 8 with Adagrad: for every distinct key k of
+ * d_keys, g = sum of d_grads[i][:] over the i with d_keys[i] == k, then one
+ * Adagrad step on k's row and state.  d_grads is fp32 [n][dim].  Absent keys
+ * are inserted first when insert_on_miss, else skipped with
+ * MLKV_ERR_NOT_FOUND recorded. */
+int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_grads,
+                    void* stream);
+
+/* Lookahead of MLKV Section 3.1 / 3.3.2 with dest = the store's buffer.  A row
+ * already resident is not copied again (Section 3.3.2); with the whole table
+ * in HBM every row is resident, so the call checks its arguments and returns.
+ * (dest = the application's cache is a Get into a buffer ahead of use.) */
+int mlkv_lookahead(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream);
+
+/* Key -> row id (int64, -1 when absent); never inserts. */
+int mlkv_find(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_rows, void* stream);
+
+/* Copies row and state of each key to d_rows / d_state (fp32 [n][dim] each;
+ * either may be null); NaN for absent keys.  Never inserts. */
+int mlkv_export(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_rows, float* d_state,
+                void* stream);
+
+/* The dedup step of the gradient apply, exposed for checking: the distinct
+ * present keys of d_keys ordered by row id, with their occurrence counts.
+ * Absent keys are left out and never inserted.  d_unique_keys: int64 [n];
+ * d_counts: int32 [n]; *d_num_unique (device int64) = number of distinct
+ * present keys. */
+int mlkv_dedup(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_unique_keys,
+               int32_t* d_counts, int64_t* d_num_unique, void* stream);
+
+/* Host-buffer forms of Get and the gradient apply: the keys (and gradients)
+ * are copied host -> device into table-owned staging on `stream`, the device
+ * call runs, and Get's output is copied back to h_out.  The first call
+ * allocates the staging (max_batch keys + max_batch x dim floats).  The call
+ * returns once the work is enqueued; h_out is valid after the stream syncs. */
+int mlkv_get_host(mlkv_table* t, const int64_t* h_keys, int64_t n, float* h_out, void* stream);
+int mlkv_apply_grad_host(mlkv_table* t, const int64_t* h_keys, int64_t n, const float* h_grads,
+                         void* stream);
+
+/* Waits for the last stream the table was used on; returns the sticky device
+ * status (MLKV_OK when none) or MLKV_ERR_CUDA. */
+int mlkv_sync(mlkv_table* t);
+
+/* Clears the sticky device status (synchronises first). */
+int mlkv_clear_status(mlkv_table* t);
+
+/* Number of distinct keys stored (synchronises). -1 on a null table. */
+int64_t mlkv_size(mlkv_table* t);
+
+/* Number of kernels this table has launched since open (host counter). */
+int64_t mlkv_launch_count(mlkv_table* t);
+
+/* Per-kernel timing with CUDA events recorded on the launching stream around
+ * every launch of kernel `kernel_id` (MLKV_K_*); 0 turns it off.  Read it with
+ * mlkv_kernel_time, which synchronises and returns the summed milliseconds and
+ * the number of timed launches since the last reset. */
+#define MLKV_K_GET_GATHER 1
+#define MLKV_K_PROBE 2
+#define MLKV_K_SORT_SCATTER 3
+#define MLKV_K_REDUCE_SHORT 4
+#define MLKV_K_REDUCE_LONG 5
+#define MLKV_K_SEGMENTS 6
+int mlkv_time_kernel(mlkv_table* t, int32_t kernel_id);
+int mlkv_kernel_time(mlkv_table* t, double* total_ms, int64_t* launches);
+
+/* Distinct keys of the last gradient apply (synchronises). */
+int64_t mlkv_last_unique(mlkv_table* t);
+
+/* Text of the last error this handle saw (static storage of the handle). */
+const char* mlkv_last_error(mlkv_table* t);
+
+/* Text of a status code. */
+const char* mlkv_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MLKV_GPU_H */

@@ -1,0 +1,501 @@
+// Hash index kernels: probe / insert-on-miss, the fused Get (probe + row
+// gather), deterministic row-id hand-out for new keys, Put, find and export.
+//
+// Index: open addressing with linear probing over 16-byte slots (two per
+// 32-byte sector), at most half full.  A key is published by one 64-bit
+// compare-and-swap on an empty slot whose row field already reads
+// ROW_PENDING, so a reader never pairs a key with a stale row.
+//
+// New keys get dense row ids in first-occurrence order (the numbering the
+// Get / Put upsert of MLKV Section 3.1 leaves open): while probing, every
+// lookup of a new key lowers the slot's `aux` to its batch position with
+// atomicMin; the lookup whose position survives is the first occurrence; an
+// exclusive scan over first-occurrence flags gives each new key its rank, and
+// row = rows handed out so far + rank.
+#include "mlkv_internal.cuh"
+
+namespace mlkv {
+
+namespace {
+
+__device__ __forceinline__ ulonglong2 ld_slot_volatile(const Slot* s) {
+    ulonglong2 v;
+    asm volatile("ld.volatile.global.v2.u64 {%0, %1}, [%2];" : "=l"(v.x), "=l"(v.y) : "l"(s));
+    return v;
+}
+
+__device__ __forceinline__ uint32_t ld_u32_volatile(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.volatile.global.u32 %0, [%1];" : "=r"(v) : "l"(p));
+    return v;
+}
+
+// Probes `key`.  Returns its row, ROW_ABSENT, or (INSERT only) ROW_PENDING
+// with `slot_out` = the slot that now holds the key and the slot's aux
+// lowered to `pos`.
+template <bool INSERT>
+__device__ __forceinline__ uint32_t probe_key(const IndexArgs& ia, unsigned long long key,
+                                              uint32_t pos, uint32_t& slot_out) {
+    if (key == EMPTY_KEY) {
+        record_error(ia.err, MLKV_ERR_INVALID);
+        return ROW_ABSENT;
+    }
+    unsigned long long s = (ia.identity_hash ? key : hash_key(key)) & ia.mask;
+    for (int i = 0; i < PROBE_LIMIT; ++i) {
+        ulonglong2 v = INSERT ? ld_slot_volatile(ia.index + s)
+                              : __ldg(reinterpret_cast<const ulonglong2*>(ia.index + s));
+        if (v.x == key) {
+            uint32_t row = (uint32_t)v.y;
+            slot_out = (uint32_t)s;
+            if (row != ROW_PENDING || !INSERT) return row == ROW_PENDING ? ROW_ABSENT : row;
+            atomicMin(&ia.index[s].aux, pos);
+            return ROW_PENDING;
+        }
+        if (v.x == EMPTY_KEY) {
+            if (!INSERT) return ROW_ABSENT;
+            unsigned long long old = atomicCAS(&ia.index[s].key, EMPTY_KEY, key);
+            if (old == EMPTY_KEY || old == key) {
+                slot_out = (uint32_t)s;
+                uint32_t row = ld_u32_volatile(&ia.index[s].row);
+                if (row != ROW_PENDING) return row;
+                atomicMin(&ia.index[s].aux, pos);
+                return ROW_PENDING;
+            }
+            // another key took this slot first: keep probing
+        }
+        s = (s + 1) & ia.mask;
+    }
+    record_error(ia.err, MLKV_ERR_PROBE_LIMIT);
+    return ROW_ABSENT;
+}
+
+// Appends (pos, slot) to the miss list with one atomic per converged group of lanes.
+__device__ __forceinline__ void append_miss(CallCounters* cur, uint32_t* miss_pos,
+                                            uint32_t* miss_slot, uint32_t pos, uint32_t slot) {
+    const unsigned m = __activemask();
+    const int lane = threadIdx.x & 31;
+    const int leader = __ffs(m) - 1;
+    uint32_t base = 0;
+    if (lane == leader) base = atomicAdd(&cur->n_miss, (uint32_t)__popc(m));
+    base = __shfl_sync(m, base, leader);
+    const uint32_t i = base + __popc(m & lanemask_lt());
+    miss_pos[i] = pos;
+    miss_slot[i] = slot;
+}
+
+__device__ __forceinline__ void zero_counters(CallCounters* nxt) {
+    if (blockIdx.x == 0 && threadIdx.x < sizeof(CallCounters) / 4)
+        reinterpret_cast<uint32_t*>(nxt)[threadIdx.x] = 0u;
+}
+
+struct RowArgs {
+    float* slots;
+    int stride;
+    int dpad;
+    int d;
+    int NV;
+    int G;
+};
+
+RowArgs row_args(mlkv_table* t) {
+    return RowArgs{t->slots, t->geom.stride, t->geom.dpad, t->geom.d, t->geom.NV, t->geom.G};
+}
+
+IndexArgs index_args(mlkv_table* t) {
+    return IndexArgs{t->index, t->index_mask, (t->cfg.flags & MLKV_IDENTITY_HASH) ? 1u : 0u,
+                     ErrSink{&t->dstate->status, t->status_dev_alias}};
+}
+
+// ---------------------------------------------------------------------------
+// One thread per lookup: row_of_pos[p] (and the slot) for every position.
+template <bool INSERT>
+__global__ void __launch_bounds__(256) k_probe(IndexArgs ia, const int64_t* __restrict__ keys,
+                                               uint32_t n, uint32_t* __restrict__ row_of_pos,
+                                               uint32_t* __restrict__ slot_of_pos,
+                                               uint32_t* miss_pos, uint32_t* miss_slot,
+                                               CallCounters* cur, CallCounters* nxt,
+                                               int report_absent) {
+    zero_counters(nxt);
+    const uint32_t p = blockIdx.x * blockDim.x + threadIdx.x;
+    if (p >= n) return;
+    uint32_t slot = 0;
+    const uint32_t row = probe_key<INSERT>(ia, (unsigned long long)keys[p], p, slot);
+    if (!INSERT && report_absent && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
+    row_of_pos[p] = row;
+    if (slot_of_pos) slot_of_pos[p] = slot;
+    if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
+}
+
+// Group-cooperative copy of one row (or NaN) into dst.
+template <int V, int KV>
+__device__ __forceinline__ void copy_row(const float* __restrict__ src, float* __restrict__ dst,
+                                         int NV, int G, int glane, bool absent) {
+    using VT = typename Vec<V>::T;
+    const VT* s = reinterpret_cast<const VT*>(src);
+    VT* o = reinterpret_cast<VT*>(dst);
+#pragma unroll
+    for (int k = 0; k < KV; ++k) {
+        const int j = glane + G * k;
+        if (j < NV) __stcs(o + j, absent ? Vec<V>::nan() : __ldg(s + j));
+    }
+}
+
+// The fused Get: each warp probes 32 consecutive lookups (one per lane), then
+// its lane groups gather the 32 rows with vector loads, streaming the output.
+// Lookups of new keys are left to the miss path.
+template <int V, int KV, bool INSERT>
+__global__ void __launch_bounds__(256) k_get(IndexArgs ia, RowArgs ra,
+                                             const int64_t* __restrict__ keys, uint32_t n,
+                                             float* __restrict__ out, uint32_t* miss_pos,
+                                             uint32_t* miss_slot, CallCounters* cur,
+                                             CallCounters* nxt) {
+    using VT = typename Vec<V>::T;
+    zero_counters(nxt);
+    const int lane = threadIdx.x & 31;
+    const uint32_t base = (blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * 32u;
+    if (base >= n) return;  // warp-uniform
+    const uint32_t p = base + lane;
+    uint32_t row = ROW_PENDING;  // lanes past the end skip the gather
+    if (p < n) {
+        uint32_t slot = 0;
+        row = probe_key<INSERT>(ia, (unsigned long long)keys[p], p, slot);
+        if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
+        if (!INSERT && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
+    }
+    const int G = ra.G, R = 32 / G, glane = lane & (G - 1), gid = lane / G;
+    constexpr int UNR = 8 / KV;
+    for (int it0 = 0; it0 < G; it0 += UNR) {
+        VT v[UNR][KV];
+        uint32_t rr[UNR];
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+            const int q = (it0 + u) * R + gid;
+            const uint32_t r = __shfl_sync(0xffffffffu, row, q & 31);
+            rr[u] = (it0 + u < G) ? r : ROW_PENDING;
+            if (rr[u] < ROW_ABSENT) {
+                const VT* src = reinterpret_cast<const VT*>(ra.slots + (size_t)rr[u] * ra.stride);
+#pragma unroll
+                for (int k = 0; k < KV; ++k) {
+                    const int j = glane + G * k;
+                    if (j < ra.NV) v[u][k] = __ldg(src + j);
+                }
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+            if (rr[u] == ROW_PENDING) continue;
+            const int q = (it0 + u) * R + gid;
+            VT* dst = reinterpret_cast<VT*>(out + (size_t)(base + q) * ra.d);
+#pragma unroll
+            for (int k = 0; k < KV; ++k) {
+                const int j = glane + G * k;
+                if (j < ra.NV) __stcs(dst + j, rr[u] == ROW_ABSENT ? Vec<V>::nan() : v[u][k]);
+            }
+        }
+    }
+}
+
+// Miss path 1/3: flag the first occurrence of every new key.
+__global__ void k_miss_flag(const Slot* __restrict__ index, const uint32_t* __restrict__ miss_pos,
+                            const uint32_t* __restrict__ miss_slot, uint32_t* __restrict__ flag,
+                            const CallCounters* cur) {
+    const uint32_t m = cur->n_miss;
+    for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < m; i += gridDim.x * blockDim.x) {
+        const uint32_t p = miss_pos[i];
+        if (index[miss_slot[i]].aux == p) flag[p] = 1u;
+    }
+}
+
+// Miss path 2/3 (after the scan of the flags): hand out rows and write the
+// new rows (init row unless Put, state_init).
+template <int V, int KV>
+__global__ void __launch_bounds__(256) k_miss_assign(IndexArgs ia, RowArgs ra,
+                                                     const int64_t* __restrict__ keys,
+                                                     const uint32_t* __restrict__ miss_pos,
+                                                     const uint32_t* __restrict__ miss_slot,
+                                                     const uint32_t* __restrict__ rank,
+                                                     const CallCounters* cur, const DevState* ds,
+                                                     unsigned long long capacity, int init_row,
+                                                     unsigned long long seed, float lo, float span,
+                                                     float state_init) {
+    using VT = typename Vec<V>::T;
+    const uint32_t m = cur->n_miss;
+    const int G = ra.G, glane = threadIdx.x & (G - 1);
+    const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
+    const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
+    const unsigned long long next = ds->next_row;
+    for (uint32_t i = group; i < m; i += ngroups) {
+        const uint32_t p = miss_pos[i], s = miss_slot[i];
+        if (ia.index[s].aux != p) continue;
+        const unsigned long long r = next + rank[p];
+        if (r >= capacity) {
+            if (glane == 0) record_error(ia.err, MLKV_ERR_FULL);
+            continue;
+        }
+        const unsigned long long key = (unsigned long long)keys[p];
+        float* w = ra.slots + (size_t)r * ra.stride;
+        VT* wv = reinterpret_cast<VT*>(w);
+        VT* gv = reinterpret_cast<VT*>(w + ra.dpad);
+#pragma unroll
+        for (int k = 0; k < KV; ++k) {
+            const int j = glane + G * k;
+            if (j >= ra.NV) continue;
+            if (init_row) {
+                float e[V];
+#pragma unroll
+                for (int c = 0; c < V; ++c) e[c] = init_element(seed, key, (uint32_t)(j * V + c), lo, span);
+                wv[j] = Vec<V>::from(e);
+            }
+            gv[j] = Vec<V>::splat(state_init);
+        }
+        if (glane == 0) ia.index[s].row = (uint32_t)r;
+    }
+}
+
+// Miss path 3/3: every missed lookup reads its key's row id (gathering the
+// row for Get), clears its flag and the slot's aux; the row counter advances.
+template <int V, int KV>
+__global__ void __launch_bounds__(256) k_miss_finish(IndexArgs ia, RowArgs ra,
+                                                     const uint32_t* __restrict__ miss_pos,
+                                                     const uint32_t* __restrict__ miss_slot,
+                                                     uint32_t* __restrict__ row_of_pos,
+                                                     uint32_t* __restrict__ flag,
+                                                     float* __restrict__ out,
+                                                     const CallCounters* cur, DevState* ds,
+                                                     unsigned long long capacity) {
+    const uint32_t m = cur->n_miss;
+    if (blockIdx.x == 0 && threadIdx.x == 0 && m) {
+        const unsigned long long nr = ds->next_row + cur->n_new;
+        ds->next_row = nr < capacity ? nr : capacity;
+    }
+    const int G = ra.G, glane = threadIdx.x & (G - 1);
+    const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
+    const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
+    for (uint32_t i = group; i < m; i += ngroups) {
+        const uint32_t p = miss_pos[i], s = miss_slot[i];
+        const uint32_t r0 = ia.index[s].row;
+        const uint32_t r = r0 == ROW_PENDING ? ROW_ABSENT : r0;
+        if (glane == 0) {
+            if (row_of_pos) row_of_pos[p] = r;
+            flag[p] = 0u;
+            ia.index[s].aux = AUX_IDLE;
+        }
+        if (out)
+            copy_row<V, KV>(ra.slots + (size_t)(r == ROW_ABSENT ? 0 : r) * ra.stride,
+                            out + (size_t)p * ra.d, ra.NV, G, glane, r == ROW_ABSENT);
+    }
+}
+
+// Put 1/2: the last occurrence of each key wins: aux = min over its
+// occurrences of (0xFFFFFFFE - p).
+__global__ void k_put_mark(Slot* __restrict__ index, const uint32_t* __restrict__ row_of_pos,
+                           const uint32_t* __restrict__ slot_of_pos, uint32_t n) {
+    const uint32_t p = blockIdx.x * blockDim.x + threadIdx.x;
+    if (p >= n || row_of_pos[p] >= ROW_ABSENT) return;
+    atomicMin(&index[slot_of_pos[p]].aux, 0xFFFFFFFEu - p);
+}
+
+// Put 2/2: the winning occurrence writes the row and puts aux back to idle.
+template <int V, int KV>
+__global__ void __launch_bounds__(256) k_put_scatter(Slot* __restrict__ index, RowArgs ra,
+                                                     const uint32_t* __restrict__ row_of_pos,
+                                                     const uint32_t* __restrict__ slot_of_pos,
+                                                     const float* __restrict__ vals, uint32_t n) {
+    using VT = typename Vec<V>::T;
+    const int lane = threadIdx.x & 31, G = ra.G, R = 32 / G, glane = lane & (G - 1), gid = lane / G;
+    const uint32_t warp = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const uint32_t nwarps = gridDim.x * (blockDim.x >> 5);
+    for (uint32_t b = warp * R; b < n; b += nwarps * R) {  // warp-uniform
+        const uint32_t p = b + gid;
+        bool win = false;
+        uint32_t r = 0, s = 0;
+        if (p < n) {
+            r = row_of_pos[p];
+            s = slot_of_pos[p];
+            win = r < ROW_ABSENT && index[s].aux == 0xFFFFFFFEu - p;
+        }
+        __syncwarp();
+        if (win) {
+            const VT* src = reinterpret_cast<const VT*>(vals + (size_t)p * ra.d);
+            VT* dst = reinterpret_cast<VT*>(ra.slots + (size_t)r * ra.stride);
+#pragma unroll
+            for (int k = 0; k < KV; ++k) {
+                const int j = glane + G * k;
+                if (j < ra.NV) dst[j] = __ldg(src + j);
+            }
+            if (glane == 0) index[s].aux = AUX_IDLE;
+        }
+    }
+}
+
+__global__ void __launch_bounds__(256) k_find(IndexArgs ia, const int64_t* __restrict__ keys,
+                                              uint32_t n, int64_t* __restrict__ rows,
+                                              CallCounters* nxt) {
+    zero_counters(nxt);
+    const uint32_t p = blockIdx.x * blockDim.x + threadIdx.x;
+    if (p >= n) return;
+    uint32_t slot = 0;
+    const uint32_t r = probe_key<false>(ia, (unsigned long long)keys[p], p, slot);
+    rows[p] = r >= ROW_ABSENT ? -1 : (int64_t)r;
+}
+
+// Export: like Get without insertion, copying row and/or state.
+template <int V, int KV>
+__global__ void __launch_bounds__(256) k_export(IndexArgs ia, RowArgs ra,
+                                                const int64_t* __restrict__ keys, uint32_t n,
+                                                float* __restrict__ rows_out,
+                                                float* __restrict__ state_out, CallCounters* nxt) {
+    zero_counters(nxt);
+    const int lane = threadIdx.x & 31;
+    const uint32_t base = (blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * 32u;
+    if (base >= n) return;
+    const uint32_t p = base + lane;
+    uint32_t row = ROW_PENDING;
+    if (p < n) {
+        uint32_t slot = 0;
+        row = probe_key<false>(ia, (unsigned long long)keys[p], p, slot);
+    }
+    const int G = ra.G, R = 32 / G, glane = lane & (G - 1), gid = lane / G;
+    for (int it = 0; it < G; ++it) {
+        const int q = it * R + gid;
+        const uint32_t r = __shfl_sync(0xffffffffu, row, q);
+        if (r == ROW_PENDING) continue;
+        const float* src = ra.slots + (size_t)(r == ROW_ABSENT ? 0 : r) * ra.stride;
+        if (rows_out) copy_row<V, KV>(src, rows_out + (size_t)(base + q) * ra.d, ra.NV, G, glane, r == ROW_ABSENT);
+        if (state_out)
+            copy_row<V, KV>(src + ra.dpad, state_out + (size_t)(base + q) * ra.d, ra.NV, G, glane, r == ROW_ABSENT);
+    }
+}
+
+// Dispatch over (V, KV) for the row kernels.
+template <template <int, int> class F, typename... A>
+cudaError_t dispatch_row(const RowGeom& g, A&&... a) {
+    if (g.V == 4) {
+        switch (g.KV) {
+            case 1: return F<4, 1>::run(a...);
+            case 2: return F<4, 2>::run(a...);
+            case 4: return F<4, 4>::run(a...);
+            default: return F<4, 8>::run(a...);
+        }
+    }
+    switch (g.KV) {
+        case 1: return F<1, 1>::run(a...);
+        case 2: return F<1, 2>::run(a...);
+        case 4: return F<1, 4>::run(a...);
+        default: return F<1, 8>::run(a...);
+    }
+}
+
+inline unsigned grid_for(int64_t items, int per_block) {
+    return (unsigned)((items + per_block - 1) / per_block);
+}
+
+inline unsigned capped_grid(mlkv_table* t, int64_t items, int per_block, int per_sm) {
+    int64_t g = (items + per_block - 1) / per_block;
+    int64_t cap = (int64_t)t->num_sms * per_sm;
+    if (g > cap) g = cap;
+    return (unsigned)(g < 1 ? 1 : g);
+}
+
+template <int V, int KV>
+struct GetRun {
+    static cudaError_t run(mlkv_table* t, const int64_t* keys, int64_t n, float* out,
+                           cudaStream_t st, CallCounters* cur, CallCounters* nxt) {
+        const unsigned grid = grid_for(n, 256);  // 8 warps x 32 lookups per block
+        if (t->cfg.insert_on_miss)
+            MLKV_LAUNCH(t, MLKV_K_GET_GATHER, (k_get<V, KV, true>), grid, 256, 0, st, index_args(t),
+                        row_args(t), keys, (uint32_t)n, out, t->s.miss_pos, t->s.miss_slot, cur, nxt);
+        else
+            MLKV_LAUNCH(t, MLKV_K_GET_GATHER, (k_get<V, KV, false>), grid, 256, 0, st, index_args(t),
+                        row_args(t), keys, (uint32_t)n, out, t->s.miss_pos, t->s.miss_slot, cur, nxt);
+        return cudaGetLastError();
+    }
+};
+
+template <int V, int KV>
+struct MissRun {
+    static cudaError_t run(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode, float* out,
+                           cudaStream_t st, CallCounters* cur) {
+        const unsigned g = capped_grid(t, n * (int64_t)t->geom.G, 256, 8);
+        const float span = t->cfg.init_hi - t->cfg.init_lo;
+        MLKV_LAUNCH(t, 0, (k_miss_assign<V, KV>), g, 256, 0, st, index_args(t), row_args(t), keys,
+                    t->s.miss_pos, t->s.miss_slot, t->s.rank, cur, t->dstate,
+                    (unsigned long long)t->cfg.capacity, mode == MissMode::Put ? 0 : 1,
+                    (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init);
+        MLKV_LAUNCH(t, 0, (k_miss_finish<V, KV>), g, 256, 0, st, index_args(t), row_args(t),
+                    t->s.miss_pos, t->s.miss_slot, t->s.row_of_pos, t->s.first_flag,
+                    mode == MissMode::Get ? out : nullptr, cur, t->dstate,
+                    (unsigned long long)t->cfg.capacity);
+        return cudaGetLastError();
+    }
+};
+
+template <int V, int KV>
+struct PutRun {
+    static cudaError_t run(mlkv_table* t, const float* vals, int64_t n, cudaStream_t st) {
+        MLKV_LAUNCH(t, 0, k_put_mark, grid_for(n, 256), 256, 0, st, t->index, t->s.row_of_pos,
+                    t->s.slot_of_pos, (uint32_t)n);
+        const unsigned g = capped_grid(t, n * (int64_t)t->geom.G, 256, 8);
+        MLKV_LAUNCH(t, 0, (k_put_scatter<V, KV>), g, 256, 0, st, t->index, row_args(t),
+                    t->s.row_of_pos, t->s.slot_of_pos, vals, (uint32_t)n);
+        return cudaGetLastError();
+    }
+};
+
+template <int V, int KV>
+struct ExportRun {
+    static cudaError_t run(mlkv_table* t, const int64_t* keys, int64_t n, float* rows, float* state,
+                           cudaStream_t st, CallCounters* nxt) {
+        MLKV_LAUNCH(t, 0, (k_export<V, KV>), grid_for(n, 256), 256, 0, st, index_args(t),
+                    row_args(t), keys, (uint32_t)n, rows, state, nxt);
+        return cudaGetLastError();
+    }
+};
+
+}  // namespace
+
+cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool insert,
+                         bool want_slot, bool report_absent, cudaStream_t st, CallCounters* cur,
+                         CallCounters* nxt) {
+    uint32_t* slot_of_pos = want_slot ? t->s.slot_of_pos : nullptr;
+    if (insert)
+        MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<true>, grid_for(n, 256), 256, 0, st, index_args(t), keys,
+                    (uint32_t)n, t->s.row_of_pos, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0);
+    else
+        MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<false>, grid_for(n, 256), 256, 0, st, index_args(t), keys,
+                    (uint32_t)n, t->s.row_of_pos, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt,
+                    report_absent ? 1 : 0);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out, cudaStream_t st,
+                       CallCounters* cur, CallCounters* nxt) {
+    return dispatch_row<GetRun>(t->geom, t, keys, n, out, st, cur, nxt);
+}
+
+cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode,
+                                  float* out, cudaStream_t st, CallCounters* cur) {
+    MLKV_LAUNCH(t, 0, k_miss_flag, capped_grid(t, n, 256, 8), 256, 0, st, t->index, t->s.miss_pos,
+                t->s.miss_slot, t->s.first_flag, cur);
+    cudaError_t e = launch_exclusive_scan(t, t->s.first_flag, t->s.rank, n, &cur->n_new,
+                                          &cur->n_miss, st);
+    if (e != cudaSuccess) return e;
+    return dispatch_row<MissRun>(t->geom, t, keys, n, mode, out, st, cur);
+}
+
+cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, int64_t n, cudaStream_t st) {
+    return dispatch_row<PutRun>(t->geom, t, vals, n, st);
+}
+
+cudaError_t launch_find(mlkv_table* t, const int64_t* keys, int64_t n, int64_t* rows,
+                        cudaStream_t st, CallCounters* nxt) {
+    MLKV_LAUNCH(t, 0, k_find, grid_for(n, 256), 256, 0, st, index_args(t), keys, (uint32_t)n, rows, nxt);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_export(mlkv_table* t, const int64_t* keys, int64_t n, float* rows, float* state,
+                          cudaStream_t st, CallCounters* nxt) {
+    return dispatch_row<ExportRun>(t->geom, t, keys, n, rows, state, st, nxt);
+}
+
+}  // namespace mlkv

@@ -1,0 +1,264 @@
+// Internal declarations of the GB300 embedding key-value store: the table
+// object, its HBM layout, device helpers and the launchers each .cu exports.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/mlkv_gpu.h"
+
+namespace mlkv {
+
+// ---------------------------------------------------------------------------
+// Index slot: 16 bytes, two per 32-byte sector.  An empty slot holds the
+// reserved key ~0 with row = ROW_PENDING and aux = AUX_IDLE, so a key made
+// visible by a compare-and-swap is always paired with a pending row.
+struct __align__(16) Slot {
+    unsigned long long key;
+    uint32_t row;  // dense row id, or ROW_PENDING while the key is being inserted
+    uint32_t aux;  // insertion: first position of the key in the batch; Put: last position
+};
+
+constexpr unsigned long long EMPTY_KEY = ~0ull;
+constexpr uint32_t ROW_PENDING = 0xFFFFFFFFu;   // key present, row not handed out yet
+constexpr uint32_t ROW_ABSENT = 0xFFFFFFFEu;    // key absent (or rejected)
+constexpr uint32_t AUX_IDLE = 0xFFFFFFFFu;
+constexpr int PROBE_LIMIT = MLKV_PROBE_LIMIT;
+
+// Per-call counters.  Two copies: a call uses cc[p] and its first kernel
+// zeroes cc[p ^ 1] for the next call, so no memset is enqueued.
+struct CallCounters {
+    uint32_t n_miss;     // lookups whose key had no row yet
+    uint32_t n_new;      // distinct new keys (first occurrences)
+    uint32_t n_unique;   // distinct rows after the sort
+    uint32_t n_valid;    // lookups with a row
+    uint32_t n_long;     // segments longer than MLKV_SEQ_SEGMENT_MAX
+    uint32_t n_items;    // chunks of the long segments
+    uint32_t pad[2];
+};
+
+struct DevState {
+    unsigned long long next_row;  // rows handed out so far
+    uint32_t status;              // first device-detected error (MLKV_ERR_*), sticky
+    uint32_t last_unique;         // distinct rows of the last gradient apply
+    CallCounters cc[2];
+};
+
+// Row-kernel geometry: a row of d floats is NV vectors of V floats; a group of
+// G lanes (a power of two <= 32) owns one row, each lane KV vectors of it.
+struct RowGeom {
+    int d;        // dim
+    int V;        // 4 (float4) or 1
+    int NV;       // vectors per row
+    int G;        // lanes per row
+    int KV;       // vectors per lane, 1/2/4/8
+    int dpad;     // row and state stride inside a slot (floats, multiple of 8)
+    int stride;   // floats per slot (row + state) = 2 * dpad
+};
+
+// The table.  Device memory layout in HBM:
+//   slots   [capacity][2 * dpad] fp32: w[0..d) | pad | G[0..d) | pad  (32-byte aligned)
+//   index   [nslots] Slot, nslots = 2^k >= 2 * capacity
+//   scratch arena sized for max_batch (see Scratch)
+struct Scratch {
+    uint32_t* row_of_pos;   // [max_batch]
+    uint32_t* slot_of_pos;  // [max_batch] (Put)
+    uint32_t* miss_pos;     // [max_batch]
+    uint32_t* miss_slot;    // [max_batch]
+    uint32_t* first_flag;   // [max_batch], zero at rest
+    uint32_t* rank;         // [max_batch]
+    uint32_t* sk[2];        // sort keys (row ids), ping-pong [max_batch]
+    uint32_t* sv[2];        // sort values (positions), ping-pong [max_batch]
+    uint32_t* hist;         // [256 * sort tiles]
+    uint32_t* tile_sums;    // [scan tiles]
+    uint32_t* seg_start;    // [max_batch + 1]
+    uint32_t* long_seg;     // [max long segments]
+    uint32_t* long_base;    // [max long segments]
+    uint32_t* long_cnt;     // [max long segments]
+    uint32_t* item_seg;     // [max items]
+    float* partial;         // [max items][dpad]
+    int64_t max_long;
+    int64_t max_items;
+    int64_t hist_len;
+    int64_t tile_sums_len;
+};
+
+struct KernelTimer {
+    int kernel_id = 0;
+    int n_events = 0;
+    static constexpr int kMax = 8192;
+    cudaEvent_t* ev = nullptr;  // 2 * kMax events, created on first use
+};
+
+}  // namespace mlkv
+
+struct mlkv_table {
+    mlkv_config cfg;
+    int device;
+    int num_sms;
+    mlkv::RowGeom geom;
+    float* slots;
+    mlkv::Slot* index;
+    unsigned long long index_mask;
+    int sort_bits;               // bits of a row id incl. the absent sentinel
+    mlkv::DevState* dstate;      // device
+    uint32_t* status_host;       // mapped pinned word the kernels also write errors to
+    uint32_t* status_dev_alias;  // its device alias
+    mlkv::Scratch s;
+    void* arena;                 // one allocation holding Scratch
+    int64_t arena_bytes;
+    int64_t* stage_keys;         // *_host staging, lazily allocated
+    float* stage_vals;
+    cudaStream_t last_stream;
+    int parity;
+    int64_t launches;
+    mlkv::KernelTimer timer;
+    double timed_ms;
+    int64_t timed_launches;
+    char last_error[512];
+};
+
+namespace mlkv {
+
+// Everything a kernel needs to record an error.
+struct ErrSink {
+    uint32_t* dev;             // DevState::status
+    volatile uint32_t* host;   // mapped pinned mirror
+};
+
+__device__ __forceinline__ void record_error(const ErrSink& e, uint32_t code) {
+    if (atomicCAS(e.dev, 0u, code) == 0u && e.host) *e.host = code;
+}
+
+// MurmurHash3 fmix64 finaliser (Appleby): spreads structured keys such as
+// table_id * 2^32 + row over the index.
+__device__ __forceinline__ unsigned long long hash_key(unsigned long long k) {
+    k ^= k >> 33;
+    k *= 0xff51afd7ed558ccdull;
+    k ^= k >> 33;
+    k *= 0xc4ceb9fe1a85ec53ull;
+    k ^= k >> 33;
+    return k;
+}
+
+// SplitMix64 output function (Steele, Lea & Flood 2014) and the counter-based
+// row initialisation stated in mlkv_gpu.h.
+__device__ __forceinline__ unsigned long long splitmix64(unsigned long long z) {
+    z += 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ float init_element(unsigned long long seed, unsigned long long key,
+                                              uint32_t j, float lo, float span) {
+    unsigned long long x = splitmix64(seed ^ splitmix64(key ^ ((unsigned long long)j * 0x9E3779B97F4A7C15ull)));
+    float u = __fmul_rn((float)(uint32_t)(x >> 40), 5.9604644775390625e-8f);  // exact: 24-bit int * 2^-24
+    return __fadd_rn(lo, __fmul_rn(u, span));
+}
+
+// One Adagrad element, each operation rounded on its own (no contraction):
+//   G' = G + g*g ; w' = w - (lr*g) / (sqrt(G') + eps)
+__device__ __forceinline__ void adagrad_element(float& w, float& G, float g, float lr, float eps) {
+    float Gn = __fadd_rn(G, __fmul_rn(g, g));
+    float den = __fadd_rn(__fsqrt_rn(Gn), eps);
+    float u = __fdiv_rn(__fmul_rn(lr, g), den);
+    G = Gn;
+    w = __fsub_rn(w, u);
+}
+
+template <int V> struct Vec;
+template <> struct Vec<4> {
+    using T = float4;
+    static __device__ __forceinline__ T zero() { return make_float4(0.f, 0.f, 0.f, 0.f); }
+    static __device__ __forceinline__ T nan() {
+        float q = __int_as_float(0x7fc00000);
+        return make_float4(q, q, q, q);
+    }
+    static __device__ __forceinline__ void add(T& a, const T& b) {
+        a.x = __fadd_rn(a.x, b.x); a.y = __fadd_rn(a.y, b.y);
+        a.z = __fadd_rn(a.z, b.z); a.w = __fadd_rn(a.w, b.w);
+    }
+    static __device__ __forceinline__ void adagrad(T& w, T& G, const T& g, float lr, float eps) {
+        adagrad_element(w.x, G.x, g.x, lr, eps); adagrad_element(w.y, G.y, g.y, lr, eps);
+        adagrad_element(w.z, G.z, g.z, lr, eps); adagrad_element(w.w, G.w, g.w, lr, eps);
+    }
+    static __device__ __forceinline__ T splat(float v) { return make_float4(v, v, v, v); }
+    static __device__ __forceinline__ T from(const float* e) { return make_float4(e[0], e[1], e[2], e[3]); }
+};
+template <> struct Vec<1> {
+    using T = float;
+    static __device__ __forceinline__ T zero() { return 0.f; }
+    static __device__ __forceinline__ T nan() { return __int_as_float(0x7fc00000); }
+    static __device__ __forceinline__ void add(T& a, const T& b) { a = __fadd_rn(a, b); }
+    static __device__ __forceinline__ void adagrad(T& w, T& G, const T& g, float lr, float eps) {
+        adagrad_element(w, G, g, lr, eps);
+    }
+    static __device__ __forceinline__ T splat(float v) { return v; }
+    static __device__ __forceinline__ T from(const float* e) { return e[0]; }
+};
+
+__device__ __forceinline__ uint32_t lanemask_lt() {
+    uint32_t m;
+    asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+    return m;
+}
+
+// Parameters shared by the index kernels.
+struct IndexArgs {
+    Slot* index;
+    unsigned long long mask;
+    uint32_t identity_hash;
+    ErrSink err;
+};
+
+// ---------------------------------------------------------------------------
+// Host-side launchers (each returns cudaGetLastError() of its launches).
+enum class MissMode : int { Init = 0, Put = 1, Get = 2 };
+
+// mlkv_index.cu
+cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool insert,
+                         bool want_slot, bool report_absent, cudaStream_t st, CallCounters* cur,
+                         CallCounters* nxt);
+cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out, cudaStream_t st,
+                       CallCounters* cur, CallCounters* nxt);
+cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode,
+                                  float* out, cudaStream_t st, CallCounters* cur);
+cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, int64_t n, cudaStream_t st);
+cudaError_t launch_find(mlkv_table* t, const int64_t* keys, int64_t n, int64_t* rows,
+                        cudaStream_t st, CallCounters* nxt);
+cudaError_t launch_export(mlkv_table* t, const int64_t* keys, int64_t n, float* rows,
+                          float* state, cudaStream_t st, CallCounters* nxt);
+
+// mlkv_sort.cu
+cudaError_t launch_exclusive_scan(mlkv_table* t, const uint32_t* in, uint32_t* out, int64_t n,
+                                  uint32_t* total, const uint32_t* enable, cudaStream_t st);
+cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow,
+                             const uint32_t** spos);
+cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, int64_t n, cudaStream_t st,
+                            CallCounters* cur);
+cudaError_t launch_dedup_out(mlkv_table* t, const int64_t* keys, const uint32_t* spos, int64_t n,
+                             int64_t* uniq, int32_t* counts, int64_t* num, cudaStream_t st,
+                             CallCounters* cur);
+
+// mlkv_apply.cu
+int64_t long_items_bound(int64_t max_batch);  // chunk items of long segments, worst case
+cudaError_t launch_reduce_apply(mlkv_table* t, const float* grads, const uint32_t* srow,
+                                const uint32_t* spos, int64_t n, cudaStream_t st,
+                                CallCounters* cur);
+
+// mlkv_table.cu: launch bookkeeping and optional per-kernel timing.
+void timer_before(mlkv_table* t, int kernel_id, cudaStream_t st);
+void timer_after(mlkv_table* t, int kernel_id, cudaStream_t st);
+int persistent_blocks(mlkv_table* t, const void* kernel, int threads);
+
+}  // namespace mlkv
+
+// Launch helper: counts the launch and records timing events when asked.
+#define MLKV_LAUNCH(t, kid, kernel, grid, block, smem, stream, ...)        \
+    do {                                                                   \
+        mlkv::timer_before((t), (kid), (stream));                          \
+        kernel<<<(grid), (block), (smem), (stream)>>>(__VA_ARGS__);        \
+        mlkv::timer_after((t), (kid), (stream));                           \
+        (t)->launches++;                                                   \
+    } while (0)

@@ -1,0 +1,463 @@
+// C ABI of the store (declared in include/mlkv_gpu.h): argument checks, the
+// table's memory, the order of kernels of each call, status and timing.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <unordered_map>
+
+#include "mlkv_internal.cuh"
+
+using namespace mlkv;
+
+namespace {
+
+int set_error(mlkv_table* t, int code, const char* fmt, ...) {
+    if (t) {
+        va_list ap;
+        va_start(ap, fmt);
+        vsnprintf(t->last_error, sizeof(t->last_error), fmt, ap);
+        va_end(ap);
+    }
+    return code;
+}
+
+int cuda_error(mlkv_table* t, cudaError_t e, const char* where) {
+    return set_error(t, MLKV_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+#define CK(t, call)                                          \
+    do {                                                     \
+        cudaError_t e_ = (call);                             \
+        if (e_ != cudaSuccess) return cuda_error((t), e_, #call); \
+    } while (0)
+
+int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+int next_pow2_int(int x) {
+    int p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+
+// Row-kernel geometry for vector width V (4 needs dim % 4 == 0).
+bool make_geom(int d, int V, RowGeom& g) {
+    if (V == 4 && d % 4) return false;
+    g.d = d;
+    g.V = V;
+    g.NV = (d + V - 1) / V;
+    g.G = next_pow2_int(g.NV) < 32 ? next_pow2_int(g.NV) : 32;
+    g.KV = (g.NV + g.G - 1) / g.G;
+    if (g.KV > 8) return false;
+    g.KV = g.KV <= 1 ? 1 : g.KV <= 2 ? 2 : g.KV <= 4 ? 4 : 8;
+    g.dpad = (int)round_up(d, 8);
+    g.stride = 2 * g.dpad;
+    return true;
+}
+
+int bit_width_u64(uint64_t x) {
+    int b = 0;
+    while (x) {
+        ++b;
+        x >>= 1;
+    }
+    return b;
+}
+
+constexpr int kScanTile = 4096;
+
+int64_t tiles_of(int64_t n) { return (n + kScanTile - 1) / kScanTile; }
+
+struct CallScope {
+    CallCounters* cur;
+    CallCounters* nxt;
+};
+
+CallScope begin_call(mlkv_table* t, cudaStream_t st) {
+    const int p = t->parity;
+    t->parity ^= 1;
+    t->last_stream = st;
+    return CallScope{&t->dstate->cc[p], &t->dstate->cc[p ^ 1]};
+}
+
+// Common argument checks.  Returns MLKV_OK, an error, or -1 for "n == 0: done".
+int check_call(mlkv_table* t, const void* keys, int64_t n, const void* buf, bool need_buf) {
+    if (!t) return MLKV_ERR_INVALID;
+    if (n < 0 || n > t->cfg.max_batch)
+        return set_error(t, MLKV_ERR_INVALID, "n = %lld outside [0, max_batch = %lld]", (long long)n,
+                         (long long)t->cfg.max_batch);
+    if (n > 0 && (!keys || (need_buf && !buf))) return set_error(t, MLKV_ERR_INVALID, "null pointer");
+    const uint32_t sticky = *(volatile uint32_t*)t->status_host;
+    if (sticky)
+        return set_error(t, (int)sticky, "sticky device status %u (%s) from an earlier call", sticky,
+                         mlkv_status_string((int)sticky));
+    return n == 0 ? -1 : MLKV_OK;
+}
+
+// Chooses the float4 kernels when every row buffer of the call is 16-byte aligned.
+int choose_geom(mlkv_table* t, const void* a, const void* b) {
+    const bool al = ((uintptr_t)a % 16 == 0) && ((uintptr_t)b % 16 == 0);
+    RowGeom g;
+    if (al && make_geom(t->cfg.dim, 4, g)) {
+        t->geom = g;
+        return MLKV_OK;
+    }
+    if (make_geom(t->cfg.dim, 1, g)) {
+        t->geom = g;
+        return MLKV_OK;
+    }
+    return set_error(t, MLKV_ERR_INVALID, "dim %d needs 16-byte aligned row buffers", t->cfg.dim);
+}
+
+}  // namespace
+
+namespace mlkv {
+
+void timer_before(mlkv_table* t, int kid, cudaStream_t st) {
+    KernelTimer& tm = t->timer;
+    if (!kid || kid != tm.kernel_id || tm.n_events >= KernelTimer::kMax) return;
+    if (!tm.ev) {
+        tm.ev = new cudaEvent_t[2 * KernelTimer::kMax];
+        for (int i = 0; i < 2 * KernelTimer::kMax; ++i) cudaEventCreate(&tm.ev[i]);
+    }
+    cudaEventRecord(tm.ev[2 * tm.n_events], st);
+}
+
+void timer_after(mlkv_table* t, int kid, cudaStream_t st) {
+    KernelTimer& tm = t->timer;
+    if (!kid || kid != tm.kernel_id || tm.n_events >= KernelTimer::kMax || !tm.ev) return;
+    cudaEventRecord(tm.ev[2 * tm.n_events + 1], st);
+    tm.n_events++;
+}
+
+int persistent_blocks(mlkv_table* t, const void* kernel, int threads) {
+    static std::mutex mu;
+    static std::unordered_map<const void*, int> cache;
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = cache.find(kernel);
+    int per_sm;
+    if (it != cache.end()) {
+        per_sm = it->second;
+    } else {
+        per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, 0) != cudaSuccess ||
+            per_sm < 1)
+            per_sm = 1;
+        cache[kernel] = per_sm;
+    }
+    return per_sm * t->num_sms;
+}
+
+}  // namespace mlkv
+
+extern "C" {
+
+const char* mlkv_status_string(int s) {
+    switch (s) {
+        case MLKV_OK: return "ok";
+        case MLKV_ERR_INVALID: return "invalid argument";
+        case MLKV_ERR_UNSUPPORTED: return "unsupported configuration";
+        case MLKV_ERR_CUDA: return "CUDA error";
+        case MLKV_ERR_NOMEM: return "out of memory";
+        case MLKV_ERR_FULL: return "table full";
+        case MLKV_ERR_PROBE_LIMIT: return "probe limit exceeded";
+        case MLKV_ERR_NOT_FOUND: return "key not found";
+        default: return "unknown status";
+    }
+}
+
+int mlkv_close(mlkv_table* t) {
+    if (!t) return MLKV_OK;
+    cudaDeviceSynchronize();
+    if (t->timer.ev) {
+        for (int i = 0; i < 2 * KernelTimer::kMax; ++i) cudaEventDestroy(t->timer.ev[i]);
+        delete[] t->timer.ev;
+    }
+    cudaFree(t->slots);
+    cudaFree(t->index);
+    cudaFree(t->dstate);
+    cudaFree(t->arena);
+    cudaFree(t->stage_keys);
+    cudaFree(t->stage_vals);
+    if (t->status_host) cudaFreeHost(t->status_host);
+    delete t;
+    return MLKV_OK;
+}
+
+int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
+    if (!cfg || !out) return MLKV_ERR_INVALID;
+    *out = nullptr;
+    const mlkv_config c = *cfg;
+    if (c.dim < 1 || c.dim > MLKV_MAX_DIM || (c.dim > 256 && c.dim % 4)) return MLKV_ERR_INVALID;
+    if (c.capacity < 1 || c.capacity >= (1ll << 31) - 2) return MLKV_ERR_INVALID;
+    if (c.max_batch < 1 || c.max_batch >= (1ll << 31) - 2) return MLKV_ERR_INVALID;
+    if (c.reserved != 0 || (c.flags & ~MLKV_IDENTITY_HASH)) return MLKV_ERR_INVALID;
+    if (!(c.init_hi >= c.init_lo)) return MLKV_ERR_INVALID;
+    if (c.staleness_bound != 0 || c.hbm_cache_rows != 0) return MLKV_ERR_UNSUPPORTED;
+
+    mlkv_table* t = new (std::nothrow) mlkv_table();
+    if (!t) return MLKV_ERR_NOMEM;
+    std::memset(t, 0, sizeof(*t));
+    t->cfg = c;
+    auto fail = [&](int code) {
+        mlkv_close(t);
+        return code;
+    };
+    if (cudaGetDevice(&t->device) != cudaSuccess) return fail(MLKV_ERR_CUDA);
+    if (cudaDeviceGetAttribute(&t->num_sms, cudaDevAttrMultiProcessorCount, t->device) != cudaSuccess)
+        return fail(MLKV_ERR_CUDA);
+    if (!make_geom(c.dim, c.dim % 4 == 0 ? 4 : 1, t->geom)) return fail(MLKV_ERR_INVALID);
+
+    const int64_t stride = t->geom.stride;
+    if (cudaMalloc(&t->slots, (size_t)c.capacity * stride * sizeof(float)) != cudaSuccess)
+        return fail(MLKV_ERR_NOMEM);
+    int64_t nslots = 64;
+    while (nslots < 2 * c.capacity) nslots <<= 1;
+    if (cudaMalloc(&t->index, (size_t)nslots * sizeof(Slot)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
+    if (cudaMemset(t->index, 0xFF, (size_t)nslots * sizeof(Slot)) != cudaSuccess) return fail(MLKV_ERR_CUDA);
+    t->index_mask = (unsigned long long)(nslots - 1);
+    t->sort_bits = bit_width_u64((uint64_t)c.capacity);
+
+    if (cudaMalloc(&t->dstate, sizeof(DevState)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
+    if (cudaMemset(t->dstate, 0, sizeof(DevState)) != cudaSuccess) return fail(MLKV_ERR_CUDA);
+    if (cudaHostAlloc(&t->status_host, sizeof(uint32_t), cudaHostAllocMapped) != cudaSuccess)
+        return fail(MLKV_ERR_NOMEM);
+    *t->status_host = 0;
+    if (cudaHostGetDevicePointer((void**)&t->status_dev_alias, t->status_host, 0) != cudaSuccess)
+        return fail(MLKV_ERR_CUDA);
+
+    // Scratch arena, carved in 256-byte aligned pieces.
+    const int64_t B = c.max_batch;
+    Scratch& s = t->s;
+    s.max_long = B / (MLKV_SEQ_SEGMENT_MAX + 1) + 1;
+    s.max_items = long_items_bound(B);
+    s.hist_len = 256 * tiles_of(B);
+    s.tile_sums_len = (tiles_of(B) > tiles_of(s.hist_len) ? tiles_of(B) : tiles_of(s.hist_len)) + 1;
+    struct Piece {
+        void** ptr;
+        int64_t bytes;
+    };
+    Piece pieces[] = {
+        {(void**)&s.row_of_pos, B * 4},     {(void**)&s.slot_of_pos, B * 4},
+        {(void**)&s.miss_pos, B * 4},       {(void**)&s.miss_slot, B * 4},
+        {(void**)&s.first_flag, B * 4},     {(void**)&s.rank, B * 4},
+        {(void**)&s.sk[0], B * 4},          {(void**)&s.sk[1], B * 4},
+        {(void**)&s.sv[0], B * 4},          {(void**)&s.sv[1], B * 4},
+        {(void**)&s.hist, s.hist_len * 4},  {(void**)&s.tile_sums, s.tile_sums_len * 4},
+        {(void**)&s.seg_start, (B + 1) * 4}, {(void**)&s.long_seg, s.max_long * 4},
+        {(void**)&s.long_base, s.max_long * 4}, {(void**)&s.long_cnt, s.max_long * 4},
+        {(void**)&s.item_seg, s.max_items * 4},
+        {(void**)&s.partial, s.max_items * t->geom.dpad * 4},
+    };
+    int64_t total = 0;
+    for (auto& p : pieces) total += round_up(p.bytes, 256);
+    if (cudaMalloc(&t->arena, (size_t)total) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
+    if (cudaMemset(t->arena, 0, (size_t)total) != cudaSuccess) return fail(MLKV_ERR_CUDA);
+    t->arena_bytes = total;
+    char* base = (char*)t->arena;
+    for (auto& p : pieces) {
+        *p.ptr = base;
+        base += round_up(p.bytes, 256);
+    }
+    if (cudaDeviceSynchronize() != cudaSuccess) return fail(MLKV_ERR_CUDA);
+    *out = t;
+    return MLKV_OK;
+}
+
+int mlkv_get(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_out, void* stream) {
+    int rc = check_call(t, d_keys, n, d_out, true);
+    if (rc) return rc < 0 ? MLKV_OK : rc;
+    if ((rc = choose_geom(t, d_out, d_out))) return rc;
+    cudaStream_t st = (cudaStream_t)stream;
+    CallScope cs = begin_call(t, st);
+    CK(t, launch_get(t, d_keys, n, d_out, st, cs.cur, cs.nxt));
+    if (t->cfg.insert_on_miss) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Get, d_out, st, cs.cur));
+    return MLKV_OK;
+}
+
+int mlkv_insert(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream) {
+    int rc = check_call(t, d_keys, n, nullptr, false);
+    if (rc) return rc < 0 ? MLKV_OK : rc;
+    if ((rc = choose_geom(t, t->slots, t->slots))) return rc;
+    cudaStream_t st = (cudaStream_t)stream;
+    CallScope cs = begin_call(t, st);
+    CK(t, launch_probe(t, d_keys, n, true, false, false, st, cs.cur, cs.nxt));
+    CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
+    return MLKV_OK;
+}
+
+int mlkv_put(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_vals, void* stream) {
+    int rc = check_call(t, d_keys, n, d_vals, true);
+    if (rc) return rc < 0 ? MLKV_OK : rc;
+    if ((rc = choose_geom(t, d_vals, d_vals))) return rc;
+    cudaStream_t st = (cudaStream_t)stream;
+    CallScope cs = begin_call(t, st);
+    CK(t, launch_probe(t, d_keys, n, true, true, false, st, cs.cur, cs.nxt));
+    CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Put, nullptr, st, cs.cur));
+    CK(t, launch_put_scatter(t, d_vals, n, st));
+    return MLKV_OK;
+}
+
+int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_grads, void* stream) {
+    int rc = check_call(t, d_keys, n, d_grads, true);
+    if (rc) return rc < 0 ? MLKV_OK : rc;
+    if ((rc = choose_geom(t, d_grads, d_grads))) return rc;
+    cudaStream_t st = (cudaStream_t)stream;
+    CallScope cs = begin_call(t, st);
+    const bool ins = t->cfg.insert_on_miss != 0;
+    CK(t, launch_probe(t, d_keys, n, ins, false, !ins, st, cs.cur, cs.nxt));
+    if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
+    const uint32_t *srow, *spos;
+    CK(t, launch_sort_rows(t, n, st, &srow, &spos));
+    CK(t, launch_segments(t, srow, n, st, cs.cur));
+    CK(t, launch_reduce_apply(t, d_grads, srow, spos, n, st, cs.cur));
+    return MLKV_OK;
+}
+
+int mlkv_lookahead(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream) {
+    (void)stream;
+    int rc = check_call(t, d_keys, n, nullptr, false);
+    return rc < 0 ? MLKV_OK : rc;
+}
+
+int mlkv_find(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_rows, void* stream) {
+    int rc = check_call(t, d_keys, n, d_rows, true);
+    if (rc) return rc < 0 ? MLKV_OK : rc;
+    cudaStream_t st = (cudaStream_t)stream;
+    CallScope cs = begin_call(t, st);
+    CK(t, launch_find(t, d_keys, n, d_rows, st, cs.nxt));
+    return MLKV_OK;
+}
+
+int mlkv_export(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_rows, float* d_state,
+                void* stream) {
+    int rc = check_call(t, d_keys, n, d_rows ? (void*)d_rows : (void*)d_state, true);
+    if (rc) return rc < 0 ? MLKV_OK : rc;
+    if ((rc = choose_geom(t, d_rows ? d_rows : d_state, d_state ? d_state : d_rows))) return rc;
+    cudaStream_t st = (cudaStream_t)stream;
+    CallScope cs = begin_call(t, st);
+    CK(t, launch_export(t, d_keys, n, d_rows, d_state, st, cs.nxt));
+    return MLKV_OK;
+}
+
+int mlkv_dedup(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_unique_keys,
+               int32_t* d_counts, int64_t* d_num_unique, void* stream) {
+    if (t && n == 0) {  // nothing to sort: report zero distinct keys
+        int rc = check_call(t, d_keys, n, nullptr, false);
+        if (rc > 0) return rc;
+        if (d_num_unique)
+            CK(t, cudaMemsetAsync(d_num_unique, 0, sizeof(int64_t), (cudaStream_t)stream));
+        return MLKV_OK;
+    }
+    int rc = check_call(t, d_keys, n, d_unique_keys, true);
+    if (rc) return rc < 0 ? MLKV_OK : rc;
+    if (!d_counts || !d_num_unique) return set_error(t, MLKV_ERR_INVALID, "null pointer");
+    cudaStream_t st = (cudaStream_t)stream;
+    CallScope cs = begin_call(t, st);
+    CK(t, launch_probe(t, d_keys, n, false, false, false, st, cs.cur, cs.nxt));
+    const uint32_t *srow, *spos;
+    CK(t, launch_sort_rows(t, n, st, &srow, &spos));
+    CK(t, launch_segments(t, srow, n, st, cs.cur));
+    CK(t, launch_dedup_out(t, d_keys, spos, n, d_unique_keys, d_counts, d_num_unique, st, cs.cur));
+    return MLKV_OK;
+}
+
+static int ensure_staging(mlkv_table* t) {
+    if (t->stage_keys) return MLKV_OK;
+    const size_t kb = (size_t)t->cfg.max_batch * sizeof(int64_t);
+    const size_t vb = (size_t)t->cfg.max_batch * t->cfg.dim * sizeof(float);
+    if (cudaMalloc(&t->stage_keys, kb) != cudaSuccess) return set_error(t, MLKV_ERR_NOMEM, "staging keys");
+    if (cudaMalloc(&t->stage_vals, vb) != cudaSuccess) {
+        cudaFree(t->stage_keys);
+        t->stage_keys = nullptr;
+        return set_error(t, MLKV_ERR_NOMEM, "staging values");
+    }
+    return MLKV_OK;
+}
+
+int mlkv_get_host(mlkv_table* t, const int64_t* h_keys, int64_t n, float* h_out, void* stream) {
+    int rc = check_call(t, h_keys, n, h_out, true);
+    if (rc) return rc < 0 ? MLKV_OK : rc;
+    if ((rc = ensure_staging(t))) return rc;
+    cudaStream_t st = (cudaStream_t)stream;
+    CK(t, cudaMemcpyAsync(t->stage_keys, h_keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
+    if ((rc = mlkv_get(t, t->stage_keys, n, t->stage_vals, stream))) return rc;
+    CK(t, cudaMemcpyAsync(h_out, t->stage_vals, (size_t)n * t->cfg.dim * 4, cudaMemcpyDeviceToHost, st));
+    return MLKV_OK;
+}
+
+int mlkv_apply_grad_host(mlkv_table* t, const int64_t* h_keys, int64_t n, const float* h_grads,
+                         void* stream) {
+    int rc = check_call(t, h_keys, n, h_grads, true);
+    if (rc) return rc < 0 ? MLKV_OK : rc;
+    if ((rc = ensure_staging(t))) return rc;
+    cudaStream_t st = (cudaStream_t)stream;
+    CK(t, cudaMemcpyAsync(t->stage_keys, h_keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
+    CK(t, cudaMemcpyAsync(t->stage_vals, h_grads, (size_t)n * t->cfg.dim * 4, cudaMemcpyHostToDevice, st));
+    return mlkv_apply_grad(t, t->stage_keys, n, t->stage_vals, stream);
+}
+
+int mlkv_sync(mlkv_table* t) {
+    if (!t) return MLKV_ERR_INVALID;
+    CK(t, cudaStreamSynchronize(t->last_stream));
+    uint32_t st = 0;
+    CK(t, cudaMemcpy(&st, &t->dstate->status, sizeof(st), cudaMemcpyDeviceToHost));
+    if (st) set_error(t, (int)st, "device status %u (%s)", st, mlkv_status_string((int)st));
+    return (int)st;
+}
+
+int mlkv_clear_status(mlkv_table* t) {
+    if (!t) return MLKV_ERR_INVALID;
+    CK(t, cudaDeviceSynchronize());
+    CK(t, cudaMemset(&t->dstate->status, 0, sizeof(uint32_t)));
+    CK(t, cudaDeviceSynchronize());
+    *(volatile uint32_t*)t->status_host = 0;
+    t->last_error[0] = 0;
+    return MLKV_OK;
+}
+
+int64_t mlkv_size(mlkv_table* t) {
+    if (!t) return -1;
+    if (cudaStreamSynchronize(t->last_stream) != cudaSuccess) return -1;
+    unsigned long long nr = 0;
+    if (cudaMemcpy(&nr, &t->dstate->next_row, sizeof(nr), cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
+    return (int64_t)nr;
+}
+
+int64_t mlkv_last_unique(mlkv_table* t) {
+    if (!t) return -1;
+    if (cudaStreamSynchronize(t->last_stream) != cudaSuccess) return -1;
+    uint32_t u = 0;
+    if (cudaMemcpy(&u, &t->dstate->last_unique, sizeof(u), cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
+    return (int64_t)u;
+}
+
+int64_t mlkv_launch_count(mlkv_table* t) { return t ? t->launches : -1; }
+
+int mlkv_time_kernel(mlkv_table* t, int32_t kernel_id) {
+    if (!t) return MLKV_ERR_INVALID;
+    t->timer.kernel_id = kernel_id;
+    t->timer.n_events = 0;
+    return MLKV_OK;
+}
+
+int mlkv_kernel_time(mlkv_table* t, double* total_ms, int64_t* launches) {
+    if (!t || !total_ms || !launches) return MLKV_ERR_INVALID;
+    double sum = 0;
+    const int n = t->timer.n_events;
+    for (int i = 0; i < n; ++i) {
+        CK(t, cudaEventSynchronize(t->timer.ev[2 * i + 1]));
+        float ms = 0;
+        CK(t, cudaEventElapsedTime(&ms, t->timer.ev[2 * i], t->timer.ev[2 * i + 1]));
+        sum += ms;
+    }
+    *total_ms = sum;
+    *launches = n;
+    t->timer.n_events = 0;
+    return MLKV_OK;
+}
+
+const char* mlkv_last_error(mlkv_table* t) { return t ? t->last_error : "null table"; }
+
+}  // extern "C"

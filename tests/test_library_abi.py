@@ -1,0 +1,77 @@
+"""The C-ABI library builds, loads without a GPU, and exports what the header declares."""
+import ctypes
+import os
+import re
+import shutil
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "mlkv_gpu.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(mlkv_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not shutil.which("nvcc") and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("nvcc not available")
+    from paper_2504_01506_gb300 import build
+
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def test_header_declares_the_interface():
+    names = declared_functions()
+    for must in ("mlkv_open", "mlkv_close", "mlkv_get", "mlkv_put", "mlkv_apply_grad", "mlkv_lookahead",
+                 "mlkv_insert", "mlkv_find", "mlkv_export", "mlkv_dedup", "mlkv_sync"):
+        assert must in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_binding_lists_every_symbol():
+    from paper_2504_01506_gb300 import _lib
+
+    assert sorted(_lib.EXPORTED) == declared_functions()
+
+
+def test_config_layout_matches_header(tmp_path):
+    """The ctypes Config mirrors struct mlkv_config field by field."""
+    from paper_2504_01506_gb300._lib import Config
+
+    fields = [f for f, _ in Config._fields_]
+    prog = tmp_path / "layout.c"
+    body = "".join(f'printf("{f} %zu\\n", offsetof(mlkv_config, {f}));' for f in fields)
+    prog.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "mlkv_gpu.h"\n'
+                    f'int main(void){{printf("size %zu\\n", sizeof(mlkv_config));{body}return 0;}}\n')
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", os.path.dirname(HEADER), str(prog), "-o", str(exe)], check=True)
+    out = dict(ln.split() for ln in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                   check=True).stdout.splitlines())
+    assert int(out["size"]) == ctypes.sizeof(Config)
+    for f in fields:
+        assert int(out[f]) == getattr(Config, f).offset, f
+
+
+def test_status_strings_without_gpu(lib):
+    lib.mlkv_status_string.restype = ctypes.c_char_p
+    assert lib.mlkv_status_string(5) == b"table full"
+    assert lib.mlkv_status_string(0) == b"ok"
+
+
+def test_null_and_bad_arguments_without_gpu(lib):
+    """Host-side checks return at once, before any CUDA call."""
+    lib.mlkv_get.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]
+    assert lib.mlkv_get(None, None, 0, None, None) == 1
+    assert lib.mlkv_open(None, None) == 1
+    assert lib.mlkv_close(None) == 0
