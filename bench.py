@@ -330,11 +330,15 @@ def run_ours(args, cfg):
     launches0 = store.launch_count()
     barrier(dist, torch)
     clocks.start()
+    if args.profile:
+        torch.cuda.profiler.start()
     ev0.record(stream)
     for i in range(args.steps):
         step(args.warmup + i)
     ev1.record(stream)
     barrier(dist, torch)
+    if args.profile:
+        torch.cuda.profiler.stop()
     clocks.stop()
     launches = store.launch_count() - launches0
     dom_ms, dom_n = store.kernel_time()
@@ -426,10 +430,16 @@ def main():
     ap.add_argument("--cpu-steps", type=int, default=6)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile", action="store_true",
+                    help="bracket the timed region with cudaProfilerStart/Stop (ncu --profile-from-start off)")
+    ap.add_argument("--scale", type=int, default=1,
+                    help="divide the table's rows by this (same batch); for small profiling cases")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     cfg = W.ALL[args.config]()
+    if args.scale > 1:
+        cfg = W.scaled(cfg, args.scale, 1)
     if args.impl == "reference":
         return run_reference(args, cfg)
     return run_ours(args, cfg)

@@ -4,31 +4,9 @@ import pytest
 
 import oracle
 import workloads as W
-from gpu_helpers import TOL, assert_bits, assert_close, dev, host, make_pair, torch_cuda
+from gpu_helpers import assert_bits, assert_close, dev, host, make_pair, torch_cuda
 
 pytestmark = pytest.mark.gpu
-
-
-def _run_steps(cfg, store, ref, steps, check_get=True, bitexact_short=True):
-    """Per step: Get then gradient apply, on both sides; returns per-key max counts."""
-    max_count = {}
-    for step in range(steps):
-        keys = cfg.batch_keys(step)
-        grads = cfg.grads(step)
-        out = host(store.get(dev(keys)))
-        want, _, _ = ref.get(keys)
-        if check_get:
-            if step == 0:
-                assert_bits(out, want, f"Get step {step}")
-            else:
-                assert_close(out, want, f"Get step {step}")
-        store.apply_grad(dev(keys), dev(grads))
-        ref.apply_grad(keys, grads)
-        u, c = np.unique(keys, return_counts=True)
-        for k, n in zip(u.tolist(), c.tolist()):
-            max_count[k] = max(max_count.get(k, 0), n)
-    assert store.sync() == 0
-    return max_count
 
 
 def test_init_rows_bit_exact():
@@ -218,7 +196,9 @@ def test_insert_on_miss_rows_match_oracle():
 def test_long_segments():
     cfg = W.scaled(W.tiny(), 100, 1)
     cfg.dim = 128
-    store, ref = make_pair(cfg, capacity=8192, max_batch=150_000)
+    # a sequential fp32 sum of 10^5 gradients carries ~1e-5 relative rounding
+    # of its own, so the reference here is the fp64 evaluation of the oracle
+    store, ref = make_pair(cfg, capacity=8192, max_batch=150_000, precision=64)
     rng = np.random.default_rng(9)
     keys = np.concatenate([np.full(100_000, 77), np.full(5_000, 78), rng.integers(100, 5000, 20_000)])
     rng.shuffle(keys)
