@@ -159,6 +159,27 @@ int mlkv_export(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_rows, 
 int mlkv_dedup(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_unique_keys,
                int32_t* d_counts, int64_t* d_num_unique, void* stream);
 
+/* Dedup of a batch of raw keys that allocates nothing.  The paper has no
+ * counterpart; it is here for callers that may not allocate device memory at
+ * the moment they need it: code that issues work while a stream is being
+ * captured in global mode (where cudaMalloc is refused), or plugins of engines
+ * that own every device allocation.  It needs no table.
+ *   d_keys: int64 [n], n <= MLKV_STATIC_MAX_KEYS (larger n: MLKV_ERR_INVALID,
+ *   nothing enqueued).  Output: the distinct keys in ascending unsigned order
+ *   in d_unique_keys (int64 [n]), their occurrence counts in d_counts
+ *   (int32 [n]) and their number in *d_num_unique (device int64).  Every key
+ *   value is allowed, -1 included.
+ * Its working memory is one fixed array in the library's device image (about
+ * 1.3 MB, held by every GPU that loads the library until the process exits),
+ * so no call allocates.  The first call on a device looks up that array's
+ * device address (cudaGetSymbolAddress, with that device current); make that
+ * first call before any stream capture.  Every call shares the array: calls
+ * that overlap on the GPU (other streams, other host threads) race and give
+ * wrong results; order them.  Call with the device of `stream` current. */
+#define MLKV_STATIC_MAX_KEYS 65536
+int mlkv_dedup_keys_static(const int64_t* d_keys, int64_t n, int64_t* d_unique_keys,
+                           int32_t* d_counts, int64_t* d_num_unique, void* stream);
+
 /* Host-buffer forms of Get and the gradient apply: the keys (and gradients)
  * are copied host -> device into table-owned staging on `stream`, the device
  * call runs, and Get's output is copied back to h_out.  The first call

@@ -34,8 +34,9 @@ EXPORTED = [
     "mlkv_lookahead", "mlkv_find", "mlkv_export", "mlkv_dedup", "mlkv_get_host",
     "mlkv_apply_grad_host", "mlkv_sync", "mlkv_clear_status", "mlkv_size", "mlkv_launch_count",
     "mlkv_time_kernel", "mlkv_kernel_time", "mlkv_last_unique", "mlkv_last_error",
-    "mlkv_status_string",
+    "mlkv_status_string", "mlkv_dedup_keys_static",
 ]
+STATIC_MAX_KEYS = 65536
 
 
 class Config(ctypes.Structure):
@@ -79,6 +80,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.mlkv_find.argtypes = [vp, vp, i64, vp, vp]
     lib.mlkv_export.argtypes = [vp, vp, i64, vp, vp, vp]
     lib.mlkv_dedup.argtypes = [vp, vp, i64, vp, vp, vp, vp]
+    lib.mlkv_dedup_keys_static.argtypes = [vp, i64, vp, vp, vp, vp]
     lib.mlkv_get_host.argtypes = [vp, vp, i64, vp, vp]
     lib.mlkv_apply_grad_host.argtypes = [vp, vp, i64, vp, vp]
     lib.mlkv_sync.argtypes = [vp]
@@ -98,7 +100,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     for name in ("mlkv_open", "mlkv_close", "mlkv_get", "mlkv_put", "mlkv_insert", "mlkv_apply_grad",
                  "mlkv_lookahead", "mlkv_find", "mlkv_export", "mlkv_dedup", "mlkv_get_host",
                  "mlkv_apply_grad_host", "mlkv_sync", "mlkv_clear_status", "mlkv_time_kernel",
-                 "mlkv_kernel_time"):
+                 "mlkv_kernel_time", "mlkv_dedup_keys_static"):
         getattr(lib, name).restype = i32
     _lib = lib
     return lib
