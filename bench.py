@@ -149,7 +149,10 @@ def batch_stats(keys: np.ndarray, d: int) -> dict:
         # reduce: gradient rows + sorted position per lookup; row and state read
         # and written once plus the segment bounds and row id per distinct key
         "reduce_short": Bs * (row + 4) + Us * (4 * row + 12),
-        "reduce_long": Bl * (row + 4) + Ul * (4 * row + 12) + items * 2 * row,
+        # long runs: gradient rows + sorted positions, chunk sums written
+        "reduce_long": Bl * (row + 4) + items * row,
+        # chunk sums read, row and state read and written once per long run
+        "long_combine": items * row + Ul * 4 * row,
         # whole step (the survey's accounting: keys twice, output + grads, index
         # sector + Get row read + row/state RMW per distinct key)
         "step": B * (16 + 2 * row) + U * (32 + 5 * row),
@@ -163,6 +166,8 @@ def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
         return stats["reduce_short"]
     if kid == 5:
         return stats["reduce_long"]
+    if kid == 7:
+        return stats["long_combine"]
     if kid == 3:
         return stats["B"] * 16.0  # per pass: (row id, position) read and written
     if kid == 2:
@@ -173,10 +178,10 @@ def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
 
 
 KERNEL_NAMES = {1: "k_get (probe + row gather)", 2: "k_probe", 3: "k_sort_scatter",
-                4: "k_reduce_short (segment sum + Adagrad)", 5: "k_reduce_long (chunked sum + Adagrad)",
-                6: "segments"}
+                4: "k_short (run sum + Adagrad)", 5: "k_long_sum (chunk sums of long runs)",
+                6: "segments", 7: "k_long_combine (chunk sums + Adagrad)"}
 KERNEL_SOURCES = {1: "mlkv_index.cu", 2: "mlkv_index.cu", 3: "mlkv_sort.cu", 4: "mlkv_apply.cu",
-                  5: "mlkv_apply.cu", 6: "mlkv_sort.cu"}
+                  5: "mlkv_apply.cu", 6: "mlkv_sort.cu", 7: "mlkv_apply.cu"}
 
 
 def traffic_for(kid: int):
@@ -312,7 +317,7 @@ def run_ours(args, cfg):
 
     # pick the dominant kernel: one step per kernel class, timed with events
     kernel_ms = {}
-    for kid in (1, 2, 3, 4, 5, 6):
+    for kid in (1, 2, 3, 4, 5, 6, 7):
         store.time_kernel(kid)
         step(0)
         ms, n = store.kernel_time()

@@ -30,7 +30,8 @@
  *     used from one host thread at a time.
  *   - Errors a host check finds are returned at once and nothing is enqueued.
  *     Errors a kernel finds (MLKV_ERR_FULL, MLKV_ERR_PROBE_LIMIT,
- *     MLKV_ERR_NOT_FOUND, MLKV_ERR_INVALID for the reserved key) are sticky:
+ *     MLKV_ERR_NOT_FOUND, MLKV_ERR_TIMEOUT, MLKV_ERR_INVALID for the reserved
+ *     key) are sticky:
  *     they are recorded in the table's status word, returned by mlkv_sync and
  *     by later calls once the GPU has reached the failing call, and cleared by
  *     mlkv_clear_status.
@@ -57,15 +58,16 @@ extern "C" {
 #define MLKV_ERR_FULL 5        /* more distinct keys than `capacity` */
 #define MLKV_ERR_PROBE_LIMIT 6 /* an index probe exceeded the probe bound */
 #define MLKV_ERR_NOT_FOUND 7   /* absent key and insert_on_miss == 0 */
+#define MLKV_ERR_TIMEOUT 8     /* a bounded wait inside a kernel ran out (the batch is not applied in full) */
 
 /* Largest dimension the row kernels take (8 vectors per lane of a warp). */
 #define MLKV_MAX_DIM 1024  /* dim > 256 needs dim % 4 == 0 */
 
 /* Segments (runs of one key in a gradient batch) of at most this many
- * occurrences are summed by one warp in occurrence order, so their Adagrad
- * step is the same op sequence as a sequential fp32 statement of it.  Longer
- * segments are summed in fixed chunks, combined in chunk order: deterministic
- * run to run, not the sequential rounding. */
+ * occurrences are summed by one lane group in occurrence order, so their
+ * Adagrad step is the same op sequence as a sequential fp32 statement of it.
+ * Longer segments are summed in chunks of 64 lookups and the chunk sums added
+ * in a fixed order: deterministic run to run, not the sequential rounding. */
 #define MLKV_SEQ_SEGMENT_MAX 32
 
 /* Flags of mlkv_config.flags. */
@@ -212,10 +214,11 @@ int64_t mlkv_launch_count(mlkv_table* t);
 #define MLKV_K_REDUCE_SHORT 4
 #define MLKV_K_REDUCE_LONG 5
 #define MLKV_K_SEGMENTS 6
+#define MLKV_K_LONG_COMBINE 7
 int mlkv_time_kernel(mlkv_table* t, int32_t kernel_id);
 int mlkv_kernel_time(mlkv_table* t, double* total_ms, int64_t* launches);
 
-/* Distinct keys of the last gradient apply (synchronises). */
+/* Distinct keys of the last gradient apply or dedup (synchronises). */
 int64_t mlkv_last_unique(mlkv_table* t);
 
 /* Text of the last error this handle saw (static storage of the handle). */

@@ -18,6 +18,7 @@ ERR_NOMEM = 4
 ERR_FULL = 5
 ERR_PROBE_LIMIT = 6
 ERR_NOT_FOUND = 7
+ERR_TIMEOUT = 8
 SEQ_SEGMENT_MAX = 32
 PROBE_LIMIT = 1024
 IDENTITY_HASH = 2
@@ -28,6 +29,7 @@ K_SORT_SCATTER = 3
 K_REDUCE_SHORT = 4
 K_REDUCE_LONG = 5
 K_SEGMENTS = 6
+K_LONG_COMBINE = 7
 
 EXPORTED = [
     "mlkv_open", "mlkv_close", "mlkv_get", "mlkv_put", "mlkv_insert", "mlkv_apply_grad",

@@ -44,7 +44,11 @@ def up_to_date() -> bool:
 
 
 def build(force: bool = False, verbose: bool = False, extra=()) -> str:
-    if not force and up_to_date():
+    # MLKV_NVCC_FLAGS: extra nvcc flags, e.g. -D overrides of the kernels'
+    # tuning constants for a sweep; a build with them is always forced.
+    env_extra = os.environ.get("MLKV_NVCC_FLAGS", "").split()
+    extra = [*extra, *env_extra]
+    if not force and not env_extra and up_to_date():
         return LIB
     os.makedirs(BUILD, exist_ok=True)
     cc = nvcc()

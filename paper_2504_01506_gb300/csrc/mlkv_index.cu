@@ -143,8 +143,17 @@ __device__ __forceinline__ void copy_row(const float* __restrict__ src, float* _
 // The fused Get: each warp probes 32 consecutive lookups (one per lane), then
 // its lane groups gather the 32 rows with vector loads, streaming the output.
 // Lookups of new keys are left to the miss path.
+// Tuning (set at build time): minimum resident blocks per SM for the Get
+// kernel's register allocation, and rows each lane group has in flight.
+#ifndef MLKV_GET_MIN_BLOCKS
+#define MLKV_GET_MIN_BLOCKS 6
+#endif
+#ifndef MLKV_GET_ROWS_IN_FLIGHT
+#define MLKV_GET_ROWS_IN_FLIGHT 4
+#endif
+
 template <int V, int KV, bool INSERT>
-__global__ void __launch_bounds__(256) k_get(IndexArgs ia, RowArgs ra,
+__global__ void __launch_bounds__(256, MLKV_GET_MIN_BLOCKS) k_get(IndexArgs ia, RowArgs ra,
                                              const int64_t* __restrict__ keys, uint32_t n,
                                              float* __restrict__ out, uint32_t* miss_pos,
                                              uint32_t* miss_slot, CallCounters* cur,
@@ -163,7 +172,7 @@ __global__ void __launch_bounds__(256) k_get(IndexArgs ia, RowArgs ra,
         if (!INSERT && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
     }
     const int G = ra.G, R = 32 / G, glane = lane & (G - 1), gid = lane / G;
-    constexpr int UNR = 8 / KV;
+    constexpr int UNR = KV >= MLKV_GET_ROWS_IN_FLIGHT ? 1 : MLKV_GET_ROWS_IN_FLIGHT / KV;
     for (int it0 = 0; it0 < G; it0 += UNR) {
         VT v[UNR][KV];
         uint32_t rr[UNR];

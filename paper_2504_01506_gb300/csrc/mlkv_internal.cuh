@@ -32,8 +32,8 @@ struct CallCounters {
     uint32_t n_new;      // distinct new keys (first occurrences)
     uint32_t n_unique;   // distinct rows after the sort
     uint32_t n_valid;    // lookups with a row
-    uint32_t n_long;     // segments longer than MLKV_SEQ_SEGMENT_MAX
-    uint32_t n_items;    // chunks of the long segments
+    uint32_t n_long;     // runs longer than MLKV_SEQ_SEGMENT_MAX
+    uint32_t n_items;    // chunks of the long runs
     uint32_t pad[2];
 };
 
@@ -71,12 +71,13 @@ struct Scratch {
     uint32_t* sv[2];        // sort values (positions), ping-pong [max_batch]
     uint32_t* hist;         // [256 * sort tiles]
     uint32_t* tile_sums;    // [scan tiles]
-    uint32_t* seg_start;    // [max_batch + 1]
-    uint32_t* long_seg;     // [max long segments]
-    uint32_t* long_base;    // [max long segments]
-    uint32_t* long_cnt;     // [max long segments]
-    uint32_t* item_seg;     // [max items]
-    float* partial;         // [max items][dpad]
+    uint32_t* seg_start;    // [max_batch + 1] run starts in sorted order
+    uint32_t* long_s;       // [max_long] long runs: first sorted position
+    uint32_t* long_e;       // [max_long] one past the last
+    uint32_t* long_row;     // [max_long]
+    uint32_t* long_base;    // [max_long] first chunk item
+    uint32_t* item_run;     // [max_items] long run of each chunk
+    float* partial;         // [max_items][dpad] chunk sums
     int64_t max_long;
     int64_t max_items;
     int64_t hist_len;
@@ -185,6 +186,10 @@ template <> struct Vec<4> {
     }
     static __device__ __forceinline__ T splat(float v) { return make_float4(v, v, v, v); }
     static __device__ __forceinline__ T from(const float* e) { return make_float4(e[0], e[1], e[2], e[3]); }
+    static __device__ __forceinline__ T shfl_down(const T& v, int delta) {
+        return make_float4(__shfl_down_sync(0xffffffffu, v.x, delta), __shfl_down_sync(0xffffffffu, v.y, delta),
+                           __shfl_down_sync(0xffffffffu, v.z, delta), __shfl_down_sync(0xffffffffu, v.w, delta));
+    }
 };
 template <> struct Vec<1> {
     using T = float;
@@ -196,6 +201,9 @@ template <> struct Vec<1> {
     }
     static __device__ __forceinline__ T splat(float v) { return v; }
     static __device__ __forceinline__ T from(const float* e) { return e[0]; }
+    static __device__ __forceinline__ T shfl_down(const T& v, int delta) {
+        return __shfl_down_sync(0xffffffffu, v, delta);
+    }
 };
 
 __device__ __forceinline__ uint32_t lanemask_lt() {
@@ -242,7 +250,8 @@ cudaError_t launch_dedup_out(mlkv_table* t, const int64_t* keys, const uint32_t*
                              CallCounters* cur);
 
 // mlkv_apply.cu
-int64_t long_items_bound(int64_t max_batch);  // chunk items of long segments, worst case
+int64_t long_runs_bound(int64_t max_batch);   // runs longer than MLKV_SEQ_SEGMENT_MAX, worst case
+int64_t long_items_bound(int64_t max_batch);  // chunks of those runs, worst case
 cudaError_t launch_reduce_apply(mlkv_table* t, const float* grads, const uint32_t* srow,
                                 const uint32_t* spos, int64_t n, cudaStream_t st,
                                 CallCounters* cur);

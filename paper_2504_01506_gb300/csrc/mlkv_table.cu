@@ -163,6 +163,7 @@ const char* mlkv_status_string(int s) {
         case MLKV_ERR_FULL: return "table full";
         case MLKV_ERR_PROBE_LIMIT: return "probe limit exceeded";
         case MLKV_ERR_NOT_FOUND: return "key not found";
+        case MLKV_ERR_TIMEOUT: return "bounded wait in a kernel ran out";
         default: return "unknown status";
     }
 }
@@ -230,7 +231,7 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     // Scratch arena, carved in 256-byte aligned pieces.
     const int64_t B = c.max_batch;
     Scratch& s = t->s;
-    s.max_long = B / (MLKV_SEQ_SEGMENT_MAX + 1) + 1;
+    s.max_long = long_runs_bound(B);
     s.max_items = long_items_bound(B);
     s.hist_len = 256 * tiles_of(B);
     s.tile_sums_len = (tiles_of(B) > tiles_of(s.hist_len) ? tiles_of(B) : tiles_of(s.hist_len)) + 1;
@@ -245,9 +246,9 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
         {(void**)&s.sk[0], B * 4},          {(void**)&s.sk[1], B * 4},
         {(void**)&s.sv[0], B * 4},          {(void**)&s.sv[1], B * 4},
         {(void**)&s.hist, s.hist_len * 4},  {(void**)&s.tile_sums, s.tile_sums_len * 4},
-        {(void**)&s.seg_start, (B + 1) * 4}, {(void**)&s.long_seg, s.max_long * 4},
-        {(void**)&s.long_base, s.max_long * 4}, {(void**)&s.long_cnt, s.max_long * 4},
-        {(void**)&s.item_seg, s.max_items * 4},
+        {(void**)&s.seg_start, (B + 1) * 4},  {(void**)&s.long_s, s.max_long * 4},
+        {(void**)&s.long_e, s.max_long * 4},   {(void**)&s.long_row, s.max_long * 4},
+        {(void**)&s.long_base, s.max_long * 4}, {(void**)&s.item_run, s.max_items * 4},
         {(void**)&s.partial, s.max_items * t->geom.dpad * 4},
     };
     int64_t total = 0;
