@@ -84,7 +84,7 @@ typedef struct mlkv_config {
     int32_t dim;             /* embedding dimension d, 1..MLKV_MAX_DIM */
     int32_t insert_on_miss;  /* 1: Get / apply_grad of an absent key insert it with the init row */
     int64_t capacity;        /* maximum number of distinct keys (rows), >= 1, < 2^31 */
-    int64_t max_batch;       /* maximum n of one call, >= 1, < 2^31 */
+    int64_t max_batch;       /* maximum n of one call, >= 1, < 2^30 */
     float lr;                /* Adagrad learning rate */
     float eps;               /* Adagrad epsilon, added to sqrt(G) */
     float state_init;        /* Adagrad state of a new row */

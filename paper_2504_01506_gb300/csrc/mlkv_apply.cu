@@ -42,6 +42,12 @@ constexpr int kChunk = 64;
 #ifndef MLKV_SHORT_MIN_BLOCKS
 #define MLKV_SHORT_MIN_BLOCKS 5
 #endif
+#ifndef MLKV_LONG_ROWS_IN_FLIGHT
+#define MLKV_LONG_ROWS_IN_FLIGHT 4
+#endif
+#ifndef MLKV_LONG_MIN_BLOCKS
+#define MLKV_LONG_MIN_BLOCKS 5
+#endif
 
 struct RowArgs {
     float* slots;
@@ -57,12 +63,15 @@ struct RunArgs {
     const uint32_t* srow;
     const uint32_t* spos;
     const uint32_t* seg_start;
+    const uint32_t* run_row;   // row of each run
+    const uint32_t* run_p0;    // first lookup position of each run
     CallCounters* cur;
     uint32_t* long_s;      // [max_long] first sorted position
     uint32_t* long_e;      // [max_long] one past the last
     uint32_t* long_row;    // [max_long]
     uint32_t* long_base;   // [max_long] first chunk item
-    uint32_t* item_run;    // [max_items] long run of each chunk item
+    uint32_t* item_s;      // [max_items] first sorted position of each chunk
+    uint32_t* item_e;      // [max_items] one past its last
     float* partial;        // [max_items][dpad]
     uint32_t max_long;
     uint32_t max_items;
@@ -77,12 +86,12 @@ __device__ __forceinline__ unsigned group_mask(int G, int gid) {
 // acc += the gradient rows of sorted positions s .. s+len-1, in that order.
 // The group loads up to G positions at a time (one per lane) and hands them
 // round with group shuffles.
-template <int V, int KV>
+template <int V, int KV, int ROWS = MLKV_REDUCE_ROWS_IN_FLIGHT>
 __device__ __forceinline__ void sum_rows(typename Vec<V>::T (&acc)[KV], const float* __restrict__ grads,
                                          const uint32_t* __restrict__ spos, uint32_t s, uint32_t len, int d,
                                          int NV, int G, int glane, unsigned gmask) {
     using VT = typename Vec<V>::T;
-    constexpr int UNR = KV >= MLKV_REDUCE_ROWS_IN_FLIGHT ? 1 : MLKV_REDUCE_ROWS_IN_FLIGHT / KV;
+    constexpr int UNR = KV >= ROWS ? 1 : ROWS / KV;
     for (uint32_t base = 0; base < len; base += G) {
         const uint32_t cnt = min((uint32_t)G, len - base);
         const uint32_t pl = (uint32_t)glane < cnt ? __ldg(spos + s + base + glane) : 0u;
@@ -143,6 +152,10 @@ __device__ __forceinline__ void adagrad_store(const RowArgs& ra, uint32_t row, t
     }
 }
 
+// One lane group per run.  Its start, end, row and first lookup position are
+// independent loads (the segment kernel wrote them side by side); then the
+// row, the state and the first gradient row are loaded together, so a run
+// of one lookup (most of them) costs two dependent round trips.
 template <int V, int KV>
 __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra, RunArgs a) {
     using VT = typename Vec<V>::T;
@@ -154,8 +167,9 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
     for (uint32_t u = group; u < U; u += ngroups) {  // uniform within the group
         const uint32_t s = __ldg(a.seg_start + u);
         const uint32_t e = u + 1 < U ? __ldg(a.seg_start + u + 1) : nv;
+        const uint32_t row = __ldg(a.run_row + u);
+        const uint32_t p0 = __ldg(a.run_p0 + u);
         const uint32_t len = e - s;
-        const uint32_t row = __ldg(a.srow + s);
         if (len > MLKV_SEQ_SEGMENT_MAX) {
             if (glane == 0) {
                 const uint32_t nit = (len + kChunk - 1) / kChunk;
@@ -166,7 +180,10 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
                     a.long_e[h] = e;
                     a.long_row[h] = row;
                     a.long_base[h] = ib;
-                    for (uint32_t k = 0; k < nit; ++k) a.item_run[ib + k] = h;
+                    for (uint32_t k = 0; k < nit; ++k) {
+                        a.item_s[ib + k] = s + k * kChunk;
+                        a.item_e[ib + k] = min(s + (k + 1) * kChunk, e);
+                    }
                 } else {
                     record_error(a.err, MLKV_ERR_FULL);
                 }
@@ -175,31 +192,33 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
         }
         VT w[KV], Gs[KV], acc[KV];
         load_row_state<V, KV>(ra, row, w, Gs, glane);
+        const VT* g0 = reinterpret_cast<const VT*>(a.grads + (size_t)p0 * ra.d);
 #pragma unroll
-        for (int k = 0; k < KV; ++k) acc[k] = Vec<V>::zero();
-        sum_rows<V, KV>(acc, a.grads, a.spos, s, len, ra.d, ra.NV, G, glane, gmask);
+        for (int k = 0; k < KV; ++k) {
+            acc[k] = Vec<V>::zero();
+            const int j = glane + G * k;
+            if (j < ra.NV) Vec<V>::add(acc[k], __ldcs(g0 + j));  // 0 + g: first term, in order
+        }
+        if (len > 1) sum_rows<V, KV>(acc, a.grads, a.spos, s + 1, len - 1, ra.d, ra.NV, G, glane, gmask);
         adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
     }
 }
 
 template <int V, int KV>
-__global__ void __launch_bounds__(256, MLKV_REDUCE_MIN_BLOCKS) k_long_sum(RowArgs ra, RunArgs a) {
+__global__ void __launch_bounds__(256, MLKV_LONG_MIN_BLOCKS) k_long_sum(RowArgs ra, RunArgs a) {
     using VT = typename Vec<V>::T;
     const uint32_t NI = min(a.cur->n_items, a.max_items);
-    const uint32_t NL = min(a.cur->n_long, a.max_long);
     const int lane = threadIdx.x & 31, G = ra.G, glane = lane & (G - 1), gid = lane / G;
     const unsigned gmask = group_mask(G, gid);
     const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
     const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
     for (uint32_t it = group; it < NI; it += ngroups) {
-        const uint32_t h = a.item_run[it];
-        if (h >= NL) continue;  // only if the run list overflowed (reported)
-        const uint32_t s = a.long_s[h] + (it - a.long_base[h]) * kChunk;
-        const uint32_t e = min(s + kChunk, a.long_e[h]);
+        const uint32_t s = __ldg(a.item_s + it), e = __ldg(a.item_e + it);
         VT acc[KV];
 #pragma unroll
         for (int k = 0; k < KV; ++k) acc[k] = Vec<V>::zero();
-        sum_rows<V, KV>(acc, a.grads, a.spos, s, e > s ? e - s : 0u, ra.d, ra.NV, G, glane, gmask);
+        sum_rows<V, KV, MLKV_LONG_ROWS_IN_FLIGHT>(acc, a.grads, a.spos, s, e > s ? e - s : 0u, ra.d, ra.NV, G,
+                                                  glane, gmask);
         VT* part = reinterpret_cast<VT*>(a.partial + (size_t)it * ra.dpad);
 #pragma unroll
         for (int k = 0; k < KV; ++k) {
@@ -276,15 +295,17 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
                        int64_t n, cudaStream_t st, CallCounters* cur) {
     (void)n;
     RowArgs ra{t->slots, t->geom.stride, t->geom.dpad, t->geom.NV, t->geom.G, t->geom.d};
-    RunArgs a{grads, srow, spos, t->s.seg_start, cur, t->s.long_s, t->s.long_e, t->s.long_row,
-              t->s.long_base, t->s.item_run, t->s.partial, (uint32_t)t->s.max_long, (uint32_t)t->s.max_items,
-              ErrSink{&t->dstate->status, t->status_dev_alias}, t->cfg.lr, t->cfg.eps};
+    RunArgs a{grads, srow, spos, t->s.seg_start, t->s.run_row, t->s.run_p0, cur, t->s.long_s, t->s.long_e,
+              t->s.long_row, t->s.long_base, t->s.item_s, t->s.item_e, t->s.partial, (uint32_t)t->s.max_long,
+              (uint32_t)t->s.max_items, ErrSink{&t->dstate->status, t->status_dev_alias}, t->cfg.lr, t->cfg.eps};
     const int gs = persistent_blocks(t, (const void*)k_short<V, KV>, 256);
     MLKV_LAUNCH(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, st, ra, a);
     const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);
     MLKV_LAUNCH(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, st, ra, a);
-    const size_t smem = (size_t)(256 / t->geom.G) * t->geom.dpad * sizeof(float);
-    MLKV_LAUNCH(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), t->num_sms * 4, 256, smem, st, ra, a,
+    // small blocks, many of them: every long run can be combined at once
+    const int cthreads = 64;
+    const size_t smem = (size_t)(cthreads / t->geom.G) * t->geom.dpad * sizeof(float);
+    MLKV_LAUNCH(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), t->num_sms * 16, cthreads, smem, st, ra, a,
                 t->dstate);
     return cudaGetLastError();
 }

@@ -18,15 +18,18 @@ namespace mlkv {
 
 namespace {
 
-__device__ __forceinline__ ulonglong2 ld_slot_volatile(const Slot* s) {
+// Device-scope relaxed loads: they see slots published by compare-and-swap in
+// the same kernel and still hit in L2 (the coherence point of GPU accesses);
+// a volatile load would be a system-scope access.
+__device__ __forceinline__ ulonglong2 ld_slot_relaxed(const Slot* s) {
     ulonglong2 v;
-    asm volatile("ld.volatile.global.v2.u64 {%0, %1}, [%2];" : "=l"(v.x), "=l"(v.y) : "l"(s));
+    asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];" : "=l"(v.x), "=l"(v.y) : "l"(s) : "memory");
     return v;
 }
 
-__device__ __forceinline__ uint32_t ld_u32_volatile(const uint32_t* p) {
+__device__ __forceinline__ uint32_t ld_u32_relaxed(const uint32_t* p) {
     uint32_t v;
-    asm volatile("ld.volatile.global.u32 %0, [%1];" : "=r"(v) : "l"(p));
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
 
@@ -42,7 +45,7 @@ __device__ __forceinline__ uint32_t probe_key(const IndexArgs& ia, unsigned long
     }
     unsigned long long s = (ia.identity_hash ? key : hash_key(key)) & ia.mask;
     for (int i = 0; i < PROBE_LIMIT; ++i) {
-        ulonglong2 v = INSERT ? ld_slot_volatile(ia.index + s)
+        ulonglong2 v = INSERT ? ld_slot_relaxed(ia.index + s)
                               : __ldg(reinterpret_cast<const ulonglong2*>(ia.index + s));
         if (v.x == key) {
             uint32_t row = (uint32_t)v.y;
@@ -56,7 +59,7 @@ __device__ __forceinline__ uint32_t probe_key(const IndexArgs& ia, unsigned long
             unsigned long long old = atomicCAS(&ia.index[s].key, EMPTY_KEY, key);
             if (old == EMPTY_KEY || old == key) {
                 slot_out = (uint32_t)s;
-                uint32_t row = ld_u32_volatile(&ia.index[s].row);
+                uint32_t row = ld_u32_relaxed(&ia.index[s].row);
                 if (row != ROW_PENDING) return row;
                 atomicMin(&ia.index[s].aux, pos);
                 return ROW_PENDING;
@@ -107,7 +110,11 @@ IndexArgs index_args(mlkv_table* t) {
 }
 
 // ---------------------------------------------------------------------------
-// One thread per lookup: row_of_pos[p] (and the slot) for every position.
+// row_of_pos[p] (and the slot) for every position.  Each thread takes
+// kProbeKeys lookups spaced a block apart, so their loads are in flight
+// together (the probe is latency-bound: a key load, then a random slot load).
+constexpr int kProbeKeys = 4;
+
 template <bool INSERT>
 __global__ void __launch_bounds__(256) k_probe(IndexArgs ia, const int64_t* __restrict__ keys,
                                                uint32_t n, uint32_t* __restrict__ row_of_pos,
@@ -116,14 +123,24 @@ __global__ void __launch_bounds__(256) k_probe(IndexArgs ia, const int64_t* __re
                                                CallCounters* cur, CallCounters* nxt,
                                                int report_absent) {
     zero_counters(nxt);
-    const uint32_t p = blockIdx.x * blockDim.x + threadIdx.x;
-    if (p >= n) return;
-    uint32_t slot = 0;
-    const uint32_t row = probe_key<INSERT>(ia, (unsigned long long)keys[p], p, slot);
-    if (!INSERT && report_absent && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
-    row_of_pos[p] = row;
-    if (slot_of_pos) slot_of_pos[p] = slot;
-    if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
+    const uint32_t base = blockIdx.x * (blockDim.x * kProbeKeys) + threadIdx.x;
+    unsigned long long k[kProbeKeys];
+#pragma unroll
+    for (int j = 0; j < kProbeKeys; ++j) {
+        const uint32_t p = base + j * blockDim.x;
+        k[j] = p < n ? (unsigned long long)__ldg(keys + p) : 0ull;
+    }
+#pragma unroll
+    for (int j = 0; j < kProbeKeys; ++j) {
+        const uint32_t p = base + j * blockDim.x;
+        if (p >= n) continue;
+        uint32_t slot = 0;
+        const uint32_t row = probe_key<INSERT>(ia, k[j], p, slot);
+        if (!INSERT && report_absent && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
+        row_of_pos[p] = row;
+        if (slot_of_pos) slot_of_pos[p] = slot;
+        if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
+    }
 }
 
 // Group-cooperative copy of one row (or NaN) into dst.
@@ -468,10 +485,10 @@ cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool ins
                          CallCounters* nxt) {
     uint32_t* slot_of_pos = want_slot ? t->s.slot_of_pos : nullptr;
     if (insert)
-        MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<true>, grid_for(n, 256), 256, 0, st, index_args(t), keys,
+        MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<true>, grid_for(n, 256 * kProbeKeys), 256, 0, st, index_args(t), keys,
                     (uint32_t)n, t->s.row_of_pos, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0);
     else
-        MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<false>, grid_for(n, 256), 256, 0, st, index_args(t), keys,
+        MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<false>, grid_for(n, 256 * kProbeKeys), 256, 0, st, index_args(t), keys,
                     (uint32_t)n, t->s.row_of_pos, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt,
                     report_absent ? 1 : 0);
     return cudaGetLastError();

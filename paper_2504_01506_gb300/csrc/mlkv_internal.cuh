@@ -24,6 +24,8 @@ constexpr uint32_t ROW_PENDING = 0xFFFFFFFFu;   // key present, row not handed o
 constexpr uint32_t ROW_ABSENT = 0xFFFFFFFEu;    // key absent (or rejected)
 constexpr uint32_t AUX_IDLE = 0xFFFFFFFFu;
 constexpr int PROBE_LIMIT = MLKV_PROBE_LIMIT;
+constexpr int kSortMaxPasses = 4;      // row ids have at most 31 bits
+constexpr int kSortMaxDigitBits = 9;   // radix <= 512
 
 // Per-call counters.  Two copies: a call uses cc[p] and its first kernel
 // zeroes cc[p ^ 1] for the next call, so no memset is enqueued.
@@ -69,14 +71,20 @@ struct Scratch {
     uint32_t* rank;         // [max_batch]
     uint32_t* sk[2];        // sort keys (row ids), ping-pong [max_batch]
     uint32_t* sv[2];        // sort values (positions), ping-pong [max_batch]
-    uint32_t* hist;         // [256 * sort tiles]
+    uint32_t* hist;         // [256 * sort tiles] (unused by the Onesweep sort)
+    uint32_t* sort_ghist;   // [kSortMaxPasses * 512] digit starts, + tile tickets and a counter
+    int64_t sort_ghist_bytes;
+    uint32_t* sort_status;  // [kSortMaxPasses][tiles][512] look-back words
     uint32_t* tile_sums;    // [scan tiles]
     uint32_t* seg_start;    // [max_batch + 1] run starts in sorted order
+    uint32_t* run_row;      // [max_batch] row of each run
+    uint32_t* run_p0;       // [max_batch] first lookup position of each run
     uint32_t* long_s;       // [max_long] long runs: first sorted position
     uint32_t* long_e;       // [max_long] one past the last
     uint32_t* long_row;     // [max_long]
     uint32_t* long_base;    // [max_long] first chunk item
-    uint32_t* item_run;     // [max_items] long run of each chunk
+    uint32_t* item_s;       // [max_items] first sorted position of each chunk
+    uint32_t* item_e;       // [max_items] one past its last
     float* partial;         // [max_items][dpad] chunk sums
     int64_t max_long;
     int64_t max_items;
@@ -243,8 +251,8 @@ cudaError_t launch_exclusive_scan(mlkv_table* t, const uint32_t* in, uint32_t* o
                                   uint32_t* total, const uint32_t* enable, cudaStream_t st);
 cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow,
                              const uint32_t** spos);
-cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, int64_t n, cudaStream_t st,
-                            CallCounters* cur);
+cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, const uint32_t* spos, int64_t n,
+                            cudaStream_t st, CallCounters* cur);
 cudaError_t launch_dedup_out(mlkv_table* t, const int64_t* keys, const uint32_t* spos, int64_t n,
                              int64_t* uniq, int32_t* counts, int64_t* num, cudaStream_t st,
                              CallCounters* cur);

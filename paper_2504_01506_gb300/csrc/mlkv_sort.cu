@@ -2,13 +2,18 @@
 // pairs, then the segment starts of the sorted row ids.
 //
 // The sort key is the 32-bit row id, not the 64-bit key: rows are dense in
-// [0, capacity), so ceil(bits / 8) passes suffice (4 for 10^8 rows) against
-// 5+ for 40-bit keys, and the sorted order visits rows in memory order.  An
-// absent lookup is given the all-ones digit pattern and sorts last.
+// [0, capacity), so 3 passes of 9 bits cover 10^8 rows (against 5+ passes for
+// 40-bit keys), and the sorted order visits rows in memory order.  An absent
+// lookup is given the all-ones digit pattern and sorts last.
 //
-// Per pass: a per-tile digit histogram, an exclusive scan of the
-// digit-major [digit][tile] counts, and a scatter whose within-tile ranks are
-// stable (warp match over each round of 32 items, rounds and warps in order).
+// The sort follows the single-pass ("Onesweep") scheme of Adinets & Merrill
+// (2022): one kernel reads the keys once and counts the digits of every pass;
+// then each pass is one kernel in which a block ranks its 4096-element tile
+// (stable: warp match over rounds of 32 in order), publishes its per-digit
+// count, and finds the count of all earlier tiles by looking back over their
+// published values (decoupled look-back).  Tiles are taken in launch order
+// from an atomic ticket, so every tile looked at is held by a running block;
+// each poll loop is bounded and reports MLKV_ERR_TIMEOUT if it runs out.
 #include "mlkv_internal.cuh"
 
 namespace mlkv {
@@ -117,36 +122,77 @@ __device__ __forceinline__ uint32_t sort_key(uint32_t r, uint32_t sent, bool fir
     return first ? (r >= ROW_ABSENT ? sent : r) : r;
 }
 
-__global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restrict__ keys, uint32_t n,
-                                                        uint32_t* __restrict__ hist, uint32_t ntiles,
-                                                        int shift, int radix, uint32_t sent, int first) {
-    __shared__ uint32_t cnt[256];
-    for (int i = threadIdx.x; i < radix; i += kThreads) cnt[i] = 0;
+constexpr int kMaxRadix = 1 << kSortMaxDigitBits;
+constexpr uint32_t kFlagAgg = 1u << 30, kFlagIncl = 2u << 30, kValMask = (1u << 30) - 1;
+constexpr int kPollIters = 1 << 22;
+
+// Look-back words are read and published with device-scope relaxed accesses
+// (value and flag share one 32-bit word, so no further ordering is needed).
+__device__ __forceinline__ uint32_t ld_word(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void st_word(uint32_t* p, uint32_t v) {
+    asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+}
+
+// Digit counts of every pass in one read; the last block to finish turns
+// them into exclusive prefix sums (per pass) and clears the look-back words.
+__global__ void __launch_bounds__(kThreads) k_sort_count(const uint32_t* __restrict__ keys, uint32_t n,
+                                                         uint32_t sent, int passes, int D, uint32_t* ghist,
+                                                         uint32_t* status, uint32_t status_len,
+                                                         uint32_t* done_ctr) {
+    __shared__ uint32_t cnt[kSortMaxPasses][kMaxRadix];
+    __shared__ bool last;
+    const int radix = 1 << D;
+    for (int i = threadIdx.x; i < kSortMaxPasses * kMaxRadix; i += kThreads) (&cnt[0][0])[i] = 0;
+    for (uint32_t i = blockIdx.x * kThreads + threadIdx.x; i < status_len; i += gridDim.x * kThreads) status[i] = 0;
     __syncthreads();
-    const uint32_t base = blockIdx.x * kTile;
-#pragma unroll 4
-    for (int k = 0; k < kItems; ++k) {
-        const uint32_t i = base + k * kThreads + threadIdx.x;
-        if (i < n) atomicAdd(&cnt[(sort_key(keys[i], sent, first) >> shift) & (radix - 1)], 1u);
+    for (uint32_t i = blockIdx.x * kThreads + threadIdx.x; i < n; i += gridDim.x * kThreads) {
+        const uint32_t k = sort_key(keys[i], sent, true);
+        for (int p = 0; p < passes; ++p) atomicAdd(&cnt[p][(k >> (p * D)) & (radix - 1)], 1u);
     }
     __syncthreads();
-    for (int d = threadIdx.x; d < radix; d += kThreads) hist[(size_t)d * ntiles + blockIdx.x] = cnt[d];
+    for (int p = 0; p < passes; ++p)
+        for (int d = threadIdx.x; d < radix; d += kThreads)
+            if (cnt[p][d]) atomicAdd(&ghist[p * kMaxRadix + d], cnt[p][d]);
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) last = atomicAdd(done_ctr, 1u) == gridDim.x - 1;
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    for (int p = 0; p < passes; ++p) {
+        // radix <= 512: two counts per thread, block scan of the pair sums
+        const int d0 = threadIdx.x * 2;
+        const uint32_t a = d0 < radix ? __ldcg(&ghist[p * kMaxRadix + d0]) : 0u;
+        const uint32_t b = d0 + 1 < radix ? __ldcg(&ghist[p * kMaxRadix + d0 + 1]) : 0u;
+        uint32_t total;
+        const uint32_t excl = block_exclusive_scan(a + b, total);
+        if (d0 < radix) ghist[p * kMaxRadix + d0] = excl;
+        if (d0 + 1 < radix) ghist[p * kMaxRadix + d0 + 1] = excl + a;
+        __syncthreads();
+    }
 }
 
 __global__ void __launch_bounds__(kThreads) k_sort_scatter(const uint32_t* __restrict__ kin,
                                                            const uint32_t* __restrict__ vin,
                                                            uint32_t* __restrict__ kout,
                                                            uint32_t* __restrict__ vout, uint32_t n,
-                                                           const uint32_t* __restrict__ hist,
-                                                           uint32_t ntiles, int shift, int radix,
-                                                           uint32_t sent, int first) {
-    __shared__ uint32_t wcnt[kWarps][256];
-    __shared__ uint32_t gbase[256];
+                                                           const uint32_t* __restrict__ gstart,
+                                                           uint32_t* status, uint32_t* tile_ctr, int shift,
+                                                           int radix, uint32_t sent, int first, ErrSink err) {
+    __shared__ uint32_t wcnt[kWarps][kMaxRadix];
+    __shared__ uint32_t gbase[kMaxRadix];
+    __shared__ uint32_t tile_s;
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    for (int i = threadIdx.x; i < kWarps * 256; i += kThreads) (&wcnt[0][0])[i] = 0;
-    for (int d = threadIdx.x; d < radix; d += kThreads) gbase[d] = hist[(size_t)d * ntiles + blockIdx.x];
+    if (threadIdx.x == 0) tile_s = atomicAdd(tile_ctr, 1u);
+    for (int i = threadIdx.x; i < kWarps * kMaxRadix; i += kThreads) (&wcnt[0][0])[i] = 0;
     __syncthreads();
-    const uint32_t base = blockIdx.x * kTile + w * (kItems * 32);
+    const uint32_t tile = tile_s;
+    const uint32_t base = tile * kTile + w * (kItems * 32);
     const uint32_t lt = lanemask_lt();
     uint32_t key[kItems], val[kItems], rnk[kItems];
 #pragma unroll
@@ -167,6 +213,8 @@ __global__ void __launch_bounds__(kThreads) k_sort_scatter(const uint32_t* __res
         rnk[r] = valid ? before + __popc(peers & lt) : 0xFFFFFFFFu;
     }
     __syncthreads();
+    // per digit: exclusive prefix over the warps, the tile's count, then the
+    // look-back for the count of all earlier tiles
     for (int d = threadIdx.x; d < radix; d += kThreads) {
         uint32_t run = 0;
 #pragma unroll
@@ -175,6 +223,27 @@ __global__ void __launch_bounds__(kThreads) k_sort_scatter(const uint32_t* __res
             wcnt[ww][d] = run;
             run += c;
         }
+        uint32_t* my = status + (size_t)tile * radix + d;
+        if (tile == 0) {
+            st_word(my, kFlagIncl | run);
+            gbase[d] = gstart[d];
+            continue;
+        }
+        st_word(my, kFlagAgg | run);
+        uint32_t excl = 0;
+        for (int t = (int)tile - 1; t >= 0; --t) {
+            const uint32_t* q = status + (size_t)t * radix + d;
+            uint32_t v = ld_word(q);
+            for (int it = 0; it < kPollIters && (v & ~kValMask) == 0; ++it) v = ld_word(q);
+            if ((v & ~kValMask) == 0) {
+                record_error(err, MLKV_ERR_TIMEOUT);
+                break;
+            }
+            excl += v & kValMask;
+            if (v & kFlagIncl) break;
+        }
+        st_word(my, kFlagIncl | (excl + run));
+        gbase[d] = gstart[d] + excl;
     }
     __syncthreads();
 #pragma unroll
@@ -205,9 +274,12 @@ __global__ void __launch_bounds__(kThreads) k_seg_reduce(const uint32_t* __restr
     if (threadIdx.x == 0) tile_sums[blockIdx.x] = total;
 }
 
-__global__ void __launch_bounds__(kThreads) k_seg_down(const uint32_t* __restrict__ srow, uint32_t n,
+__global__ void __launch_bounds__(kThreads) k_seg_down(const uint32_t* __restrict__ srow,
+                                                       const uint32_t* __restrict__ spos, uint32_t n,
                                                        uint32_t sent, const uint32_t* __restrict__ tile_sums,
-                                                       uint32_t* __restrict__ seg_start, CallCounters* cur,
+                                                       uint32_t* __restrict__ seg_start,
+                                                       uint32_t* __restrict__ run_row,
+                                                       uint32_t* __restrict__ run_p0, CallCounters* cur,
                                                        DevState* ds) {
     const uint32_t base = blockIdx.x * kTile;
     const uint32_t prefix = tiles_before(tile_sums, blockIdx.x);
@@ -227,7 +299,13 @@ __global__ void __launch_bounds__(kThreads) k_seg_down(const uint32_t* __restric
     uint32_t run = block_exclusive_scan(cnt, block_total) + prefix;
 #pragma unroll
     for (int k = 0; k < kItems; ++k)
-        if (flags & (1u << k)) seg_start[run++] = first + k;
+        if (flags & (1u << k)) {
+            const uint32_t p = first + k;
+            seg_start[run] = p;
+            run_row[run] = srow[p];
+            run_p0[run] = spos[p];
+            ++run;
+        }
     if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) {
         cur->n_unique = prefix + block_total;
         ds->last_unique = prefix + block_total;
@@ -262,24 +340,30 @@ cudaError_t launch_exclusive_scan(mlkv_table* t, const uint32_t* in, uint32_t* o
 cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow,
                              const uint32_t** spos) {
     const int bits = t->sort_bits;
-    const int passes = (bits + 7) / 8;
+    const int passes = (bits + kSortMaxDigitBits - 1) / kSortMaxDigitBits;
     const int D = (bits + passes - 1) / passes;
     const int radix = 1 << D;
     const uint32_t sent = (uint32_t)((1ull << bits) - 1);
     const unsigned nt = tiles(n);
+    // digit counts, tile tickets and the completion counter start at zero
+    cudaError_t e = cudaMemsetAsync(t->s.sort_ghist, 0, t->s.sort_ghist_bytes, st);
+    if (e != cudaSuccess) return e;
+    uint32_t* ghist = t->s.sort_ghist;
+    uint32_t* tile_ctr = ghist + kSortMaxPasses * kMaxRadix;
+    uint32_t* done_ctr = tile_ctr + kSortMaxPasses;
+    const uint32_t status_len = (uint32_t)((int64_t)passes * nt * radix);
+    int64_t cg = nt;
+    if (cg > (int64_t)t->num_sms * 4) cg = (int64_t)t->num_sms * 4;
+    MLKV_LAUNCH(t, 0, k_sort_count, (unsigned)cg, kThreads, 0, st, t->s.row_of_pos, (uint32_t)n, sent, passes,
+                D, ghist, t->s.sort_status, status_len, done_ctr);
+    const ErrSink err{&t->dstate->status, t->status_dev_alias};
     const uint32_t* kin = t->s.row_of_pos;
     const uint32_t* vin = nullptr;
     int out = 0;
     for (int p = 0; p < passes; ++p) {
-        const int first = p == 0;
-        const int shift = p * D;
-        MLKV_LAUNCH(t, 0, k_sort_hist, nt, kThreads, 0, st, kin, (uint32_t)n, t->s.hist, nt, shift, radix,
-                    sent, first);
-        cudaError_t e = launch_exclusive_scan(t, t->s.hist, t->s.hist, (int64_t)radix * nt, nullptr,
-                                              nullptr, st);
-        if (e != cudaSuccess) return e;
         MLKV_LAUNCH(t, MLKV_K_SORT_SCATTER, k_sort_scatter, nt, kThreads, 0, st, kin, vin, t->s.sk[out],
-                    t->s.sv[out], (uint32_t)n, t->s.hist, nt, shift, radix, sent, first);
+                    t->s.sv[out], (uint32_t)n, ghist + p * kMaxRadix,
+                    t->s.sort_status + (size_t)p * nt * radix, tile_ctr + p, p * D, radix, sent, p == 0, err);
         kin = t->s.sk[out];
         vin = t->s.sv[out];
         out ^= 1;
@@ -289,13 +373,13 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
     return cudaGetLastError();
 }
 
-cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, int64_t n, cudaStream_t st,
-                            CallCounters* cur) {
+cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, const uint32_t* spos, int64_t n,
+                            cudaStream_t st, CallCounters* cur) {
     const uint32_t sent = (uint32_t)((1ull << t->sort_bits) - 1);
     const unsigned nt = tiles(n);
     MLKV_LAUNCH(t, MLKV_K_SEGMENTS, k_seg_reduce, nt, kThreads, 0, st, srow, (uint32_t)n, sent, t->s.tile_sums);
-    MLKV_LAUNCH(t, MLKV_K_SEGMENTS, k_seg_down, nt, kThreads, 0, st, srow, (uint32_t)n, sent, t->s.tile_sums,
-                t->s.seg_start, cur, t->dstate);
+    MLKV_LAUNCH(t, MLKV_K_SEGMENTS, k_seg_down, nt, kThreads, 0, st, srow, spos, (uint32_t)n, sent,
+                t->s.tile_sums, t->s.seg_start, t->s.run_row, t->s.run_p0, cur, t->dstate);
     return cudaGetLastError();
 }
 

@@ -192,7 +192,7 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     const mlkv_config c = *cfg;
     if (c.dim < 1 || c.dim > MLKV_MAX_DIM || (c.dim > 256 && c.dim % 4)) return MLKV_ERR_INVALID;
     if (c.capacity < 1 || c.capacity >= (1ll << 31) - 2) return MLKV_ERR_INVALID;
-    if (c.max_batch < 1 || c.max_batch >= (1ll << 31) - 2) return MLKV_ERR_INVALID;
+    if (c.max_batch < 1 || c.max_batch >= (1ll << 30)) return MLKV_ERR_INVALID;
     if (c.reserved != 0 || (c.flags & ~MLKV_IDENTITY_HASH)) return MLKV_ERR_INVALID;
     if (!(c.init_hi >= c.init_lo)) return MLKV_ERR_INVALID;
     if (c.staleness_bound != 0 || c.hbm_cache_rows != 0) return MLKV_ERR_UNSUPPORTED;
@@ -234,6 +234,7 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     s.max_long = long_runs_bound(B);
     s.max_items = long_items_bound(B);
     s.hist_len = 256 * tiles_of(B);
+    s.sort_ghist_bytes = (kSortMaxPasses * 512 + kSortMaxPasses + 4) * 4;
     s.tile_sums_len = (tiles_of(B) > tiles_of(s.hist_len) ? tiles_of(B) : tiles_of(s.hist_len)) + 1;
     struct Piece {
         void** ptr;
@@ -246,9 +247,13 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
         {(void**)&s.sk[0], B * 4},          {(void**)&s.sk[1], B * 4},
         {(void**)&s.sv[0], B * 4},          {(void**)&s.sv[1], B * 4},
         {(void**)&s.hist, s.hist_len * 4},  {(void**)&s.tile_sums, s.tile_sums_len * 4},
+        {(void**)&s.sort_ghist, s.sort_ghist_bytes},
+        {(void**)&s.sort_status, (int64_t)kSortMaxPasses * tiles_of(B) * 512 * 4},
         {(void**)&s.seg_start, (B + 1) * 4},  {(void**)&s.long_s, s.max_long * 4},
         {(void**)&s.long_e, s.max_long * 4},   {(void**)&s.long_row, s.max_long * 4},
-        {(void**)&s.long_base, s.max_long * 4}, {(void**)&s.item_run, s.max_items * 4},
+        {(void**)&s.long_base, s.max_long * 4}, {(void**)&s.item_s, s.max_items * 4},
+        {(void**)&s.item_e, s.max_items * 4},   {(void**)&s.run_row, B * 4},
+        {(void**)&s.run_p0, B * 4},
         {(void**)&s.partial, s.max_items * t->geom.dpad * 4},
     };
     int64_t total = 0;
@@ -311,7 +316,7 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
     if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
     const uint32_t *srow, *spos;
     CK(t, launch_sort_rows(t, n, st, &srow, &spos));
-    CK(t, launch_segments(t, srow, n, st, cs.cur));
+    CK(t, launch_segments(t, srow, spos, n, st, cs.cur));
     CK(t, launch_reduce_apply(t, d_grads, srow, spos, n, st, cs.cur));
     return MLKV_OK;
 }
@@ -359,7 +364,7 @@ int mlkv_dedup(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_uniqu
     CK(t, launch_probe(t, d_keys, n, false, false, false, st, cs.cur, cs.nxt));
     const uint32_t *srow, *spos;
     CK(t, launch_sort_rows(t, n, st, &srow, &spos));
-    CK(t, launch_segments(t, srow, n, st, cs.cur));
+    CK(t, launch_segments(t, srow, spos, n, st, cs.cur));
     CK(t, launch_dedup_out(t, d_keys, spos, n, d_unique_keys, d_counts, d_num_unique, st, cs.cur));
     return MLKV_OK;
 }
