@@ -179,9 +179,10 @@ def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
 
 KERNEL_NAMES = {1: "k_get (probe + row gather)", 2: "k_probe", 3: "k_sort_scatter",
                 4: "k_short (run sum + Adagrad)", 5: "k_long_sum (chunk sums of long runs)",
-                6: "segments", 7: "k_long_combine (chunk sums + Adagrad)"}
+                6: "segments", 7: "k_long_combine (chunk sums + Adagrad)",
+                8: "k_tier_fetch (host <-> HBM row swap)"}
 KERNEL_SOURCES = {1: "mlkv_index.cu", 2: "mlkv_index.cu", 3: "mlkv_sort.cu", 4: "mlkv_apply.cu",
-                  5: "mlkv_apply.cu", 6: "mlkv_sort.cu", 7: "mlkv_apply.cu"}
+                  5: "mlkv_apply.cu", 6: "mlkv_sort.cu", 7: "mlkv_apply.cu", 8: "mlkv_tier.cu"}
 
 
 def traffic_for(kid: int):
@@ -268,8 +269,29 @@ def run_reference(args, cfg):
     return 0
 
 
+def dma_peak(torch, dev) -> dict:
+    """Pinned host <-> device copy bandwidth (1 GiB, best of 3), GB/s."""
+    n = 1 << 28
+    h = torch.empty(n, dtype=torch.float32).pin_memory()
+    d = torch.empty(n, dtype=torch.float32, device=dev)
+    out = {}
+    for name, fn in (("h2d", lambda: d.copy_(h, non_blocking=True)), ("d2h", lambda: h.copy_(d, non_blocking=True))):
+        best = 0.0
+        for _ in range(3):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            torch.cuda.synchronize()
+            best = max(best, 4 * n / (e0.elapsed_time(e1) / 1e3) / 1e9)
+        out[name] = best
+    return out
+
+
 def workload_config(cfg) -> dict:
-    c = {"workload": f"{cfg.name}: {cfg.n_keys:,} rows x dim {cfg.dim} fp32 (+ Adagrad state) in HBM, "
+    where = (f"in host memory behind an HBM cache of {cfg.hbm_cache_rows:,} rows" if cfg.hbm_cache_rows
+             else "in HBM")
+    c = {"workload": f"{cfg.name}: {cfg.n_keys:,} rows x dim {cfg.dim} fp32 (+ Adagrad state) {where}, "
                      f"{cfg.batch:,} lookups/step",
          "rows": cfg.n_keys, "dim": cfg.dim, "batch_lookups": cfg.batch, "lr": cfg.lr,
          "l2": "inputs larger than L2 every step (gradients and Get output 4*dim B per lookup)"}
@@ -289,21 +311,40 @@ def run_ours(args, cfg):
     dev = torch.device("cuda", local)
     hbm_peak, peak_kind = peaks()
 
+    tiered = cfg.hbm_cache_rows > 0
     store = EmbeddingStore(dim=cfg.dim, capacity=cfg.n_keys, max_batch=cfg.batch, lr=cfg.lr, eps=cfg.eps,
                            state_init=cfg.state_init, init_lo=cfg.init_lo, init_hi=cfg.init_hi,
-                           seed=cfg.seed, device=dev)
+                           seed=cfg.seed, hbm_cache_rows=cfg.hbm_cache_rows, device=dev)
     # preload every key of the table (untimed), in preload order
     chunk = cfg.batch
     for s in range(0, cfg.n_keys, chunk):
         store.insert(torch.from_numpy(cfg.preload_keys(s, s + chunk)).to(dev))
     assert store.sync() == 0, "preload failed"
 
-    pool = max(1, min(args.pool, args.steps + args.warmup))
+    if tiered and args.tier_prefill:
+        # fill the HBM cache with rows of random keys, each updated once (so the
+        # cache starts full, as in a long run, and the timed steps evict)
+        rng = np.random.default_rng(5)
+        fill = rng.choice(cfg.n_keys, size=min(cfg.hbm_cache_rows, cfg.n_keys), replace=False).astype(np.int64)
+        zeros = torch.zeros((cfg.batch, cfg.dim), dtype=torch.float32, device=dev)
+        for s0 in range(0, len(fill), cfg.batch):
+            k = torch.from_numpy(fill[s0:s0 + cfg.batch]).to(dev)  # tiered keys are 0..n_keys-1
+            store.get(k)
+            store.apply_grad(k, zeros[:k.numel()])
+        assert store.sync() == 0, "prefill failed"
+
+    # The HBM store cycles a pool of batches.  The tiered store gets a fresh batch
+    # every step (a cycled pool would end up resident in its cache): one per
+    # kernel-class prepass step, warm-up step, timed step, and the last look-ahead.
+    kinds = (1, 2, 3, 4, 5, 6, 7) + ((8,) if tiered else ())
+    base = len(kinds) if tiered else 0
+    pool = base + args.warmup + args.steps + 1 if tiered else max(1, min(args.pool, args.steps + args.warmup))
+    ngrad = max(1, min(args.pool, pool))
     keys_h = [cfg.batch_keys(s) for s in range(pool)]
     keys_d = [torch.from_numpy(k).to(dev) for k in keys_h]
     gen = torch.Generator(device=dev)
     grads_d = []
-    for s in range(pool):
+    for s in range(ngrad):
         gen.manual_seed(cfg.seed * 1000 + s)
         grads_d.append(torch.randn((cfg.batch, cfg.dim), generator=gen, device=dev) * cfg.grad_sigma)
     out = torch.empty((cfg.batch, cfg.dim), dtype=torch.float32, device=dev)
@@ -313,19 +354,21 @@ def run_ours(args, cfg):
     def step(i):
         j = i % pool
         store.get(keys_d[j], out=out)
-        store.apply_grad(keys_d[j], grads_d[j])
+        if tiered:  # Lookahead(next keys) runs beside this step's apply
+            store.lookahead(keys_d[(i + 1) % pool])
+        store.apply_grad(keys_d[j], grads_d[i % ngrad])
 
     # pick the dominant kernel: one step per kernel class, timed with events
     kernel_ms = {}
-    for kid in (1, 2, 3, 4, 5, 6, 7):
+    for idx, kid in enumerate(kinds):
         store.time_kernel(kid)
-        step(0)
+        step(idx if tiered else 0)
         ms, n = store.kernel_time()
         kernel_ms[kid] = ms
     store.time_kernel(0)
     dominant = max(kernel_ms, key=kernel_ms.get)
     for i in range(args.warmup):
-        step(i)
+        step(base + i)
     assert store.sync() == 0
 
     stream = torch.cuda.current_stream(dev)
@@ -333,19 +376,21 @@ def run_ours(args, cfg):
     clocks = ClockSampler(local)
     store.time_kernel(dominant)
     launches0 = store.launch_count()
+    tier0 = store.tier_stats()
     barrier(dist, torch)
     clocks.start()
     if args.profile:
         torch.cuda.profiler.start()
     ev0.record(stream)
     for i in range(args.steps):
-        step(args.warmup + i)
+        step(base + args.warmup + i)
     ev1.record(stream)
     barrier(dist, torch)
     if args.profile:
         torch.cuda.profiler.stop()
     clocks.stop()
     launches = store.launch_count() - launches0
+    tier1 = store.tier_stats()
     dom_ms, dom_n = store.kernel_time()
     store.time_kernel(0)
     assert store.sync() == 0, "device status set during the timed region"
@@ -357,24 +402,44 @@ def run_ours(args, cfg):
     achieved_step = step_bytes * args.steps / (elapsed_ms / 1e3) / 1e9
 
     # roofline of the dominant kernel over the timed region
-    steps_idx = [(args.warmup + i) % pool for i in range(args.steps)]
-    per_launch_bytes = np.mean([kernel_bytes(stats[j], dominant, passes) for j in steps_idx])
-    if dominant in (3, 6):  # several launches per step
-        per_launch_bytes = per_launch_bytes  # per launch of that kernel
     avg_ms = dom_ms / max(dom_n, 1)
-    achieved = per_launch_bytes / (avg_ms / 1e3) / 1e9
-    roofline = {"bound": "hbm", "kernel": KERNEL_NAMES[dominant], "achieved": achieved, "peak": hbm_peak,
-                "unit": "GB/s", "frac": achieved / hbm_peak, "peak_kind": peak_kind,
-                "traffic": traffic_for(dominant), "bytes_per_launch": per_launch_bytes,
-                "avg_launch_ms": avg_ms, "launches": dom_n,
-                "share_of_step": dom_ms / elapsed_ms if elapsed_ms else None}
+    tier = None
+    if tiered:
+        slot_bytes = 2 * ((cfg.dim + 7) // 8 * 8) * 4
+        fetched, written = tier1[0] - tier0[0], tier1[1] - tier0[1]
+        link_bytes = (fetched + written) * slot_bytes
+        link_gbs = link_bytes / (elapsed_ms / 1e3) / 1e9
+        peak = dma_peak(torch, dev)
+        tier = {"host_rows": cfg.n_keys, "cache_rows": cfg.hbm_cache_rows, "rows_fetched_per_step": fetched / args.steps,
+                "rows_written_back_per_step": written / args.steps,
+                "sweep_lines_per_step": (tier1[2] - tier0[2]) / args.steps,
+                "link_bytes_per_step": link_bytes / args.steps, "link_gbs_over_step": link_gbs,
+                "dma_peak_gbs": peak}
+    if dominant == 8:
+        # the swap kernel moves each fetched row in and each victim out over the host link
+        per_launch_bytes = link_bytes / max(dom_n, 1)
+        achieved = per_launch_bytes / (avg_ms / 1e3) / 1e9
+        roofline = {"bound": "host-link", "kernel": KERNEL_NAMES[8], "achieved": achieved, "peak": peak["h2d"],
+                    "unit": "GB/s", "frac": achieved / peak["h2d"],
+                    "peak_kind": "measured in this run (pinned cudaMemcpyAsync H2D, 1 GiB, sequential)",
+                    "traffic": None, "bytes_per_launch": per_launch_bytes, "avg_launch_ms": avg_ms,
+                    "launches": dom_n, "share_of_step": dom_ms / elapsed_ms if elapsed_ms else None}
+    else:
+        steps_idx = [(base + args.warmup + i) % pool for i in range(args.steps)]
+        per_launch_bytes = np.mean([kernel_bytes(stats[j], dominant, passes) for j in steps_idx])
+        achieved = per_launch_bytes / (avg_ms / 1e3) / 1e9
+        roofline = {"bound": "hbm", "kernel": KERNEL_NAMES[dominant], "achieved": achieved, "peak": hbm_peak,
+                    "unit": "GB/s", "frac": achieved / hbm_peak, "peak_kind": peak_kind,
+                    "traffic": traffic_for(dominant), "bytes_per_launch": per_launch_bytes,
+                    "avg_launch_ms": avg_ms, "launches": dom_n,
+                    "share_of_step": dom_ms / elapsed_ms if elapsed_ms else None}
 
     # end to end through the host-buffer calls (copies inside the timed region)
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not tiered:
         e2e_pool = min(pool, 2)
         hk = [torch.from_numpy(keys_h[j]).pin_memory() for j in range(e2e_pool)]
-        hg = [grads_d[j].cpu().pin_memory() for j in range(e2e_pool)]
+        hg = [grads_d[j % ngrad].cpu().pin_memory() for j in range(e2e_pool)]
         hout = torch.empty((cfg.batch, cfg.dim), dtype=torch.float32).pin_memory()
         e2e_steps = max(1, min(args.steps, 20))
         for i in range(2):
@@ -417,6 +482,8 @@ def run_ours(args, cfg):
             "roofline": roofline, "kernel_ms_one_step": {KERNEL_NAMES[k]: v for k, v in kernel_ms.items()},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clocks.summary(),
         }
+        if tier is not None:
+            line["tier"] = tier
         print(json.dumps(line), flush=True)
     store.close()
     if dist is not None:
@@ -437,12 +504,25 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile", action="store_true",
                     help="bracket the timed region with cudaProfilerStart/Stop (ncu --profile-from-start off)")
+    ap.add_argument("--tier-rows", type=int, default=96_000_000,
+                    help="tiered config: rows of the host tier (1 KiB each with state)")
+    ap.add_argument("--tier-cache-rows", type=int, default=0,
+                    help="tiered config: rows cached in HBM (default: the workload's 120 GB cache over "
+                         "400M rows, scaled with --tier-rows)")
+    ap.add_argument("--no-tier-prefill", dest="tier_prefill", action="store_false",
+                    help="tiered config: start with an empty HBM cache")
     ap.add_argument("--scale", type=int, default=1,
                     help="divide the table's rows by this (same batch); for small profiling cases")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     cfg = W.ALL[args.config]()
+    if args.config == "tiered":
+        # the host tier must fit the machine's host memory: scale the row count, and
+        # the HBM cache with it (same cached fraction of the rows)
+        full_rows, full_cache = cfg.n_keys, cfg.hbm_cache_rows
+        cfg.n_keys = args.tier_rows
+        cfg.hbm_cache_rows = args.tier_cache_rows or int(full_cache * args.tier_rows / full_rows)
     if args.scale > 1:
         cfg = W.scaled(cfg, args.scale, 1)
     if args.impl == "reference":

@@ -91,7 +91,9 @@ typedef struct mlkv_config {
     float init_lo, init_hi;  /* a new row is drawn U[init_lo, init_hi) by the counter-based init */
     uint64_t seed;           /* seed of the counter-based init */
     int64_t staleness_bound; /* MLKV's consistency bound; 0 (bulk-synchronous) is the only one accepted */
-    int64_t hbm_cache_rows;  /* 0: the whole table is resident in HBM; > 0 is not accepted yet */
+    int64_t hbm_cache_rows;  /* 0: rows + state resident in HBM.  > 0: rows + state live in host
+                                memory (the tier) and this many rows are cached in HBM; it must be
+                                >= 2 * max_batch + 64 (a call and a look-ahead in flight) */
     uint32_t flags;          /* 0 or MLKV_IDENTITY_HASH */
     uint32_t reserved;       /* 0 */
 } mlkv_config;
@@ -106,10 +108,15 @@ typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
 
 /* Creates a table on the current CUDA device.  Allocates rows + state
  * (capacity x 2 x dim fp32, rows padded to 32 bytes), the index (a power of
- * two >= 2 x capacity slots of 16 bytes) and scratch for max_batch.
+ * two >= 2 x capacity slots of 16 bytes) and scratch for max_batch.  With
+ * hbm_cache_rows > 0 the rows + state are allocated in host memory instead
+ * (capacity slots, huge-page backed, registered with CUDA and mapped), with an
+ * HBM cache of hbm_cache_rows rows, a row -> location map (cache line or host
+ * slot; a row fetched into the cache hands its host slot to the row it
+ * evicts), and a side stream for look-ahead.
  * Returns MLKV_ERR_INVALID (bad field), MLKV_ERR_UNSUPPORTED
- * (staleness_bound != 0, hbm_cache_rows != 0), MLKV_ERR_NOMEM or
- * MLKV_ERR_CUDA.  On success *out owns everything; free it with mlkv_close. */
+ * (staleness_bound != 0), MLKV_ERR_NOMEM or MLKV_ERR_CUDA.  On success *out
+ * owns everything; free it with mlkv_close. */
 int mlkv_open(const mlkv_config* cfg, mlkv_table** out);
 
 /* Waits for the table's work, frees all its memory.  Null is a no-op. */
@@ -135,13 +142,24 @@ int mlkv_insert(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream);
  * d_keys, g = sum of d_grads[i][:] over the i with d_keys[i] == k, then one
  * Adagrad step on k's row and state.  d_grads is fp32 [n][dim].  Absent keys
  * are inserted first when insert_on_miss, else skipped with
- * MLKV_ERR_NOT_FOUND recorded. */
+ * MLKV_ERR_NOT_FOUND recorded.
+ * Tiered table with a look-ahead in flight: this call runs beside the
+ * look-ahead (they overlap on the GPU); it may then only update keys that the
+ * Get before the look-ahead returned (the training-loop order Get(t),
+ * Lookahead(t+1), apply(t)); other keys are skipped with MLKV_ERR_INVALID
+ * (absent ones with MLKV_ERR_NOT_FOUND) recorded. */
 int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_grads,
                     void* stream);
 
-/* Lookahead of MLKV Section 3.1 / 3.3.2 with dest = the store's buffer.  A row
- * already resident is not copied again (Section 3.3.2); with the whole table
- * in HBM every row is resident, so the call checks its arguments and returns.
+/* Lookahead of MLKV Section 3.1 / 3.3.2 with dest = the store's buffer: the
+ * rows of d_keys are brought into the HBM cache ahead of use.  A row already
+ * resident is not copied again (Section 3.3.2).  With the whole table in HBM
+ * every row is resident, so the call checks its arguments and returns.  On a
+ * tiered table the work (probe, cache-line hand-out, host <-> HBM swap of
+ * each fetched row with the row it evicts) runs on the table's side stream after everything issued
+ * on `stream` before it; it does not wait for, and may overlap, the next
+ * apply_grad; every other later call waits for it.  Absent keys are skipped
+ * (not inserted).  d_keys must stay valid until the look-ahead completes.
  * (dest = the application's cache is a Get into a buffer ahead of use.) */
 int mlkv_lookahead(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream);
 
@@ -204,6 +222,11 @@ int64_t mlkv_size(mlkv_table* t);
 /* Number of kernels this table has launched since open (host counter). */
 int64_t mlkv_launch_count(mlkv_table* t);
 
+/* Tiered table, since open (synchronises; zeros for an HBM-resident table):
+ * rows copied host -> HBM cache, rows written back HBM -> host (every evicted
+ * row), and cache lines the clock sweep looked at to find victims. */
+int mlkv_tier_stats(mlkv_table* t, int64_t* rows_fetched, int64_t* rows_written_back, int64_t* sweep_lines);
+
 /* Per-kernel timing with CUDA events recorded on the launching stream around
  * every launch of kernel `kernel_id` (MLKV_K_*); 0 turns it off.  Read it with
  * mlkv_kernel_time, which synchronises and returns the summed milliseconds and
@@ -215,6 +238,7 @@ int64_t mlkv_launch_count(mlkv_table* t);
 #define MLKV_K_REDUCE_LONG 5
 #define MLKV_K_SEGMENTS 6
 #define MLKV_K_LONG_COMBINE 7
+#define MLKV_K_TIER_FETCH 8
 int mlkv_time_kernel(mlkv_table* t, int32_t kernel_id);
 int mlkv_kernel_time(mlkv_table* t, double* total_ms, int64_t* launches);
 

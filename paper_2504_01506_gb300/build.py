@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 ROOT = os.path.dirname(HERE)
 LIB = os.path.join(HERE, "libmlkv_gb300.so")
 BUILD = os.path.join(ROOT, "_build")
-SOURCES = ["mlkv_index.cu", "mlkv_sort.cu", "mlkv_apply.cu", "mlkv_table.cu", "mlkv_static.cu"]
+SOURCES = ["mlkv_index.cu", "mlkv_sort.cu", "mlkv_apply.cu", "mlkv_table.cu", "mlkv_tier.cu", "mlkv_static.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "--fmad=false", "-Xcompiler", "-fPIC",
          "-Xcompiler", "-ffp-contract=off", f"-I{os.path.join(ROOT, 'include')}"]

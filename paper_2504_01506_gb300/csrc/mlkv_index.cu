@@ -87,7 +87,7 @@ __device__ __forceinline__ void append_miss(CallCounters* cur, uint32_t* miss_po
 }
 
 __device__ __forceinline__ void zero_counters(CallCounters* nxt) {
-    if (blockIdx.x == 0 && threadIdx.x < sizeof(CallCounters) / 4)
+    if (nxt && blockIdx.x == 0 && threadIdx.x < sizeof(CallCounters) / 4)
         reinterpret_cast<uint32_t*>(nxt)[threadIdx.x] = 0u;
 }
 
@@ -366,11 +366,20 @@ __global__ void __launch_bounds__(256) k_find(IndexArgs ia, const int64_t* __res
 }
 
 // Export: like Get without insertion, copying row and/or state.
+// With a tier, a row is read from its cache line when it has one, else from
+// its host slot.
+struct ExportTier {
+    const uint32_t* row_loc;
+    const float* cache;
+    const float* host;
+};
+
 template <int V, int KV>
 __global__ void __launch_bounds__(256) k_export(IndexArgs ia, RowArgs ra,
                                                 const int64_t* __restrict__ keys, uint32_t n,
                                                 float* __restrict__ rows_out,
-                                                float* __restrict__ state_out, CallCounters* nxt) {
+                                                float* __restrict__ state_out, CallCounters* nxt,
+                                                ExportTier et) {
     zero_counters(nxt);
     const int lane = threadIdx.x & 31;
     const uint32_t base = (blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * 32u;
@@ -387,6 +396,10 @@ __global__ void __launch_bounds__(256) k_export(IndexArgs ia, RowArgs ra,
         const uint32_t r = __shfl_sync(0xffffffffu, row, q);
         if (r == ROW_PENDING) continue;
         const float* src = ra.slots + (size_t)(r == ROW_ABSENT ? 0 : r) * ra.stride;
+        if (et.row_loc && r != ROW_ABSENT) {
+            const uint32_t l = et.row_loc[r];
+            src = l < LOC_HOST ? et.cache + (size_t)l * ra.stride : et.host + (size_t)(l & ~LOC_HOST) * ra.stride;
+        }
         if (rows_out) copy_row<V, KV>(src, rows_out + (size_t)(base + q) * ra.d, ra.NV, G, glane, r == ROW_ABSENT);
         if (state_out)
             copy_row<V, KV>(src + ra.dpad, state_out + (size_t)(base + q) * ra.d, ra.NV, G, glane, r == ROW_ABSENT);
@@ -444,11 +457,13 @@ struct MissRun {
                            cudaStream_t st, CallCounters* cur) {
         const unsigned g = capped_grid(t, n * (int64_t)t->geom.G, 256, 8);
         const float span = t->cfg.init_hi - t->cfg.init_lo;
-        MLKV_LAUNCH(t, 0, (k_miss_assign<V, KV>), g, 256, 0, st, index_args(t), row_args(t), keys,
+        RowArgs init_ra = row_args(t);  // new rows live in the host tier when tiered
+        if (t->tiered) init_ra.slots = t->tier.host_dev;
+        MLKV_LAUNCH(t, 0, (k_miss_assign<V, KV>), g, 256, 0, st, index_args(t), init_ra, keys,
                     t->s.miss_pos, t->s.miss_slot, t->s.rank, cur, t->dstate,
                     (unsigned long long)t->cfg.capacity, mode == MissMode::Put ? 0 : 1,
                     (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init);
-        MLKV_LAUNCH(t, 0, (k_miss_finish<V, KV>), g, 256, 0, st, index_args(t), row_args(t),
+        MLKV_LAUNCH(t, 0, (k_miss_finish<V, KV>), g, 256, 0, st, index_args(t), init_ra,
                     t->s.miss_pos, t->s.miss_slot, t->s.row_of_pos, t->s.first_flag,
                     mode == MissMode::Get ? out : nullptr, cur, t->dstate,
                     (unsigned long long)t->cfg.capacity);
@@ -472,8 +487,10 @@ template <int V, int KV>
 struct ExportRun {
     static cudaError_t run(mlkv_table* t, const int64_t* keys, int64_t n, float* rows, float* state,
                            cudaStream_t st, CallCounters* nxt) {
+        ExportTier et{nullptr, nullptr, nullptr};
+        if (t->tiered) et = ExportTier{t->tier.row_loc, t->tier.cache, t->tier.host_dev};
         MLKV_LAUNCH(t, 0, (k_export<V, KV>), grid_for(n, 256), 256, 0, st, index_args(t),
-                    row_args(t), keys, (uint32_t)n, rows, state, nxt);
+                    row_args(t), keys, (uint32_t)n, rows, state, nxt, et);
         return cudaGetLastError();
     }
 };
@@ -482,14 +499,15 @@ struct ExportRun {
 
 cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool insert,
                          bool want_slot, bool report_absent, cudaStream_t st, CallCounters* cur,
-                         CallCounters* nxt) {
+                         CallCounters* nxt, uint32_t* rows_out) {
     uint32_t* slot_of_pos = want_slot ? t->s.slot_of_pos : nullptr;
+    uint32_t* rows = rows_out ? rows_out : t->s.row_of_pos;
     if (insert)
         MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<true>, grid_for(n, 256 * kProbeKeys), 256, 0, st, index_args(t), keys,
-                    (uint32_t)n, t->s.row_of_pos, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0);
+                    (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0);
     else
         MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<false>, grid_for(n, 256 * kProbeKeys), 256, 0, st, index_args(t), keys,
-                    (uint32_t)n, t->s.row_of_pos, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt,
+                    (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt,
                     report_absent ? 1 : 0);
     return cudaGetLastError();
 }

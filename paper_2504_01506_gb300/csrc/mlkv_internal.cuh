@@ -92,6 +92,29 @@ struct Scratch {
     int64_t tile_sums_len;
 };
 
+// Tiered store (hbm_cache_rows > 0): see mlkv_tier.cu.
+struct Tier {
+    float* host_dev;        // host tier [capacity][stride]: pinned host memory mapped for the device
+    size_t host_bytes;      // mapped bytes (whole chunks)
+    size_t host_chunk;      // bytes per allocation handle
+    unsigned long long* host_handles;  // one per chunk (CUmemGenericAllocationHandle)
+    int64_t host_mapped;    // chunks mapped so far
+    float* cache;           // HBM cache [C][stride]
+    uint32_t* row_loc;      // [capacity] cache line, LOC_HOST | host slot, or LOC_CLAIMED
+    uint32_t* line_row;     // [C]
+    uint32_t* line_stamp;   // [C]
+    unsigned long long* ctr;  // free_next, clock, rows fetched, rows written back
+    uint2* fetch;           // [max_batch] (row, host slot) to fetch, main calls
+    uint32_t* n_fetch;
+    uint32_t* la_rows;      // [max_batch] row of each look-ahead key
+    uint2* la_fetch;        // [max_batch]
+    uint32_t* la_n_fetch;
+    cudaStream_t la_stream;
+    cudaEvent_t ev_main, ev_la;
+    uint32_t epoch;         // epoch of the latest call (host side)
+    int la_pending;         // a look-ahead was issued and not yet waited for
+};
+
 struct KernelTimer {
     int kernel_id = 0;
     int n_events = 0;
@@ -106,10 +129,14 @@ struct mlkv_table {
     int device;
     int num_sms;
     mlkv::RowGeom geom;
-    float* slots;
+    float* slots;                // slot array the row kernels use: the table, or the HBM cache
     mlkv::Slot* index;
     unsigned long long index_mask;
-    int sort_bits;               // bits of a row id incl. the absent sentinel
+    int sort_bits;               // bits of the ids being sorted incl. the absent sentinel
+    int bits_rows;               // ... for row ids
+    int bits_lines;              // ... for cache line ids (tiered)
+    int tiered;
+    mlkv::Tier tier;
     mlkv::DevState* dstate;      // device
     uint32_t* status_host;       // mapped pinned word the kernels also write errors to
     uint32_t* status_dev_alias;  // its device alias
@@ -138,6 +165,27 @@ struct ErrSink {
 __device__ __forceinline__ void record_error(const ErrSink& e, uint32_t code) {
     if (atomicCAS(e.dev, 0u, code) == 0u && e.host) *e.host = code;
 }
+
+// row_loc encoding of the tiered store
+constexpr uint32_t LOC_HOST = 0x80000000u;     // | host slot: the row is in the host tier
+constexpr uint32_t LOC_CLAIMED = 0xFFFFFFFFu;  // a fetch of the row is in progress
+
+struct TierArgs {
+    uint32_t* row_loc;
+    uint32_t* line_row;
+    uint32_t* line_stamp;
+    float* cache;
+    float* host;
+    int stride;
+    uint32_t C;
+    unsigned long long* free_next;
+    unsigned long long* clock;
+    unsigned long long* totals;
+    uint32_t epoch;
+    uint32_t keep_from;   // lines stamped >= keep_from are not taken
+    uint32_t strict;      // 1: no fetch; hits must be stamped >= keep_from
+    ErrSink err;
+};
 
 // MurmurHash3 fmix64 finaliser (Appleby): spreads structured keys such as
 // table_id * 2^32 + row over the index.
@@ -235,7 +283,7 @@ enum class MissMode : int { Init = 0, Put = 1, Get = 2 };
 // mlkv_index.cu
 cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool insert,
                          bool want_slot, bool report_absent, cudaStream_t st, CallCounters* cur,
-                         CallCounters* nxt);
+                         CallCounters* nxt, uint32_t* rows_out = nullptr);
 cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out, cudaStream_t st,
                        CallCounters* cur, CallCounters* nxt);
 cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode,
@@ -256,6 +304,13 @@ cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, const uint32_t*
 cudaError_t launch_dedup_out(mlkv_table* t, const int64_t* keys, const uint32_t* spos, int64_t n,
                              int64_t* uniq, int32_t* counts, int64_t* num, cudaStream_t st,
                              CallCounters* cur);
+
+// mlkv_tier.cu
+TierArgs tier_args(mlkv_table* t, uint32_t epoch, uint32_t keep_from, int strict);
+cudaError_t launch_tier_resolve(mlkv_table* t, const TierArgs& ta, uint32_t* row_of_pos, int64_t n,
+                                uint2* fetch, uint32_t* n_fetch, bool remap, cudaStream_t st);
+cudaError_t launch_tier_init(mlkv_table* t, cudaStream_t st);
+cudaError_t launch_gather_lines(mlkv_table* t, const uint32_t* rows, int64_t n, float* out, cudaStream_t st);
 
 // mlkv_apply.cu
 int64_t long_runs_bound(int64_t max_batch);   // runs longer than MLKV_SEQ_SEGMENT_MAX, worst case

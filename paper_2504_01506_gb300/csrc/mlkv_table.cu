@@ -1,11 +1,15 @@
 // C ABI of the store (declared in include/mlkv_gpu.h): argument checks, the
 // table's memory, the order of kernels of each call, status and timing.
+#include <algorithm>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
 #include <new>
 #include <unordered_map>
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
 
 #include "mlkv_internal.cuh"
 
@@ -34,6 +38,113 @@ int cuda_error(mlkv_table* t, cudaError_t e, const char* where) {
     } while (0)
 
 int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+// The host tier is pinned host memory from the driver's virtual-memory API
+// (cuMemCreate on the host NUMA node nearest the GPU), mapped for the device
+// alone.  The GPU then reaches it through its own page tables, in 2 MB pages.
+// Host memory that the OS manages (mmap + cudaHostRegister) is reached through
+// the CPU's page tables instead, which the OS keeps rewriting (huge pages
+// split, NUMA scans); random rows over tens of GB of it moved an order of
+// magnitude slower.  The CPU never touches the tier: rows are initialised,
+// fetched, written back and exported by kernels.  The entry points come from
+// the runtime, so the library does not link the driver library itself.
+struct VmmApi {
+    PFN_cuMemCreate_v10020 create = nullptr;
+    PFN_cuMemRelease_v10020 release = nullptr;
+    PFN_cuMemAddressReserve_v10020 reserve = nullptr;
+    PFN_cuMemAddressFree_v10020 addr_free = nullptr;
+    PFN_cuMemMap_v10020 map = nullptr;
+    PFN_cuMemUnmap_v10020 unmap = nullptr;
+    PFN_cuMemSetAccess_v10020 set_access = nullptr;
+    PFN_cuMemGetAllocationGranularity_v10020 granularity = nullptr;
+    bool ok = false;
+};
+
+const VmmApi& vmm_api() {
+    static const VmmApi api = [] {
+        VmmApi a;
+        auto get = [](const char* name, void** fn) {
+            cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+            return cudaGetDriverEntryPointByVersion(name, fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+                   q == cudaDriverEntryPointSuccess && *fn;
+        };
+        a.ok = get("cuMemCreate", (void**)&a.create) && get("cuMemRelease", (void**)&a.release) &&
+               get("cuMemAddressReserve", (void**)&a.reserve) && get("cuMemAddressFree", (void**)&a.addr_free) &&
+               get("cuMemMap", (void**)&a.map) && get("cuMemUnmap", (void**)&a.unmap) &&
+               get("cuMemSetAccess", (void**)&a.set_access) &&
+               get("cuMemGetAllocationGranularity", (void**)&a.granularity);
+        return a;
+    }();
+    return api;
+}
+
+void host_tier_free(Tier& tr) {
+    const VmmApi& v = vmm_api();
+    if (v.ok && tr.host_dev) {
+        const CUdeviceptr va = (CUdeviceptr)tr.host_dev;
+        for (int64_t i = 0; i < tr.host_mapped; ++i) {
+            v.unmap(va + (size_t)i * tr.host_chunk, tr.host_chunk);
+            v.release((CUmemGenericAllocationHandle)tr.host_handles[i]);
+        }
+        v.addr_free(va, tr.host_bytes);
+    }
+    delete[] tr.host_handles;
+    tr.host_handles = nullptr;
+    tr.host_dev = nullptr;
+    tr.host_mapped = 0;
+}
+
+// Reserves, creates and maps `bytes` (rounded up to whole chunks) of pinned host
+// memory readable and writable by the table's device.
+int host_tier_alloc(mlkv_table* t, size_t bytes) {
+    Tier& tr = t->tier;
+    const VmmApi& v = vmm_api();
+    if (!v.ok) return set_error(t, MLKV_ERR_CUDA, "driver virtual-memory entry points unavailable");
+    int numa = -1;
+    if (cudaDeviceGetAttribute(&numa, cudaDevAttrHostNumaId, t->device) != cudaSuccess) {
+        cudaGetLastError();
+        numa = -1;
+    }
+    CUmemAllocationProp prop;
+    std::memset(&prop, 0, sizeof(prop));
+    prop.type = CU_MEM_ALLOCATION_TYPE_PINNED;
+    prop.location.type = numa >= 0 ? CU_MEM_LOCATION_TYPE_HOST_NUMA : CU_MEM_LOCATION_TYPE_HOST;
+    prop.location.id = numa >= 0 ? numa : 0;
+    size_t gran = 0;
+    if (v.granularity(&gran, &prop, CU_MEM_ALLOC_GRANULARITY_RECOMMENDED) != CUDA_SUCCESS || gran == 0)
+        return set_error(t, MLKV_ERR_CUDA, "host-tier allocation granularity");
+    tr.host_chunk = (size_t)round_up((int64_t)std::min<size_t>(bytes, (size_t)1 << 30), (int64_t)gran);
+    const int64_t n = (int64_t)((bytes + tr.host_chunk - 1) / tr.host_chunk);
+    tr.host_bytes = (size_t)n * tr.host_chunk;
+    tr.host_handles = new (std::nothrow) unsigned long long[n];
+    if (!tr.host_handles) return MLKV_ERR_NOMEM;
+    CUdeviceptr va = 0;
+    if (v.reserve(&va, tr.host_bytes, gran, 0, 0) != CUDA_SUCCESS) {
+        tr.host_bytes = 0;
+        return set_error(t, MLKV_ERR_NOMEM, "host-tier address reservation of %zu bytes", (size_t)n * tr.host_chunk);
+    }
+    tr.host_dev = (float*)va;
+    for (int64_t i = 0; i < n; ++i) {
+        CUmemGenericAllocationHandle h;
+        if (v.create(&h, tr.host_chunk, &prop, 0) != CUDA_SUCCESS)
+            return set_error(t, MLKV_ERR_NOMEM, "host tier: %lld of %lld chunks of %zu bytes", (long long)i,
+                             (long long)n, tr.host_chunk);
+        if (v.map(va + (size_t)i * tr.host_chunk, tr.host_chunk, 0, h, 0) != CUDA_SUCCESS) {
+            v.release(h);
+            return set_error(t, MLKV_ERR_CUDA, "host tier: mapping chunk %lld", (long long)i);
+        }
+        tr.host_handles[i] = (unsigned long long)h;
+        tr.host_mapped = i + 1;
+    }
+    CUmemAccessDesc acc;
+    std::memset(&acc, 0, sizeof(acc));
+    acc.location.type = CU_MEM_LOCATION_TYPE_DEVICE;
+    acc.location.id = t->device;
+    acc.flags = CU_MEM_ACCESS_FLAGS_PROT_READWRITE;
+    if (v.set_access(va, tr.host_bytes, &acc, 1) != CUDA_SUCCESS)
+        return set_error(t, MLKV_ERR_CUDA, "host tier: device access");
+    return MLKV_OK;
+}
 
 int next_pow2_int(int x) {
     int p = 1;
@@ -175,7 +286,25 @@ int mlkv_close(mlkv_table* t) {
         for (int i = 0; i < 2 * KernelTimer::kMax; ++i) cudaEventDestroy(t->timer.ev[i]);
         delete[] t->timer.ev;
     }
-    cudaFree(t->slots);
+    if (t->tiered) {
+        Tier& tr = t->tier;
+        if (tr.la_stream) cudaStreamDestroy(tr.la_stream);
+        if (tr.ev_main) cudaEventDestroy(tr.ev_main);
+        if (tr.ev_la) cudaEventDestroy(tr.ev_la);
+        host_tier_free(tr);
+        cudaFree(tr.cache);
+        cudaFree(tr.row_loc);
+        cudaFree(tr.line_row);
+        cudaFree(tr.line_stamp);
+        cudaFree(tr.ctr);
+        cudaFree(tr.fetch);
+        cudaFree(tr.n_fetch);
+        cudaFree(tr.la_rows);
+        cudaFree(tr.la_fetch);
+        cudaFree(tr.la_n_fetch);
+    } else {
+        cudaFree(t->slots);
+    }
     cudaFree(t->index);
     cudaFree(t->dstate);
     cudaFree(t->arena);
@@ -195,7 +324,10 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     if (c.max_batch < 1 || c.max_batch >= (1ll << 30)) return MLKV_ERR_INVALID;
     if (c.reserved != 0 || (c.flags & ~MLKV_IDENTITY_HASH)) return MLKV_ERR_INVALID;
     if (!(c.init_hi >= c.init_lo)) return MLKV_ERR_INVALID;
-    if (c.staleness_bound != 0 || c.hbm_cache_rows != 0) return MLKV_ERR_UNSUPPORTED;
+    if (c.staleness_bound != 0) return MLKV_ERR_UNSUPPORTED;
+    // a tier needs room for two batches' rows at once (a call and a look-ahead in flight)
+    if (c.hbm_cache_rows < 0 || c.hbm_cache_rows >= (1ll << 31) - 2) return MLKV_ERR_INVALID;
+    if (c.hbm_cache_rows > 0 && c.hbm_cache_rows < 2 * c.max_batch + 64) return MLKV_ERR_INVALID;
 
     mlkv_table* t = new (std::nothrow) mlkv_table();
     if (!t) return MLKV_ERR_NOMEM;
@@ -211,14 +343,46 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     if (!make_geom(c.dim, c.dim % 4 == 0 ? 4 : 1, t->geom)) return fail(MLKV_ERR_INVALID);
 
     const int64_t stride = t->geom.stride;
-    if (cudaMalloc(&t->slots, (size_t)c.capacity * stride * sizeof(float)) != cudaSuccess)
-        return fail(MLKV_ERR_NOMEM);
+    t->tiered = c.hbm_cache_rows > 0;
+    if (!t->tiered) {
+        if (cudaMalloc(&t->slots, (size_t)c.capacity * stride * sizeof(float)) != cudaSuccess)
+            return fail(MLKV_ERR_NOMEM);
+    } else {
+        Tier& tr = t->tier;
+        const int64_t C = c.hbm_cache_rows;
+        int rc = host_tier_alloc(t, (size_t)c.capacity * stride * sizeof(float));
+        if (rc != MLKV_OK) return fail(rc);
+        if (cudaMalloc(&tr.cache, (size_t)C * stride * sizeof(float)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
+        if (cudaMalloc(&tr.row_loc, (size_t)c.capacity * 4) != cudaSuccess ||
+            cudaMalloc(&tr.line_row, (size_t)C * 4) != cudaSuccess ||
+            cudaMalloc(&tr.line_stamp, (size_t)C * 4) != cudaSuccess ||
+            cudaMalloc(&tr.ctr, 4 * sizeof(unsigned long long)) != cudaSuccess ||
+            cudaMalloc(&tr.fetch, (size_t)c.max_batch * sizeof(uint2)) != cudaSuccess ||
+            cudaMalloc(&tr.n_fetch, 4) != cudaSuccess ||
+            cudaMalloc(&tr.la_rows, (size_t)c.max_batch * 4) != cudaSuccess ||
+            cudaMalloc(&tr.la_fetch, (size_t)c.max_batch * sizeof(uint2)) != cudaSuccess ||
+            cudaMalloc(&tr.la_n_fetch, 4) != cudaSuccess)
+            return fail(MLKV_ERR_NOMEM);
+        if (launch_tier_init(t, 0) != cudaSuccess ||  // row r starts in host slot r
+            cudaMemset(tr.line_row, 0xFF, (size_t)C * 4) != cudaSuccess ||
+            cudaMemset(tr.line_stamp, 0xFF, (size_t)C * 4) != cudaSuccess ||  // never handed out
+            cudaMemset(tr.ctr, 0, 4 * sizeof(unsigned long long)) != cudaSuccess)
+            return fail(MLKV_ERR_CUDA);
+        if (cudaStreamCreateWithFlags(&tr.la_stream, cudaStreamNonBlocking) != cudaSuccess ||
+            cudaEventCreateWithFlags(&tr.ev_main, cudaEventDisableTiming) != cudaSuccess ||
+            cudaEventCreateWithFlags(&tr.ev_la, cudaEventDisableTiming) != cudaSuccess)
+            return fail(MLKV_ERR_CUDA);
+        tr.epoch = 1;
+        t->slots = tr.cache;
+    }
     int64_t nslots = 64;
     while (nslots < 2 * c.capacity) nslots <<= 1;
     if (cudaMalloc(&t->index, (size_t)nslots * sizeof(Slot)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
     if (cudaMemset(t->index, 0xFF, (size_t)nslots * sizeof(Slot)) != cudaSuccess) return fail(MLKV_ERR_CUDA);
     t->index_mask = (unsigned long long)(nslots - 1);
-    t->sort_bits = bit_width_u64((uint64_t)c.capacity);
+    t->bits_rows = bit_width_u64((uint64_t)c.capacity);
+    t->bits_lines = t->tiered ? bit_width_u64((uint64_t)c.hbm_cache_rows) : t->bits_rows;
+    t->sort_bits = t->bits_rows;
 
     if (cudaMalloc(&t->dstate, sizeof(DevState)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
     if (cudaMemset(t->dstate, 0, sizeof(DevState)) != cudaSuccess) return fail(MLKV_ERR_CUDA);
@@ -271,11 +435,48 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     return MLKV_OK;
 }
 
+}  // extern "C"
+
+namespace {
+
+// On a tiered table every call first waits for a look-ahead in flight, except
+// an apply_grad, which may run beside it (see mlkv_lookahead).
+int wait_lookahead(mlkv_table* t, cudaStream_t st) {
+    if (t->tiered && t->tier.la_pending) {
+        CK(t, cudaStreamWaitEvent(st, t->tier.ev_la, 0));
+        t->tier.la_pending = 0;
+    }
+    return MLKV_OK;
+}
+
+// Rows of the lookups -> cache lines (fetching the missing rows); the row
+// kernels that follow use the cache as their slot array.
+int tier_map(mlkv_table* t, uint32_t epoch, int strict, int64_t n, cudaStream_t st) {
+    CK(t, launch_tier_resolve(t, tier_args(t, epoch, epoch, strict), t->s.row_of_pos, n, t->tier.fetch,
+                              t->tier.n_fetch, true, st));
+    return MLKV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
 int mlkv_get(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_out, void* stream) {
     int rc = check_call(t, d_keys, n, d_out, true);
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if ((rc = choose_geom(t, d_out, d_out))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
+    if (t->tiered) {
+        if ((rc = wait_lookahead(t, st))) return rc;
+        CallScope cs = begin_call(t, st);
+        const uint32_t e = ++t->tier.epoch;
+        const bool ins = t->cfg.insert_on_miss != 0;
+        CK(t, launch_probe(t, d_keys, n, ins, false, !ins, st, cs.cur, cs.nxt));
+        if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
+        if ((rc = tier_map(t, e, 0, n, st))) return rc;
+        CK(t, launch_gather_lines(t, t->s.row_of_pos, n, d_out, st));
+        return MLKV_OK;
+    }
     CallScope cs = begin_call(t, st);
     CK(t, launch_get(t, d_keys, n, d_out, st, cs.cur, cs.nxt));
     if (t->cfg.insert_on_miss) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Get, d_out, st, cs.cur));
@@ -287,6 +488,7 @@ int mlkv_insert(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream) {
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if ((rc = choose_geom(t, t->slots, t->slots))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
+    if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
     CK(t, launch_probe(t, d_keys, n, true, false, false, st, cs.cur, cs.nxt));
     CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
@@ -298,9 +500,11 @@ int mlkv_put(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_val
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if ((rc = choose_geom(t, d_vals, d_vals))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
+    if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
     CK(t, launch_probe(t, d_keys, n, true, true, false, st, cs.cur, cs.nxt));
     CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Put, nullptr, st, cs.cur));
+    if (t->tiered && (rc = tier_map(t, ++t->tier.epoch, 0, n, st))) return rc;
     CK(t, launch_put_scatter(t, d_vals, n, st));
     return MLKV_OK;
 }
@@ -310,27 +514,52 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if ((rc = choose_geom(t, d_grads, d_grads))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
+    // A tiered apply issued while a look-ahead is in flight runs beside it: it
+    // may only use cache lines of the preceding Get (no insert, no fetch).
+    const bool beside = t->tiered && t->tier.la_pending;
     CallScope cs = begin_call(t, st);
-    const bool ins = t->cfg.insert_on_miss != 0;
+    const bool ins = t->cfg.insert_on_miss != 0 && !beside;
     CK(t, launch_probe(t, d_keys, n, ins, false, !ins, st, cs.cur, cs.nxt));
     if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
+    if (t->tiered) {
+        const uint32_t e = beside ? t->tier.epoch : ++t->tier.epoch;
+        if ((rc = tier_map(t, e, beside ? 1 : 0, n, st))) return rc;
+        t->sort_bits = t->bits_lines;
+    }
     const uint32_t *srow, *spos;
-    CK(t, launch_sort_rows(t, n, st, &srow, &spos));
-    CK(t, launch_segments(t, srow, spos, n, st, cs.cur));
-    CK(t, launch_reduce_apply(t, d_grads, srow, spos, n, st, cs.cur));
+    cudaError_t err = launch_sort_rows(t, n, st, &srow, &spos);
+    if (err == cudaSuccess) err = launch_segments(t, srow, spos, n, st, cs.cur);
+    if (err == cudaSuccess) err = launch_reduce_apply(t, d_grads, srow, spos, n, st, cs.cur);
+    t->sort_bits = t->bits_rows;
+    if (err != cudaSuccess) return cuda_error(t, err, "apply_grad launches");
     return MLKV_OK;
 }
 
 int mlkv_lookahead(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream) {
-    (void)stream;
     int rc = check_call(t, d_keys, n, nullptr, false);
-    return rc < 0 ? MLKV_OK : rc;
+    if (rc) return rc < 0 ? MLKV_OK : rc;
+    if (!t->tiered) return MLKV_OK;  // every row is resident already
+    cudaStream_t st = (cudaStream_t)stream;
+    Tier& tr = t->tier;
+    // the look-ahead starts after everything the caller issued before it, and
+    // runs on the table's side stream; it is stamped with the next call's epoch
+    // and never takes lines stamped by the current one
+    CK(t, cudaEventRecord(tr.ev_main, st));
+    CK(t, cudaStreamWaitEvent(tr.la_stream, tr.ev_main, 0));
+    const uint32_t e = tr.epoch + 1;
+    CK(t, launch_probe(t, d_keys, n, false, false, false, tr.la_stream, nullptr, nullptr, tr.la_rows));
+    CK(t, launch_tier_resolve(t, tier_args(t, e, tr.epoch, 0), tr.la_rows, n, tr.la_fetch, tr.la_n_fetch, false,
+                              tr.la_stream));
+    CK(t, cudaEventRecord(tr.ev_la, tr.la_stream));
+    tr.la_pending = 1;
+    return MLKV_OK;
 }
 
 int mlkv_find(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_rows, void* stream) {
     int rc = check_call(t, d_keys, n, d_rows, true);
     if (rc) return rc < 0 ? MLKV_OK : rc;
     cudaStream_t st = (cudaStream_t)stream;
+    if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
     CK(t, launch_find(t, d_keys, n, d_rows, st, cs.nxt));
     return MLKV_OK;
@@ -342,6 +571,7 @@ int mlkv_export(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_rows, 
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if ((rc = choose_geom(t, d_rows ? d_rows : d_state, d_state ? d_state : d_rows))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
+    if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
     CK(t, launch_export(t, d_keys, n, d_rows, d_state, st, cs.nxt));
     return MLKV_OK;
@@ -360,6 +590,7 @@ int mlkv_dedup(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_uniqu
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if (!d_counts || !d_num_unique) return set_error(t, MLKV_ERR_INVALID, "null pointer");
     cudaStream_t st = (cudaStream_t)stream;
+    if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
     CK(t, launch_probe(t, d_keys, n, false, false, false, st, cs.cur, cs.nxt));
     const uint32_t *srow, *spos;
@@ -407,6 +638,7 @@ int mlkv_apply_grad_host(mlkv_table* t, const int64_t* h_keys, int64_t n, const 
 int mlkv_sync(mlkv_table* t) {
     if (!t) return MLKV_ERR_INVALID;
     CK(t, cudaStreamSynchronize(t->last_stream));
+    if (t->tiered) CK(t, cudaStreamSynchronize(t->tier.la_stream));
     uint32_t st = 0;
     CK(t, cudaMemcpy(&st, &t->dstate->status, sizeof(st), cudaMemcpyDeviceToHost));
     if (st) set_error(t, (int)st, "device status %u (%s)", st, mlkv_status_string((int)st));
@@ -426,6 +658,7 @@ int mlkv_clear_status(mlkv_table* t) {
 int64_t mlkv_size(mlkv_table* t) {
     if (!t) return -1;
     if (cudaStreamSynchronize(t->last_stream) != cudaSuccess) return -1;
+    if (t->tiered && cudaStreamSynchronize(t->tier.la_stream) != cudaSuccess) return -1;
     unsigned long long nr = 0;
     if (cudaMemcpy(&nr, &t->dstate->next_row, sizeof(nr), cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
     return (int64_t)nr;
@@ -440,6 +673,21 @@ int64_t mlkv_last_unique(mlkv_table* t) {
 }
 
 int64_t mlkv_launch_count(mlkv_table* t) { return t ? t->launches : -1; }
+
+int mlkv_tier_stats(mlkv_table* t, int64_t* rows_fetched, int64_t* rows_written_back, int64_t* sweep_lines) {
+    if (!t || !rows_fetched || !rows_written_back || !sweep_lines) return MLKV_ERR_INVALID;
+    *rows_fetched = 0;
+    *rows_written_back = 0;
+    *sweep_lines = 0;
+    if (!t->tiered) return MLKV_OK;
+    CK(t, cudaDeviceSynchronize());
+    unsigned long long c[4];
+    CK(t, cudaMemcpy(c, t->tier.ctr, sizeof(c), cudaMemcpyDeviceToHost));
+    *rows_fetched = (int64_t)c[2];
+    *rows_written_back = (int64_t)c[3];
+    *sweep_lines = (int64_t)c[1];
+    return MLKV_OK;
+}
 
 int mlkv_time_kernel(mlkv_table* t, int32_t kernel_id) {
     if (!t) return MLKV_ERR_INVALID;

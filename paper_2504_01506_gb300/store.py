@@ -158,6 +158,13 @@ class EmbeddingStore:
     def last_unique(self) -> int:
         return int(self.lib.mlkv_last_unique(self.h))
 
+    def tier_stats(self):
+        """(rows fetched host -> HBM, rows written back, cache lines swept for victims)
+        since open; zeros when not tiered."""
+        f, w, c = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
+        self._check(self.lib.mlkv_tier_stats(self.h, ctypes.byref(f), ctypes.byref(w), ctypes.byref(c)))
+        return f.value, w.value, c.value
+
     def launch_count(self) -> int:
         return int(self.lib.mlkv_launch_count(self.h))
 

@@ -23,17 +23,38 @@ STEPS = 4
 N_HOT, N_RANDOM, N_COLD = 24, 400, 16
 
 
+# The tiered store in the benchmark's configuration: the host tier is scaled to
+# the machine's host memory (96M rows x 1 KiB), with a 4M-row HBM cache.
+TIER_ROWS, TIER_CACHE = 96_000_000, 4_000_000
+
+
+def _config(name):
+    cfg = W.ALL[name]()
+    if name == "tiered":
+        cfg.n_keys = TIER_ROWS
+        cfg.hbm_cache_rows = TIER_CACHE
+    return cfg
+
+
 def _store(cfg):
+    import os
+
     torch = torch_cuda()
     from paper_2504_01506_gb300 import EmbeddingStore
 
+    slot = 2 * ((cfg.dim + 7) // 8 * 8) * 4
     free, _ = torch.cuda.mem_get_info()
-    need = cfg.n_keys * 2 * ((cfg.dim + 7) // 8 * 8) * 4 + cfg.n_keys * 64 + (8 << 30)
+    dev_rows = cfg.hbm_cache_rows or cfg.n_keys
+    need = dev_rows * slot + cfg.n_keys * 68 + (8 << 30)
     if free < need:
         pytest.skip(f"needs {need / 2**30:.0f} GiB of device memory")
+    if cfg.hbm_cache_rows:
+        host_free = os.sysconf("SC_AVPHYS_PAGES") * os.sysconf("SC_PAGE_SIZE")
+        if host_free < cfg.n_keys * slot + (24 << 30):
+            pytest.skip("not enough host memory for the host tier")
     return EmbeddingStore(dim=cfg.dim, capacity=cfg.n_keys, max_batch=cfg.batch, lr=cfg.lr, eps=cfg.eps,
                           state_init=cfg.state_init, init_lo=cfg.init_lo, init_hi=cfg.init_hi, seed=cfg.seed,
-                          device="cuda:0")
+                          hbm_cache_rows=cfg.hbm_cache_rows, device="cuda:0")
 
 
 def _oracles(cfg):
@@ -42,10 +63,10 @@ def _oracles(cfg):
     return oracle.Table(cfg.dim, precision=32, **kw), oracle.Table(cfg.dim, precision=64, **kw)
 
 
-@pytest.mark.parametrize("name", ["dlrm", "kg", "gnn"])
+@pytest.mark.parametrize("name", ["dlrm", "kg", "gnn", "tiered"])
 def test_full_size_parity(name):
     torch = torch_cuda()
-    cfg = W.ALL[name]()
+    cfg = _config(name)
     store = _store(cfg)
     dev = torch.device("cuda:0")
     # preload every key in preload order; row ids must be 0..n-1 in that order
@@ -59,12 +80,12 @@ def test_full_size_parity(name):
         want = torch.arange(s, s + k.numel(), device=dev, dtype=torch.int64)
         assert torch.equal(rows, want), f"key -> row mismatch in preload chunk at {s}"
 
-    batches = [cfg.batch_keys(step) for step in range(STEPS)]
+    batches = [cfg.batch_keys(step) for step in range(STEPS + 1)]
     # sample: hottest keys of step 0, random touched keys, untouched keys
     u0, c0 = np.unique(batches[0], return_counts=True)
     hot = u0[np.argsort(-c0)[:N_HOT]]
     rng = np.random.default_rng(7)
-    touched = np.unique(np.concatenate(batches))
+    touched = np.unique(np.concatenate(batches[:STEPS]))
     rand = rng.choice(touched, N_RANDOM, replace=False)
     allk = cfg.preload_keys(0, min(cfg.n_keys, 4_000_000))
     cold = rng.choice(np.setdiff1d(allk, touched)[:100_000], N_COLD, replace=False)
@@ -75,7 +96,7 @@ def test_full_size_parity(name):
     tracker = CountTracker()
 
     out = torch.empty((cfg.batch, cfg.dim), dtype=torch.float32, device=dev)
-    for step, keys in enumerate(batches):
+    for step, keys in enumerate(batches[:STEPS]):
         grads = cfg.grads(step)
         kd = torch.from_numpy(keys).to(dev)
         store.get(kd, out=out)
@@ -90,6 +111,9 @@ def test_full_size_parity(name):
             # Get is a bit-exact copy of the stored rows, on the whole batch
             w_now, _ = store.export(kd)
             assert torch.equal(out.view(torch.int32), w_now.view(torch.int32))
+        if cfg.hbm_cache_rows:  # the next batch is prefetched beside this apply
+            nxt = torch.from_numpy(batches[step + 1]).to(dev)
+            store.lookahead(nxt)
         store.apply_grad(kd, torch.from_numpy(grads).to(dev))
         ref32.apply_grad(keys[sel], grads[sel])
         ref64.apply_grad(keys[sel], grads[sel])
@@ -111,4 +135,7 @@ def test_full_size_parity(name):
     o, g = np.argsort(ou), np.argsort(uniq)
     assert np.array_equal(uniq[g], ou[o]) and np.array_equal(counts[g].astype(np.int64), oc[o])
     assert store.last_unique() == len(ou)
+    if cfg.hbm_cache_rows:
+        fetched, _, _ = store.tier_stats()
+        assert fetched > 0
     store.close()
