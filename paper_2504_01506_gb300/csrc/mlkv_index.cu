@@ -121,25 +121,36 @@ __global__ void __launch_bounds__(256) k_probe(IndexArgs ia, const int64_t* __re
                                                uint32_t* __restrict__ slot_of_pos,
                                                uint32_t* miss_pos, uint32_t* miss_slot,
                                                CallCounters* cur, CallCounters* nxt,
-                                               int report_absent) {
+                                               int report_absent, Memo memo, int memo_use) {
     zero_counters(nxt);
     const uint32_t base = blockIdx.x * (blockDim.x * kProbeKeys) + threadIdx.x;
     unsigned long long k[kProbeKeys];
+    uint32_t known[kProbeKeys];
 #pragma unroll
     for (int j = 0; j < kProbeKeys; ++j) {
         const uint32_t p = base + j * blockDim.x;
         k[j] = p < n ? (unsigned long long)__ldg(keys + p) : 0ull;
+        known[j] = ROW_PENDING;
+        if (memo_use == (int)MemoUse::Read && p < n && (unsigned long long)memo.key[p] == k[j]) known[j] = memo.row[p];
     }
 #pragma unroll
     for (int j = 0; j < kProbeKeys; ++j) {
         const uint32_t p = base + j * blockDim.x;
         if (p >= n) continue;
+        if (known[j] < ROW_ABSENT) {  // the row the last Get found for this key here
+            row_of_pos[p] = known[j];
+            continue;
+        }
         uint32_t slot = 0;
         const uint32_t row = probe_key<INSERT>(ia, k[j], p, slot);
         if (!INSERT && report_absent && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
         row_of_pos[p] = row;
         if (slot_of_pos) slot_of_pos[p] = slot;
         if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
+        if (memo_use == (int)MemoUse::Save) {
+            memo.key[p] = (int64_t)k[j];
+            memo.row[p] = row;
+        }
     }
 }
 
@@ -174,7 +185,7 @@ __global__ void __launch_bounds__(256, MLKV_GET_MIN_BLOCKS) k_get(IndexArgs ia, 
                                              const int64_t* __restrict__ keys, uint32_t n,
                                              float* __restrict__ out, uint32_t* miss_pos,
                                              uint32_t* miss_slot, CallCounters* cur,
-                                             CallCounters* nxt) {
+                                             CallCounters* nxt, Memo memo) {
     using VT = typename Vec<V>::T;
     zero_counters(nxt);
     const int lane = threadIdx.x & 31;
@@ -184,9 +195,12 @@ __global__ void __launch_bounds__(256, MLKV_GET_MIN_BLOCKS) k_get(IndexArgs ia, 
     uint32_t row = ROW_PENDING;  // lanes past the end skip the gather
     if (p < n) {
         uint32_t slot = 0;
-        row = probe_key<INSERT>(ia, (unsigned long long)keys[p], p, slot);
+        const int64_t key = keys[p];
+        row = probe_key<INSERT>(ia, (unsigned long long)key, p, slot);
         if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
         if (!INSERT && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
+        memo.key[p] = key;
+        memo.row[p] = row;
     }
     const int G = ra.G, R = 32 / G, glane = lane & (G - 1), gid = lane / G;
     constexpr int UNR = KV >= MLKV_GET_ROWS_IN_FLIGHT ? 1 : MLKV_GET_ROWS_IN_FLIGHT / KV;
@@ -443,10 +457,12 @@ struct GetRun {
         const unsigned grid = grid_for(n, 256);  // 8 warps x 32 lookups per block
         if (t->cfg.insert_on_miss)
             MLKV_LAUNCH(t, MLKV_K_GET_GATHER, (k_get<V, KV, true>), grid, 256, 0, st, index_args(t),
-                        row_args(t), keys, (uint32_t)n, out, t->s.miss_pos, t->s.miss_slot, cur, nxt);
+                        row_args(t), keys, (uint32_t)n, out, t->s.miss_pos, t->s.miss_slot, cur, nxt,
+                        Memo{t->s.memo_key, t->s.memo_row});
         else
             MLKV_LAUNCH(t, MLKV_K_GET_GATHER, (k_get<V, KV, false>), grid, 256, 0, st, index_args(t),
-                        row_args(t), keys, (uint32_t)n, out, t->s.miss_pos, t->s.miss_slot, cur, nxt);
+                        row_args(t), keys, (uint32_t)n, out, t->s.miss_pos, t->s.miss_slot, cur, nxt,
+                        Memo{t->s.memo_key, t->s.memo_row});
         return cudaGetLastError();
     }
 };
@@ -497,18 +513,20 @@ struct ExportRun {
 
 }  // namespace
 
-cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool insert,
+cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool insert, MemoUse memo,
                          bool want_slot, bool report_absent, cudaStream_t st, CallCounters* cur,
                          CallCounters* nxt, uint32_t* rows_out) {
     uint32_t* slot_of_pos = want_slot ? t->s.slot_of_pos : nullptr;
     uint32_t* rows = rows_out ? rows_out : t->s.row_of_pos;
+    if (want_slot && memo == MemoUse::Read) memo = MemoUse::None;  // the memo holds no slots
+    const Memo m{t->s.memo_key, t->s.memo_row};
     if (insert)
         MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<true>, grid_for(n, 256 * kProbeKeys), 256, 0, st, index_args(t), keys,
-                    (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0);
+                    (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0, m, (int)memo);
     else
         MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<false>, grid_for(n, 256 * kProbeKeys), 256, 0, st, index_args(t), keys,
                     (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt,
-                    report_absent ? 1 : 0);
+                    report_absent ? 1 : 0, m, (int)memo);
     return cudaGetLastError();
 }
 

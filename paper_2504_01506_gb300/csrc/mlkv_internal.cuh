@@ -65,16 +65,15 @@ struct RowGeom {
 struct Scratch {
     uint32_t* row_of_pos;   // [max_batch]
     uint32_t* slot_of_pos;  // [max_batch] (Put)
+    int64_t* memo_key;      // [max_batch] key of each position of the last Get (see Memo)
+    uint32_t* memo_row;     // [max_batch] its row, ROW_PENDING at open
     uint32_t* miss_pos;     // [max_batch]
     uint32_t* miss_slot;    // [max_batch]
     uint32_t* first_flag;   // [max_batch], zero at rest
     uint32_t* rank;         // [max_batch]
     uint32_t* sk[2];        // sort keys (row ids), ping-pong [max_batch]
     uint32_t* sv[2];        // sort values (positions), ping-pong [max_batch]
-    uint32_t* hist;         // [256 * sort tiles] (unused by the Onesweep sort)
-    uint32_t* sort_ghist;   // [kSortMaxPasses * 512] digit starts, + tile tickets and a counter
-    int64_t sort_ghist_bytes;
-    uint32_t* sort_status;  // [kSortMaxPasses][tiles][512] look-back words
+    uint32_t* sort_counts;  // [512][tiles] digit counts of a sort pass, then their output offsets
     uint32_t* tile_sums;    // [scan tiles]
     uint32_t* seg_start;    // [max_batch + 1] run starts in sorted order
     uint32_t* run_row;      // [max_batch] row of each run
@@ -88,7 +87,6 @@ struct Scratch {
     float* partial;         // [max_items][dpad] chunk sums
     int64_t max_long;
     int64_t max_items;
-    int64_t hist_len;
     int64_t tile_sums_len;
 };
 
@@ -276,12 +274,23 @@ struct IndexArgs {
     ErrSink err;
 };
 
+// The (key, row) of every lookup position of the last Get.  A key's row never
+// changes once handed out, so a later probe whose key at position p equals
+// memo key[p] may take memo row[p] (when it is a row: pending and absent
+// lookups are probed again) instead of walking the index; the gradient apply
+// that follows a Get on the same keys then costs no index accesses.
+struct Memo {
+    int64_t* key;
+    uint32_t* row;
+};
+enum class MemoUse { None, Read, Save };
+
 // ---------------------------------------------------------------------------
 // Host-side launchers (each returns cudaGetLastError() of its launches).
 enum class MissMode : int { Init = 0, Put = 1, Get = 2 };
 
 // mlkv_index.cu
-cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool insert,
+cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool insert, MemoUse memo,
                          bool want_slot, bool report_absent, cudaStream_t st, CallCounters* cur,
                          CallCounters* nxt, uint32_t* rows_out = nullptr);
 cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out, cudaStream_t st,

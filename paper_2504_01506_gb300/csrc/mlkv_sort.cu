@@ -6,14 +6,15 @@
 // 40-bit keys), and the sorted order visits rows in memory order.  An absent
 // lookup is given the all-ones digit pattern and sorts last.
 //
-// The sort follows the single-pass ("Onesweep") scheme of Adinets & Merrill
-// (2022): one kernel reads the keys once and counts the digits of every pass;
-// then each pass is one kernel in which a block ranks its 4096-element tile
-// (stable: warp match over rounds of 32 in order), publishes its per-digit
-// count, and finds the count of all earlier tiles by looking back over their
-// published values (decoupled look-back).  Tiles are taken in launch order
-// from an atomic ticket, so every tile looked at is held by a running block;
-// each poll loop is bounded and reports MLKV_ERR_TIMEOUT if it runs out.
+// Each pass is a reduce-then-scan pass over 4096-element tiles: one kernel
+// counts the digits of every tile into a digit-major matrix counts[d][tile];
+// one exclusive scan of that matrix, read in digit-major order, gives every
+// (digit, tile) the output position of its first element; a second kernel
+// ranks each tile's elements stably (warp match over rounds of 32, in order)
+// and scatters them.  No block waits on another, so a pass costs the same when
+// the sort shares the GPU with other kernels.  (A single-pass decoupled
+// look-back sort was slower here: a batch is about one wave of tiles, and
+// the chain of tiles that know their prefix grows one window per round trip.)
 #include "mlkv_internal.cuh"
 
 namespace mlkv {
@@ -123,136 +124,150 @@ __device__ __forceinline__ uint32_t sort_key(uint32_t r, uint32_t sent, bool fir
 }
 
 constexpr int kMaxRadix = 1 << kSortMaxDigitBits;
-constexpr uint32_t kFlagAgg = 1u << 30, kFlagIncl = 2u << 30, kValMask = (1u << 30) - 1;
-constexpr int kPollIters = 1 << 22;
 
-// Look-back words are read and published with device-scope relaxed accesses
-// (value and flag share one 32-bit word, so no further ordering is needed).
-__device__ __forceinline__ uint32_t ld_word(const uint32_t* p) {
-    uint32_t v;
-    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
+#ifndef MLKV_SORT_RANK_BALLOT
+#define MLKV_SORT_RANK_BALLOT 1
+#endif
 
-__device__ __forceinline__ void st_word(uint32_t* p, uint32_t v) {
-    asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
-}
-
-// Digit counts of every pass in one read; the last block to finish turns
-// them into exclusive prefix sums (per pass) and clears the look-back words.
-__global__ void __launch_bounds__(kThreads) k_sort_count(const uint32_t* __restrict__ keys, uint32_t n,
-                                                         uint32_t sent, int passes, int D, uint32_t* ghist,
-                                                         uint32_t* status, uint32_t status_len,
-                                                         uint32_t* done_ctr) {
-    __shared__ uint32_t cnt[kSortMaxPasses][kMaxRadix];
-    __shared__ bool last;
-    const int radix = 1 << D;
-    for (int i = threadIdx.x; i < kSortMaxPasses * kMaxRadix; i += kThreads) (&cnt[0][0])[i] = 0;
-    for (uint32_t i = blockIdx.x * kThreads + threadIdx.x; i < status_len; i += gridDim.x * kThreads) status[i] = 0;
-    __syncthreads();
-    for (uint32_t i = blockIdx.x * kThreads + threadIdx.x; i < n; i += gridDim.x * kThreads) {
-        const uint32_t k = sort_key(keys[i], sent, true);
-        for (int p = 0; p < passes; ++p) atomicAdd(&cnt[p][(k >> (p * D)) & (radix - 1)], 1u);
+// Lanes of the warp whose (valid, digit) equals this lane's: a warp match, or
+// one ballot per digit bit.
+__device__ __forceinline__ uint32_t digit_peers(uint32_t dig, bool valid, int bits) {
+#if MLKV_SORT_RANK_BALLOT
+    const uint32_t vm = __ballot_sync(0xffffffffu, valid);
+    uint32_t peers = valid ? vm : ~vm;
+    for (int b = 0; b < bits; ++b) {
+        const bool one = (dig >> b) & 1u;
+        const uint32_t m = __ballot_sync(0xffffffffu, one);
+        peers &= one ? m : ~m;
     }
-    __syncthreads();
-    for (int p = 0; p < passes; ++p)
-        for (int d = threadIdx.x; d < radix; d += kThreads)
-            if (cnt[p][d]) atomicAdd(&ghist[p * kMaxRadix + d], cnt[p][d]);
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) last = atomicAdd(done_ctr, 1u) == gridDim.x - 1;
-    __syncthreads();
-    if (!last) return;
-    __threadfence();
-    for (int p = 0; p < passes; ++p) {
-        // radix <= 512: two counts per thread, block scan of the pair sums
-        const int d0 = threadIdx.x * 2;
-        const uint32_t a = d0 < radix ? __ldcg(&ghist[p * kMaxRadix + d0]) : 0u;
-        const uint32_t b = d0 + 1 < radix ? __ldcg(&ghist[p * kMaxRadix + d0 + 1]) : 0u;
-        uint32_t total;
-        const uint32_t excl = block_exclusive_scan(a + b, total);
-        if (d0 < radix) ghist[p * kMaxRadix + d0] = excl;
-        if (d0 + 1 < radix) ghist[p * kMaxRadix + d0 + 1] = excl + a;
-        __syncthreads();
-    }
+    return peers;
+#else
+    (void)bits;
+    return __match_any_sync(0xffffffffu, valid ? dig : 0xFFFFFFFFu);
+#endif
 }
 
-__global__ void __launch_bounds__(kThreads) k_sort_scatter(const uint32_t* __restrict__ kin,
-                                                           const uint32_t* __restrict__ vin,
-                                                           uint32_t* __restrict__ kout,
-                                                           uint32_t* __restrict__ vout, uint32_t n,
-                                                           const uint32_t* __restrict__ gstart,
-                                                           uint32_t* status, uint32_t* tile_ctr, int shift,
-                                                           int radix, uint32_t sent, int first, ErrSink err) {
-    __shared__ uint32_t wcnt[kWarps][kMaxRadix];
-    __shared__ uint32_t gbase[kMaxRadix];
-    __shared__ uint32_t tile_s;
+// Digit counts of one tile, written to column `tile` of the digit-major
+// matrix counts[d * ntiles + tile].
+__global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restrict__ kin, uint32_t n,
+                                                        uint32_t* __restrict__ counts, uint32_t ntiles, int shift,
+                                                        int radix, uint32_t sent, int first) {
+    __shared__ uint32_t hist[kMaxRadix];
+    for (int d = threadIdx.x; d < radix; d += kThreads) hist[d] = 0;
+    __syncthreads();
+    const uint32_t base = blockIdx.x * kTile;
+    uint32_t key[kItems];
+#pragma unroll
+    for (int r = 0; r < kItems; ++r) {
+        const uint32_t i = base + r * kThreads + threadIdx.x;
+        key[r] = i < n ? sort_key(kin[i], sent, first) : 0xFFFFFFFFu;
+    }
+#pragma unroll
+    for (int r = 0; r < kItems; ++r)
+        if (base + r * kThreads + threadIdx.x < n) atomicAdd(&hist[(key[r] >> shift) & (radix - 1)], 1u);
+    __syncthreads();
+    for (int d = threadIdx.x; d < radix; d += kThreads) counts[(size_t)d * ntiles + blockIdx.x] = hist[d];
+}
+
+// Stable rank of each element of the tile among equal digits; the tile is
+// then laid out in shared memory in sorted order and written out so that
+// consecutive threads write consecutive addresses of a digit's run (a direct
+// scatter from registers costs one L2 sector per element).  Warp w owns
+// elements w*512 .. w*512+511 of the tile, in rounds of 32 consecutive
+// elements.  An element of digit d goes to offsets[d * ntiles + tile] plus its
+// rank among the tile's elements of digit d.
+__global__ void __launch_bounds__(kThreads, 3) k_sort_scatter(const uint32_t* __restrict__ kin,
+                                                              const uint32_t* __restrict__ vin,
+                                                              uint32_t* __restrict__ kout,
+                                                              uint32_t* __restrict__ vout, uint32_t n,
+                                                              const uint32_t* __restrict__ offsets,
+                                                              uint32_t ntiles, int shift, int radix, uint32_t sent,
+                                                              int first) {
+    // the per-warp digit counts, then (once every position is known) the sorted tile
+    __shared__ uint32_t pool[2 * kTile];
+    static_assert(kWarps * kMaxRadix <= 2 * kTile, "counts fit the tile buffer");
+    uint32_t (*wcnt)[kMaxRadix] = reinterpret_cast<uint32_t (*)[kMaxRadix]>(pool);
+    uint32_t* skey = pool;
+    uint32_t* sval = pool + kTile;
+    __shared__ uint32_t gbase[kMaxRadix];   // output position of the tile's first element of each digit
+    __shared__ uint32_t lbase[kMaxRadix];   // position in the sorted tile of its first element of each digit
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    if (threadIdx.x == 0) tile_s = atomicAdd(tile_ctr, 1u);
     for (int i = threadIdx.x; i < kWarps * kMaxRadix; i += kThreads) (&wcnt[0][0])[i] = 0;
+    for (int d = threadIdx.x; d < radix; d += kThreads) gbase[d] = offsets[(size_t)d * ntiles + blockIdx.x];
     __syncthreads();
-    const uint32_t tile = tile_s;
-    const uint32_t base = tile * kTile + w * (kItems * 32);
+    const uint32_t tile0 = blockIdx.x * kTile;
+    const uint32_t base = tile0 + w * (kItems * 32);
+    const int digit_bits = __ffs(radix) - 1;
     const uint32_t lt = lanemask_lt();
     uint32_t key[kItems], val[kItems], rnk[kItems];
+    // all loads first, so they are in flight together
 #pragma unroll
     for (int r = 0; r < kItems; ++r) {
         const uint32_t i = base + r * 32 + lane;
-        const bool valid = i < n;
-        const uint32_t k = valid ? sort_key(kin[i], sent, first) : 0u;
-        const uint32_t v = valid ? (first ? i : vin[i]) : 0u;
-        const uint32_t dig = (k >> shift) & (radix - 1);
-        const uint32_t peers = __match_any_sync(0xffffffffu, valid ? dig : 0xFFFFFFFFu);
+        key[r] = i < n ? sort_key(kin[i], sent, first) : 0u;
+        val[r] = i < n ? (first ? i : vin[i]) : 0u;
+    }
+#pragma unroll
+    for (int r = 0; r < kItems; ++r) {
+        const bool valid = base + r * 32 + lane < n;
+        const uint32_t dig = (key[r] >> shift) & (radix - 1);
+        const uint32_t peers = digit_peers(dig, valid, digit_bits);
         uint32_t before = 0;
         if (valid) before = wcnt[w][dig];
         __syncwarp();
         if (valid && lane == __ffs(peers) - 1) wcnt[w][dig] = before + __popc(peers);
         __syncwarp();
-        key[r] = k;
-        val[r] = v;
         rnk[r] = valid ? before + __popc(peers & lt) : 0xFFFFFFFFu;
     }
     __syncthreads();
-    // per digit: exclusive prefix over the warps, the tile's count, then the
-    // look-back for the count of all earlier tiles
-    for (int d = threadIdx.x; d < radix; d += kThreads) {
-        uint32_t run = 0;
+    // per digit: exclusive prefix over the warps; per tile: exclusive prefix
+    // over the digits (thread t owns digits t*dpt .. t*dpt+dpt-1, in order)
+    const int dpt = radix > kThreads ? radix / kThreads : 1;
+    uint32_t tot[kMaxRadix / kThreads], mine = 0;
+#pragma unroll
+    for (int j = 0; j < kMaxRadix / kThreads; ++j) {
+        const int d = threadIdx.x * dpt + j;
+        tot[j] = 0;
+        if (j >= dpt || d >= radix) continue;
 #pragma unroll
         for (int ww = 0; ww < kWarps; ++ww) {
             const uint32_t c = wcnt[ww][d];
-            wcnt[ww][d] = run;
-            run += c;
+            wcnt[ww][d] = tot[j];
+            tot[j] += c;
         }
-        uint32_t* my = status + (size_t)tile * radix + d;
-        if (tile == 0) {
-            st_word(my, kFlagIncl | run);
-            gbase[d] = gstart[d];
-            continue;
-        }
-        st_word(my, kFlagAgg | run);
-        uint32_t excl = 0;
-        for (int t = (int)tile - 1; t >= 0; --t) {
-            const uint32_t* q = status + (size_t)t * radix + d;
-            uint32_t v = ld_word(q);
-            for (int it = 0; it < kPollIters && (v & ~kValMask) == 0; ++it) v = ld_word(q);
-            if ((v & ~kValMask) == 0) {
-                record_error(err, MLKV_ERR_TIMEOUT);
-                break;
-            }
-            excl += v & kValMask;
-            if (v & kFlagIncl) break;
-        }
-        st_word(my, kFlagIncl | (excl + run));
-        gbase[d] = gstart[d] + excl;
+        mine += tot[j];
+    }
+    uint32_t all;
+    uint32_t run = block_exclusive_scan(mine, all);
+#pragma unroll
+    for (int j = 0; j < kMaxRadix / kThreads; ++j) {
+        const int d = threadIdx.x * dpt + j;
+        if (j >= dpt || d >= radix) continue;
+        lbase[d] = run;
+        run += tot[j];
     }
     __syncthreads();
 #pragma unroll
     for (int r = 0; r < kItems; ++r) {
         if (rnk[r] == 0xFFFFFFFFu) continue;
         const uint32_t dig = (key[r] >> shift) & (radix - 1);
-        const uint32_t dst = gbase[dig] + wcnt[w][dig] + rnk[r];
-        kout[dst] = key[r];
-        vout[dst] = val[r];
+        rnk[r] += lbase[dig] + wcnt[w][dig];  // position in the sorted tile
+    }
+    __syncthreads();  // the counts are dead: the buffer takes the sorted tile
+#pragma unroll
+    for (int r = 0; r < kItems; ++r) {
+        if (rnk[r] == 0xFFFFFFFFu) continue;
+        skey[rnk[r]] = key[r];
+        sval[rnk[r]] = val[r];
+    }
+    __syncthreads();
+    const uint32_t cnt = n - tile0 < (uint32_t)kTile ? n - tile0 : (uint32_t)kTile;
+    for (uint32_t l = threadIdx.x; l < cnt; l += kThreads) {
+        const uint32_t k = skey[l];
+        const uint32_t dig = (k >> shift) & (radix - 1);
+        const uint32_t dst = gbase[dig] + (l - lbase[dig]);
+        kout[dst] = k;
+        vout[dst] = sval[l];
     }
 }
 
@@ -345,25 +360,18 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
     const int radix = 1 << D;
     const uint32_t sent = (uint32_t)((1ull << bits) - 1);
     const unsigned nt = tiles(n);
-    // digit counts, tile tickets and the completion counter start at zero
-    cudaError_t e = cudaMemsetAsync(t->s.sort_ghist, 0, t->s.sort_ghist_bytes, st);
-    if (e != cudaSuccess) return e;
-    uint32_t* ghist = t->s.sort_ghist;
-    uint32_t* tile_ctr = ghist + kSortMaxPasses * kMaxRadix;
-    uint32_t* done_ctr = tile_ctr + kSortMaxPasses;
-    const uint32_t status_len = (uint32_t)((int64_t)passes * nt * radix);
-    int64_t cg = nt;
-    if (cg > (int64_t)t->num_sms * 4) cg = (int64_t)t->num_sms * 4;
-    MLKV_LAUNCH(t, 0, k_sort_count, (unsigned)cg, kThreads, 0, st, t->s.row_of_pos, (uint32_t)n, sent, passes,
-                D, ghist, t->s.sort_status, status_len, done_ctr);
-    const ErrSink err{&t->dstate->status, t->status_dev_alias};
+    uint32_t* counts = t->s.sort_counts;
     const uint32_t* kin = t->s.row_of_pos;
     const uint32_t* vin = nullptr;
     int out = 0;
     for (int p = 0; p < passes; ++p) {
+        const int first = p == 0;
+        MLKV_LAUNCH(t, 0, k_sort_hist, nt, kThreads, 0, st, kin, (uint32_t)n, counts, nt, p * D,
+                    radix, sent, first);
+        cudaError_t e = launch_exclusive_scan(t, counts, counts, (int64_t)radix * nt, nullptr, nullptr, st);
+        if (e != cudaSuccess) return e;
         MLKV_LAUNCH(t, MLKV_K_SORT_SCATTER, k_sort_scatter, nt, kThreads, 0, st, kin, vin, t->s.sk[out],
-                    t->s.sv[out], (uint32_t)n, ghist + p * kMaxRadix,
-                    t->s.sort_status + (size_t)p * nt * radix, tile_ctr + p, p * D, radix, sent, p == 0, err);
+                    t->s.sv[out], (uint32_t)n, counts, nt, p * D, radix, sent, first);
         kin = t->s.sk[out];
         vin = t->s.sv[out];
         out ^= 1;

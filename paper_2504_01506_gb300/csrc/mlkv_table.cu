@@ -397,22 +397,21 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     Scratch& s = t->s;
     s.max_long = long_runs_bound(B);
     s.max_items = long_items_bound(B);
-    s.hist_len = 256 * tiles_of(B);
-    s.sort_ghist_bytes = (kSortMaxPasses * 512 + kSortMaxPasses + 4) * 4;
-    s.tile_sums_len = (tiles_of(B) > tiles_of(s.hist_len) ? tiles_of(B) : tiles_of(s.hist_len)) + 1;
+    // the scans run over B lookups and over a sort pass's 512 x tiles_of(B) counts
+    s.tile_sums_len = std::max(tiles_of(B), tiles_of(512 * tiles_of(B))) + 1;
     struct Piece {
         void** ptr;
         int64_t bytes;
     };
     Piece pieces[] = {
         {(void**)&s.row_of_pos, B * 4},     {(void**)&s.slot_of_pos, B * 4},
+        {(void**)&s.memo_key, B * 8},       {(void**)&s.memo_row, B * 4},
         {(void**)&s.miss_pos, B * 4},       {(void**)&s.miss_slot, B * 4},
         {(void**)&s.first_flag, B * 4},     {(void**)&s.rank, B * 4},
         {(void**)&s.sk[0], B * 4},          {(void**)&s.sk[1], B * 4},
         {(void**)&s.sv[0], B * 4},          {(void**)&s.sv[1], B * 4},
-        {(void**)&s.hist, s.hist_len * 4},  {(void**)&s.tile_sums, s.tile_sums_len * 4},
-        {(void**)&s.sort_ghist, s.sort_ghist_bytes},
-        {(void**)&s.sort_status, (int64_t)kSortMaxPasses * tiles_of(B) * 512 * 4},
+        {(void**)&s.tile_sums, s.tile_sums_len * 4},
+        {(void**)&s.sort_counts, 512 * tiles_of(B) * 4},
         {(void**)&s.seg_start, (B + 1) * 4},  {(void**)&s.long_s, s.max_long * 4},
         {(void**)&s.long_e, s.max_long * 4},   {(void**)&s.long_row, s.max_long * 4},
         {(void**)&s.long_base, s.max_long * 4}, {(void**)&s.item_s, s.max_items * 4},
@@ -430,6 +429,8 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
         *p.ptr = base;
         base += round_up(p.bytes, 256);
     }
+    // no position has a remembered row yet
+    if (cudaMemset(s.memo_row, 0xFF, (size_t)B * 4) != cudaSuccess) return fail(MLKV_ERR_CUDA);
     if (cudaDeviceSynchronize() != cudaSuccess) return fail(MLKV_ERR_CUDA);
     *out = t;
     return MLKV_OK;
@@ -471,7 +472,7 @@ int mlkv_get(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_out, void
         CallScope cs = begin_call(t, st);
         const uint32_t e = ++t->tier.epoch;
         const bool ins = t->cfg.insert_on_miss != 0;
-        CK(t, launch_probe(t, d_keys, n, ins, false, !ins, st, cs.cur, cs.nxt));
+        CK(t, launch_probe(t, d_keys, n, ins, MemoUse::Save, false, !ins, st, cs.cur, cs.nxt));
         if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
         if ((rc = tier_map(t, e, 0, n, st))) return rc;
         CK(t, launch_gather_lines(t, t->s.row_of_pos, n, d_out, st));
@@ -490,7 +491,7 @@ int mlkv_insert(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream) {
     cudaStream_t st = (cudaStream_t)stream;
     if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
-    CK(t, launch_probe(t, d_keys, n, true, false, false, st, cs.cur, cs.nxt));
+    CK(t, launch_probe(t, d_keys, n, true, MemoUse::None, false, false, st, cs.cur, cs.nxt));
     CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
     return MLKV_OK;
 }
@@ -502,7 +503,7 @@ int mlkv_put(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_val
     cudaStream_t st = (cudaStream_t)stream;
     if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
-    CK(t, launch_probe(t, d_keys, n, true, true, false, st, cs.cur, cs.nxt));
+    CK(t, launch_probe(t, d_keys, n, true, MemoUse::None, true, false, st, cs.cur, cs.nxt));
     CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Put, nullptr, st, cs.cur));
     if (t->tiered && (rc = tier_map(t, ++t->tier.epoch, 0, n, st))) return rc;
     CK(t, launch_put_scatter(t, d_vals, n, st));
@@ -519,7 +520,7 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
     const bool beside = t->tiered && t->tier.la_pending;
     CallScope cs = begin_call(t, st);
     const bool ins = t->cfg.insert_on_miss != 0 && !beside;
-    CK(t, launch_probe(t, d_keys, n, ins, false, !ins, st, cs.cur, cs.nxt));
+    CK(t, launch_probe(t, d_keys, n, ins, MemoUse::Read, false, !ins, st, cs.cur, cs.nxt));
     if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
     if (t->tiered) {
         const uint32_t e = beside ? t->tier.epoch : ++t->tier.epoch;
@@ -547,7 +548,7 @@ int mlkv_lookahead(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream
     CK(t, cudaEventRecord(tr.ev_main, st));
     CK(t, cudaStreamWaitEvent(tr.la_stream, tr.ev_main, 0));
     const uint32_t e = tr.epoch + 1;
-    CK(t, launch_probe(t, d_keys, n, false, false, false, tr.la_stream, nullptr, nullptr, tr.la_rows));
+    CK(t, launch_probe(t, d_keys, n, false, MemoUse::None, false, false, tr.la_stream, nullptr, nullptr, tr.la_rows));
     CK(t, launch_tier_resolve(t, tier_args(t, e, tr.epoch, 0), tr.la_rows, n, tr.la_fetch, tr.la_n_fetch, false,
                               tr.la_stream));
     CK(t, cudaEventRecord(tr.ev_la, tr.la_stream));
@@ -592,7 +593,7 @@ int mlkv_dedup(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_uniqu
     cudaStream_t st = (cudaStream_t)stream;
     if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
-    CK(t, launch_probe(t, d_keys, n, false, false, false, st, cs.cur, cs.nxt));
+    CK(t, launch_probe(t, d_keys, n, false, MemoUse::None, false, false, st, cs.cur, cs.nxt));
     const uint32_t *srow, *spos;
     CK(t, launch_sort_rows(t, n, st, &srow, &spos));
     CK(t, launch_segments(t, srow, spos, n, st, cs.cur));

@@ -21,11 +21,12 @@
 //            out to that same slot;
 //   remap    per lookup: row id -> line id; the Get / apply kernels then work
 //            on the cache as their slot array.
-// The swap is what makes the tier fast.  Random rows over a host tier of tens
-// of GB are bound by the GPU's address translations, not by link bandwidth, and
-// writing the victim to the 1 KiB just read costs no second translation, while
-// a write-back to the victim's own home would.  So every victim is written
-// back, changed or not: a swap takes as long as a plain fetch.
+// With the swap no row has a fixed home and no dirty flags are kept: every
+// victim is written back, changed or not (under Adagrad every cached row has
+// changed).  Writing it to the 1 KiB just read needs no second address
+// translation, which halves the cost on host memory reached through the CPU's
+// page tables; on the driver-allocated tier it costs the same as a write-back
+// elsewhere.
 // Host-tier rows are moved by the GPU itself (zero-copy loads and stores over
 // the mapped host memory): the fetch list never leaves the device, so the
 // copies overlap other work without a host round trip.

@@ -225,3 +225,84 @@ def test_deterministic_runs():
         store.close()
     assert_bits(outs[0][0], outs[1][0], "rows run to run")
     assert_bits(outs[0][1], outs[1][1], "state run to run")
+
+
+def test_apply_after_get_of_other_keys():
+    """The gradient apply takes each position's row from the Get before it when
+    the key there is the same, and probes otherwise: applies on keys that match
+    the Get's only in part, on a shorter batch, on new keys, after a Put, and
+    on keys absent from a store without insert-on-miss, all match the oracle."""
+    torch_cuda()
+    cfg = W.scaled(W.tiny(), 20, 4)  # 5,000 keys, 1,024 lookups, dim 16
+    store, ref32 = make_pair(cfg, capacity=cfg.n_keys + 1_000, max_batch=cfg.n_keys + 1_000)  # room for new keys
+    ref64 = oracle.Table(cfg.dim, lr=cfg.lr, eps=cfg.eps, state_init=cfg.state_init, init_lo=cfg.init_lo,
+                         init_hi=cfg.init_hi, seed=cfg.seed, precision=64)
+    pre = cfg.preload_keys()
+    store.insert(dev(pre))
+    ref32.insert(pre)
+    ref64.insert(pre)
+    rng = np.random.default_rng(3)
+    tracker = CountTracker()
+    touched = set(pre.tolist())
+
+    def apply(keys, grads):
+        store.apply_grad(dev(keys), dev(grads))
+        ref32.apply_grad(keys, grads)
+        ref64.apply_grad(keys, grads)
+        tracker.add(keys)
+        touched.update(np.asarray(keys).tolist())
+
+    def get(keys):
+        out = host(store.get(dev(keys)))
+        want, _, _ = ref32.get(keys)
+        ref64.get(keys)
+        touched.update(np.asarray(keys).tolist())
+        exact = ~tracker.long_mask(keys)
+        assert_bits(out[exact], want[exact], "Get")
+
+    for step in range(6):
+        keys = cfg.batch_keys(step)
+        grads = cfg.grads(step)
+        get(keys)
+        other = keys.copy()
+        swap = rng.random(len(keys)) < 0.5
+        other[swap] = rng.choice(pre, int(swap.sum()))          # present keys at other positions
+        new = rng.random(len(keys)) < 0.05
+        other[new] = (1 << 41) + step * 10_000 + np.arange(int(new.sum()))  # new keys
+        if step % 2:
+            other = other[: len(other) // 2]                     # a shorter batch
+        apply(other, grads[: len(other)])
+        if step == 3:  # a Put between a Get and the apply of its keys
+            vals = (rng.standard_normal((len(keys), cfg.dim)) * 0.01).astype(np.float32)
+            get(keys)
+            store.put(dev(keys), dev(vals))
+            ref32.put(keys, vals)
+            ref64.put(keys, vals)
+            apply(keys, grads)
+    assert store.sync() == 0
+    keys = np.array(sorted(touched), dtype=np.int64)
+    w, G = store.export(dev(keys))
+    assert_table_parity(host(w), host(G), keys, ref32, ref64, tracker, what="memo")
+    assert store.size() == ref32.size()
+
+    # without insert-on-miss: an absent key at a position the Get resolved is
+    # skipped and reported, never given the Get's row
+    store2, ref2 = make_pair(cfg, insert_on_miss=False)
+    ref2_64 = oracle.Table(cfg.dim, lr=cfg.lr, eps=cfg.eps, state_init=cfg.state_init, init_lo=cfg.init_lo,
+                           init_hi=cfg.init_hi, seed=cfg.seed, precision=64, insert_on_miss=False)
+    store2.insert(dev(pre))
+    ref2.insert(pre)
+    ref2_64.insert(pre)
+    keys = cfg.batch_keys(0)
+    store2.get(dev(keys))
+    absent = keys.copy()
+    absent[::7] = (1 << 42) + np.arange(len(absent[::7]))
+    store2.apply_grad(dev(absent), dev(cfg.grads(0)))
+    ref2.apply_grad(absent, cfg.grads(0))
+    ref2_64.apply_grad(absent, cfg.grads(0))
+    assert store2.sync() == 7  # MLKV_ERR_NOT_FOUND
+    store2.clear_status()
+    w2, G2 = store2.export(dev(pre))
+    tracker2 = CountTracker()
+    tracker2.add(absent)
+    assert_table_parity(host(w2), host(G2), pre, ref2, ref2_64, tracker2, what="without insert-on-miss")
