@@ -146,9 +146,9 @@ def batch_stats(keys: np.ndarray, d: int) -> dict:
         "B": B, "U": U, "Bs": Bs, "Us": Us, "Bl": Bl, "Ul": Ul, "items": items,
         # Get: keys + output per lookup; index sector + row per distinct key
         "get_gather": B * (8 + row) + U * (32 + row),
-        # reduce: gradient rows + sorted position per lookup; row and state read
-        # and written once plus the segment bounds and row id per distinct key
-        "reduce_short": Bs * (row + 4) + Us * (4 * row + 12),
+        # short runs: gradient rows + sorted position per lookup; row and state
+        # read and written once plus the run's bounds, row and first position
+        "reduce_short": Bs * (row + 4) + Us * (4 * row + 16),
         # long runs: gradient rows + sorted positions, chunk sums written
         "reduce_long": Bl * (row + 4) + items * row,
         # chunk sums read, row and state read and written once per long run
@@ -172,14 +172,14 @@ def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
         return stats["B"] * 16.0  # per pass: (row id, position) read and written
     if kid == 2:
         return stats["B"] * 12.0 + stats["U"] * 32.0
-    if kid == 6:
-        return stats["B"] * 4.0 + stats["U"] * 4.0
+    if kid == 6:  # each sorted row id read twice, short-run records written
+        return stats["B"] * 8.0 + stats["Us"] * 20.0
     return 0.0
 
 
 KERNEL_NAMES = {1: "k_get (probe + row gather)", 2: "k_probe", 3: "k_sort_scatter",
                 4: "k_short (run sum + Adagrad)", 5: "k_long_sum (chunk sums of long runs)",
-                6: "segments", 7: "k_long_combine (chunk sums + Adagrad)",
+                6: "k_heads (runs found in the sorted ids)", 7: "k_long_combine (chunk sums + Adagrad)",
                 8: "k_tier_fetch (host <-> HBM row swap)"}
 KERNEL_SOURCES = {1: "mlkv_index.cu", 2: "mlkv_index.cu", 3: "mlkv_sort.cu", 4: "mlkv_apply.cu",
                   5: "mlkv_apply.cu", 6: "mlkv_sort.cu", 7: "mlkv_apply.cu", 8: "mlkv_tier.cu"}

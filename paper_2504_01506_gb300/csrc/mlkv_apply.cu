@@ -1,20 +1,22 @@
 // Segmented gradient reduction fused with the sparse Adagrad read-modify-write.
 //
 // After the sort, the lookups of one row form a run (segment) of consecutive
-// sorted positions, in occurrence order (the sort is stable); the segment
-// kernels list the run starts.  For every run the sum g of its gradient rows
-// is formed and one Adagrad step is applied to the row and its state, each
-// read once and written once:
+// sorted positions, in occurrence order (the sort is stable).  For every run
+// the sum g of its gradient rows is formed and one Adagrad step is applied to
+// the row and its state, each read once and written once:
 //     G += g*g ;  w -= lr * g / (sqrt(G) + eps)          (element-wise)
 // This is the per-key Rmw of MLKV Section 3.2 step 8, with the gradient of the
 // embedding map E (Section 2.1) summed over the key's lookups.
 //
-//  k_short        one lane group per run; a run of <= MLKV_SEQ_SEGMENT_MAX
-//                 lookups is summed in occurrence order and its row updated.
-//                 Its positions are loaded lane-parallel and the row and state
-//                 loads are issued next to the gradient loads, so a run costs
-//                 about three dependent memory round trips.  Longer runs are
-//                 listed for the next two kernels.
+//  k_heads        a warp per window of 32 sorted positions finds the runs
+//                 that start there (a row id unlike its left neighbour) and
+//                 their lengths; runs of <= MLKV_SEQ_SEGMENT_MAX lookups are
+//                 appended to a list with one atomic per warp (any order: every
+//                 run is summed on its own), longer ones are measured (a
+//                 warp-wide search for their end) and listed for k_long_*.
+//  k_short        one lane group per listed run: the row, the state and the
+//                 first gradient row are loaded together, the rest summed in
+//                 occurrence order, then the Adagrad step.
 //  k_long_sum     one lane group per chunk of kChunk lookups of a long run
 //                 (Zipf-hot keys reach 10^4-10^5 lookups): chunk sum to scratch.
 //  k_long_combine one block per long run: the chunk sums are split over the
@@ -40,7 +42,7 @@ constexpr int kChunk = 64;
 #define MLKV_REDUCE_MIN_BLOCKS 5
 #endif
 #ifndef MLKV_SHORT_MIN_BLOCKS
-#define MLKV_SHORT_MIN_BLOCKS 5
+#define MLKV_SHORT_MIN_BLOCKS 4
 #endif
 #ifndef MLKV_LONG_ROWS_IN_FLIGHT
 #define MLKV_LONG_ROWS_IN_FLIGHT 4
@@ -60,12 +62,13 @@ struct RowArgs {
 
 struct RunArgs {
     const float* grads;
-    const uint32_t* srow;
-    const uint32_t* spos;
-    const uint32_t* seg_start;
-    const uint32_t* run_row;   // row of each run
-    const uint32_t* run_p0;    // first lookup position of each run
+    const uint32_t* srow;  // sorted row ids; lookups without a row hold `sent` and come last
+    const uint32_t* spos;  // their lookup positions
+    uint32_t n;
+    uint32_t sent;
     CallCounters* cur;
+    uint4* runs;           // [max_batch] short runs: (first sorted position, one past the last, row,
+                           //   first lookup position)
     uint32_t* long_s;      // [max_long] first sorted position
     uint32_t* long_e;      // [max_long] one past the last
     uint32_t* long_row;    // [max_long]
@@ -152,55 +155,296 @@ __device__ __forceinline__ void adagrad_store(const RowArgs& ra, uint32_t row, t
     }
 }
 
-// One lane group per run.  Its start, end, row and first lookup position are
-// independent loads (the segment kernel wrote them side by side); then the
-// row, the state and the first gradient row are loaded together, so a run
-// of one lookup (most of them) costs two dependent round trips.
+// Where the run of `row` that starts at sorted position s ends: the first
+// later position holding another row, or n.  The whole warp searches: 32
+// probes at doubling distances, then rounds of 32 evenly spaced probes, each
+// round narrowing [lo, hi) (srow[lo] == row; hi == n or srow[hi] != row) 32-fold.
+__device__ __forceinline__ uint32_t run_end(const uint32_t* __restrict__ srow, uint32_t n, uint32_t s,
+                                            uint32_t row, int lane) {
+    uint32_t lo = s, hi = n;
+    {
+        const unsigned long long q = (unsigned long long)s + (64ull << lane);
+        const bool eq = q < hi && __ldg(srow + q) == row;
+        const int k = __popc(__ballot_sync(0xffffffffu, eq));  // the equal probes are the first k lanes
+        if (k) lo = (uint32_t)((unsigned long long)s + (64ull << (k - 1)));
+        const unsigned long long qh = (unsigned long long)s + (64ull << k);
+        if (qh < hi) hi = (uint32_t)qh;
+    }
+    while (hi - lo > 1) {
+        const uint32_t step = (hi - lo + 31) / 32;
+        const unsigned long long q = (unsigned long long)lo + (unsigned long long)step * (lane + 1);
+        const bool eq = q < hi && __ldg(srow + q) == row;
+        const uint32_t c = __popc(__ballot_sync(0xffffffffu, eq));
+        const unsigned long long nhi = (unsigned long long)lo + (unsigned long long)step * (c + 1);
+        lo += step * c;
+        if (nhi < hi) hi = (uint32_t)nhi;
+    }
+    return hi;
+}
+
+// The same, for a run of `row` that covers position q0 - 1 (q0 a multiple of
+// 32): first the next 1024 positions in one round (32 consecutive per lane,
+// 16-byte loads), which ends most runs; beyond that, run_end.
+__device__ __forceinline__ uint32_t scan_end(const uint32_t* __restrict__ srow, uint32_t n, uint32_t q0,
+                                             uint32_t row, int lane) {
+    if (q0 >= n) return n;
+    const uint32_t b = q0 + 32u * lane;
+    int first = 32;  // first position of this lane's 32 with another row
+    if (b + 32 <= n) {
+        const uint4* v = reinterpret_cast<const uint4*>(srow + b);
+#pragma unroll
+        for (int k = 7; k >= 0; --k) {
+            const uint4 x = __ldg(v + k);
+            if (x.w != row) first = 4 * k + 3;
+            if (x.z != row) first = 4 * k + 2;
+            if (x.y != row) first = 4 * k + 1;
+            if (x.x != row) first = 4 * k;
+        }
+    } else {
+        for (int k = 31; k >= 0; --k)
+            if (b + k >= n || __ldg(srow + b + k) != row) first = k;
+    }
+    const unsigned m = __ballot_sync(0xffffffffu, first < 32);
+    if (m) {
+        const int l = __ffs(m) - 1;
+        return q0 + 32u * l + (uint32_t)__shfl_sync(0xffffffffu, first, l);
+    }
+    return run_end(srow, n, q0 + 1023u, row, lane);
+}
+
+// Chunks of kChunk lookups of the long runs qs[k] .. qe[k] (k < nq): this
+// lane's run's count, and the exclusive prefix over the lanes (the whole warp).
+__device__ __forceinline__ uint32_t long_chunks(const uint32_t* qs, const uint32_t* qe, int nq, int lane,
+                                                uint32_t& excl) {
+    const uint32_t nit = lane < nq ? (qe[lane] - qs[lane] + kChunk - 1) / kChunk : 0u;
+    uint32_t x = nit;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    excl = x - nit;
+    return __shfl_sync(0xffffffffu, x, 31);  // all the runs' chunks
+}
+
+// Writes the long runs qs[k], qe[k], qr[k] (k < nq: start, end, row) at list
+// entries h0.. and their chunks at items ib0.. for k_long_sum / k_long_combine
+// (the whole warp).
+__device__ __forceinline__ void write_long_runs(const RunArgs& a, const uint32_t* qs, const uint32_t* qe,
+                                                const uint32_t* qr, int nq, uint32_t h0, uint32_t ib0,
+                                                int lane) {
+    uint32_t excl;
+    long_chunks(qs, qe, nq, lane, excl);
+    if (lane < nq) {
+        a.long_s[h0 + lane] = qs[lane];
+        a.long_e[h0 + lane] = qe[lane];
+        a.long_row[h0 + lane] = qr[lane];
+        a.long_base[h0 + lane] = ib0 + excl;
+    }
+    for (int k = 0; k < nq; ++k) {
+        const uint32_t s = qs[k], e = qe[k];
+        const uint32_t m = (e - s + kChunk - 1) / kChunk;
+        const uint32_t ib = ib0 + __shfl_sync(0xffffffffu, excl, k);
+        for (uint32_t c = lane; c < m; c += 32) {
+            a.item_s[ib + c] = s + c * kChunk;
+            a.item_e[ib + c] = min(s + (c + 1) * kChunk, e);
+        }
+    }
+}
+
+// One short run [s, s + len) of `row`, first lookup p0, by one lane group: the
+// row, the state and the first gradient row are loaded together, the rest of
+// the gradient rows are added in occurrence order, then the Adagrad step.
+template <int V, int KV>
+__device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, uint32_t s, uint32_t len,
+                                          uint32_t row, uint32_t p0, int glane, unsigned gmask) {
+    using VT = typename Vec<V>::T;
+    VT w[KV], Gs[KV], acc[KV];
+    load_row_state<V, KV>(ra, row, w, Gs, glane);
+    const VT* g0 = reinterpret_cast<const VT*>(a.grads + (size_t)p0 * ra.d);
+#pragma unroll
+    for (int k = 0; k < KV; ++k) {
+        acc[k] = Vec<V>::zero();
+        const int j = glane + ra.G * k;
+        if (j < ra.NV) Vec<V>::add(acc[k], __ldcs(g0 + j));  // 0 + g: first term, in order
+    }
+    if (len > 1) sum_rows<V, KV>(acc, a.grads, a.spos, s + 1, len - 1, ra.d, ra.NV, ra.G, glane, gmask);
+    adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
+}
+
+// A warp per window of 32 sorted positions (windows dealt out grid-stride).
+// A run starts where a row id differs from its left neighbour; it ends at the
+// next change of value in the window (the next run, or the absent lookups
+// that sort last) or, for the window's last run, where the next window's row
+// ids first differ (past that, it is long and its end is searched for after
+// the windows).  Runs of <= MLKV_SEQ_SEGMENT_MAX lookups are staged in the
+// warp's shared-memory list, long ones in its queue; at the end the block
+// reserves room in the short-run list, the long-run list and the chunk list
+// with one atomic each and the warps copy their runs out.  (Counters that
+// every warp bumps queue up at the end of the kernel.)
+__global__ void __launch_bounds__(256) k_heads(RunArgs a) {
+    constexpr int kList = 128, kQueue = 16;
+    __shared__ uint4 lst[8][kList];  // (start, end, row, first lookup) of short runs
+    __shared__ uint32_t qs[8][kQueue], qr[8][kQueue], qe[8][kQueue];  // long runs: start, row, end (0: unknown)
+    __shared__ uint32_t wsh[8], wlg[8], wit[8];  // per warp: short runs, long runs, chunks; then their bases
+    const uint32_t n = a.n, sent = a.sent;
+    const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+    const uint32_t lt = lanemask_lt();
+    const uint32_t warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const uint32_t nwarps = (gridDim.x * blockDim.x) >> 5;
+    const uint32_t nwin = (n + 31) >> 5;
+    int cnt = 0, nq = 0;  // warp-uniform
+    // a full list or queue goes out at once (only batches far above a few
+    // runs per window and warp get here)
+    auto flush = [&]() {
+        __syncwarp();
+        uint32_t base = 0;
+        if (lane == 0 && cnt) base = atomicAdd(&a.cur->n_short, (uint32_t)cnt);
+        base = __shfl_sync(0xffffffffu, base, 0);
+        for (int k = lane; k < cnt; k += 32) a.runs[base + k] = lst[wib][k];
+        cnt = 0;
+        __syncwarp();
+    };
+    auto measure = [&]() {  // fills in the unknown ends of the queued long runs
+        __syncwarp();
+        for (int k = 0; k < nq; ++k) {
+            // an unknown end lies past the window after the run's first one
+            if (qe[wib][k] == 0u) {
+                const uint32_t e = scan_end(a.srow, n, (qs[wib][k] & ~31u) + 64u, qr[wib][k], lane);
+                __syncwarp();
+                if (lane == 0) qe[wib][k] = e;
+                __syncwarp();
+            }
+        }
+    };
+    auto emit_long = [&](uint32_t h0, uint32_t ib0) {
+        if (nq) write_long_runs(a, qs[wib], qe[wib], qr[wib], nq, h0, ib0, lane);
+        nq = 0;
+        __syncwarp();
+    };
+    // a window's row ids, the next window's, the left neighbour and the
+    // positions, loaded one window ahead
+    auto load = [&](uint32_t w, uint32_t& r, uint32_t& nr, uint32_t& l0, uint32_t& pos) {
+        const uint32_t p = (w << 5) + lane;
+        r = p < n ? __ldg(a.srow + p) : sent;
+        nr = p + 32 < n ? __ldg(a.srow + p + 32) : sent;
+        pos = p < n ? __ldg(a.spos + p) : 0u;
+        l0 = lane == 0 && p > 0 && p <= n ? __ldg(a.srow + p - 1) : ~r;
+    };
+    uint32_t xr = sent, xnr = sent, xl0 = 0u, xpos = 0u;
+    if (warp < nwin) load(warp, xr, xnr, xl0, xpos);
+    for (uint32_t w = warp; w < nwin; w += nwarps) {  // warp-uniform
+        const uint32_t p = (w << 5) + lane;
+        const uint32_t r = xr, nr = xnr, pos = xpos;
+        uint32_t left = __shfl_up_sync(0xffffffffu, r, 1);
+        if (lane == 0) left = xl0;
+        if (w + nwarps < nwin) load(w + nwarps, xr, xnr, xl0, xpos);
+        const unsigned em = __ballot_sync(0xffffffffu, r != left);  // a run, or the absent tail, starts here
+        const bool head = r != sent && r != left;
+        const unsigned hm = __ballot_sync(0xffffffffu, head);
+        if (!hm) continue;
+        const uint32_t lrow = __shfl_sync(0xffffffffu, r, 31 - __clz(hm));
+        const unsigned diff = __ballot_sync(0xffffffffu, nr != lrow);  // for the window's last run
+        const unsigned after = lane == 31 ? 0u : em & (0xFFFFFFFEu << lane);
+        uint32_t len = 0;
+        bool lng = false;
+        if (head) {
+            if (after) len = (uint32_t)(__ffs(after) - 1 - lane);
+            else if (diff) len = 32 - lane + (__ffs(diff) - 1);
+            else lng = true;
+            lng = lng || len > MLKV_SEQ_SEGMENT_MAX;
+        }
+        const unsigned sm = __ballot_sync(0xffffffffu, head && !lng);
+        if (cnt + __popc(sm) > kList) flush();
+        if (head && !lng) lst[wib][cnt + __popc(sm & lt)] = make_uint4(p, p + len, r, pos);
+        cnt += __popc(sm);
+        for (unsigned lm = __ballot_sync(0xffffffffu, head && lng); lm; lm &= lm - 1) {
+            const int i = __ffs(lm) - 1;
+            if (nq == kQueue) {
+                measure();
+                uint32_t excl, h0 = 0, ib0 = 0;
+                const uint32_t items = long_chunks(qs[wib], qe[wib], nq, lane, excl);
+                if (lane == 0) {
+                    h0 = atomicAdd(&a.cur->n_long, (uint32_t)nq);
+                    ib0 = atomicAdd(&a.cur->n_items, items);
+                }
+                h0 = __shfl_sync(0xffffffffu, h0, 0);
+                ib0 = __shfl_sync(0xffffffffu, ib0, 0);
+                if (h0 + nq > a.max_long || ib0 + items > a.max_items) {
+                    if (lane == 0) record_error(a.err, MLKV_ERR_FULL);
+                    nq = 0;
+                } else {
+                    emit_long(h0, ib0);
+                }
+            }
+            const uint32_t row = __shfl_sync(0xffffffffu, r, i);
+            const uint32_t ln = __shfl_sync(0xffffffffu, len, i);  // 0 when the end is past the next window
+            if (lane == 0) {
+                qs[wib][nq] = (w << 5) + i;
+                qr[wib][nq] = row;
+                qe[wib][nq] = ln ? (w << 5) + i + ln : 0u;
+            }
+            ++nq;
+        }
+    }
+    measure();
+    uint32_t excl;
+    const uint32_t items = long_chunks(qs[wib], qe[wib], nq, lane, excl);
+    if (lane == 0) {
+        wsh[wib] = (uint32_t)cnt;
+        wlg[wib] = (uint32_t)nq;
+        wit[wib] = items;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t ts = 0, tl = 0, ti = 0;
+        for (int k = 0; k < 8; ++k) {
+            ts += wsh[k];
+            tl += wlg[k];
+            ti += wit[k];
+        }
+        uint32_t bs = ts ? atomicAdd(&a.cur->n_short, ts) : 0u;
+        uint32_t bl = tl ? atomicAdd(&a.cur->n_long, tl) : 0u;
+        uint32_t bi = ti ? atomicAdd(&a.cur->n_items, ti) : 0u;
+        for (int k = 0; k < 8; ++k) {
+            const uint32_t c0 = wsh[k], c1 = wlg[k], c2 = wit[k];
+            wsh[k] = bs;
+            wlg[k] = bl;
+            wit[k] = bi;
+            bs += c0;
+            bl += c1;
+            bi += c2;
+        }
+    }
+    __syncthreads();
+    for (int k = lane; k < cnt; k += 32) a.runs[wsh[wib] + k] = lst[wib][k];
+    if (wlg[wib] + nq > a.max_long || wit[wib] + items > a.max_items) {
+        if (lane == 0 && nq) record_error(a.err, MLKV_ERR_FULL);
+        return;
+    }
+    emit_long(wlg[wib], wit[wib]);
+}
+
+// One lane group per listed short run.  The run's bounds, row and first lookup
+// position are independent loads, issued one run ahead: while a run's row,
+// state and first gradient row are being loaded, the next run's are already on
+// their way, so a run of one lookup (most of them) costs about one round trip.
+__device__ __forceinline__ uint4 run_meta(const RunArgs& a, uint32_t u, uint32_t U) {
+    return u < U ? __ldg(a.runs + u) : make_uint4(0u, 0u, 0u, 0u);
+}
+
 template <int V, int KV>
 __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra, RunArgs a) {
-    using VT = typename Vec<V>::T;
-    const uint32_t U = a.cur->n_unique, nv = a.cur->n_valid;
+    const uint32_t U = a.cur->n_short;
     const int lane = threadIdx.x & 31, G = ra.G, glane = lane & (G - 1), gid = lane / G;
     const unsigned gmask = group_mask(G, gid);
     const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
     const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
+    uint4 next = run_meta(a, group, U);
     for (uint32_t u = group; u < U; u += ngroups) {  // uniform within the group
-        const uint32_t s = __ldg(a.seg_start + u);
-        const uint32_t e = u + 1 < U ? __ldg(a.seg_start + u + 1) : nv;
-        const uint32_t row = __ldg(a.run_row + u);
-        const uint32_t p0 = __ldg(a.run_p0 + u);
-        const uint32_t len = e - s;
-        if (len > MLKV_SEQ_SEGMENT_MAX) {
-            if (glane == 0) {
-                const uint32_t nit = (len + kChunk - 1) / kChunk;
-                const uint32_t h = atomicAdd(&a.cur->n_long, 1u);
-                const uint32_t ib = atomicAdd(&a.cur->n_items, nit);
-                if (h < a.max_long && ib + nit <= a.max_items) {
-                    a.long_s[h] = s;
-                    a.long_e[h] = e;
-                    a.long_row[h] = row;
-                    a.long_base[h] = ib;
-                    for (uint32_t k = 0; k < nit; ++k) {
-                        a.item_s[ib + k] = s + k * kChunk;
-                        a.item_e[ib + k] = min(s + (k + 1) * kChunk, e);
-                    }
-                } else {
-                    record_error(a.err, MLKV_ERR_FULL);
-                }
-            }
-            continue;
-        }
-        VT w[KV], Gs[KV], acc[KV];
-        load_row_state<V, KV>(ra, row, w, Gs, glane);
-        const VT* g0 = reinterpret_cast<const VT*>(a.grads + (size_t)p0 * ra.d);
-#pragma unroll
-        for (int k = 0; k < KV; ++k) {
-            acc[k] = Vec<V>::zero();
-            const int j = glane + G * k;
-            if (j < ra.NV) Vec<V>::add(acc[k], __ldcs(g0 + j));  // 0 + g: first term, in order
-        }
-        if (len > 1) sum_rows<V, KV>(acc, a.grads, a.spos, s + 1, len - 1, ra.d, ra.NV, G, glane, gmask);
-        adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
+        const uint4 m = next;  // (start, end, row, first lookup)
+        next = run_meta(a, u + ngroups, U);
+        short_run<V, KV>(ra, a, m.x, m.y - m.x, m.z, m.w, glane, gmask);
     }
 }
 
@@ -233,7 +477,7 @@ __global__ void __launch_bounds__(256) k_long_combine(RowArgs ra, RunArgs a, Dev
     using VT = typename Vec<V>::T;
     extern __shared__ float sh[];  // [groups][dpad]
     const uint32_t nl = min(a.cur->n_long, a.max_long);
-    if (blockIdx.x == 0 && threadIdx.x == 0) ds->last_unique = a.cur->n_unique;
+    if (blockIdx.x == 0 && threadIdx.x == 0) ds->last_unique = a.cur->n_short + a.cur->n_long;  // one run per row
     const int G = ra.G, glane = threadIdx.x & (G - 1);
     const int group = threadIdx.x / G;
     const int ngroups = blockDim.x / G;
@@ -292,12 +536,15 @@ __global__ void __launch_bounds__(256) k_long_combine(RowArgs ra, RunArgs a, Dev
 
 template <int V, int KV>
 cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, const uint32_t* spos,
-                       int64_t n, cudaStream_t st, CallCounters* cur) {
-    (void)n;
+                       int64_t n, uint32_t sent, cudaStream_t st, CallCounters* cur) {
     RowArgs ra{t->slots, t->geom.stride, t->geom.dpad, t->geom.NV, t->geom.G, t->geom.d};
-    RunArgs a{grads, srow, spos, t->s.seg_start, t->s.run_row, t->s.run_p0, cur, t->s.long_s, t->s.long_e,
+    RunArgs a{grads, srow, spos, (uint32_t)n, sent, cur, t->s.short_runs, t->s.long_s, t->s.long_e,
               t->s.long_row, t->s.long_base, t->s.item_s, t->s.item_e, t->s.partial, (uint32_t)t->s.max_long,
               (uint32_t)t->s.max_items, ErrSink{&t->dstate->status, t->status_dev_alias}, t->cfg.lr, t->cfg.eps};
+    int64_t gh = (n + 255) / 256;  // a warp per 32 positions, at most 8 blocks per SM
+    if (gh > (int64_t)t->num_sms * 8) gh = (int64_t)t->num_sms * 8;
+    if (gh < 1) gh = 1;
+    MLKV_LAUNCH(t, MLKV_K_SEGMENTS, k_heads, (unsigned)gh, 256, 0, st, a);
     const int gs = persistent_blocks(t, (const void*)k_short<V, KV>, 256);
     MLKV_LAUNCH(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, st, ra, a);
     const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);
@@ -317,21 +564,22 @@ int64_t long_runs_bound(int64_t max_batch) { return max_batch / (MLKV_SEQ_SEGMEN
 int64_t long_items_bound(int64_t max_batch) { return max_batch / kChunk + long_runs_bound(max_batch) + 1; }
 
 cudaError_t launch_reduce_apply(mlkv_table* t, const float* grads, const uint32_t* srow,
-                                const uint32_t* spos, int64_t n, cudaStream_t st, CallCounters* cur) {
+                                const uint32_t* spos, int64_t n, uint32_t sent, cudaStream_t st,
+                                CallCounters* cur) {
     const RowGeom& g = t->geom;
     if (g.V == 4) {
         switch (g.KV) {
-            case 1: return run_reduce<4, 1>(t, grads, srow, spos, n, st, cur);
-            case 2: return run_reduce<4, 2>(t, grads, srow, spos, n, st, cur);
-            case 4: return run_reduce<4, 4>(t, grads, srow, spos, n, st, cur);
-            default: return run_reduce<4, 8>(t, grads, srow, spos, n, st, cur);
+            case 1: return run_reduce<4, 1>(t, grads, srow, spos, n, sent, st, cur);
+            case 2: return run_reduce<4, 2>(t, grads, srow, spos, n, sent, st, cur);
+            case 4: return run_reduce<4, 4>(t, grads, srow, spos, n, sent, st, cur);
+            default: return run_reduce<4, 8>(t, grads, srow, spos, n, sent, st, cur);
         }
     }
     switch (g.KV) {
-        case 1: return run_reduce<1, 1>(t, grads, srow, spos, n, st, cur);
-        case 2: return run_reduce<1, 2>(t, grads, srow, spos, n, st, cur);
-        case 4: return run_reduce<1, 4>(t, grads, srow, spos, n, st, cur);
-        default: return run_reduce<1, 8>(t, grads, srow, spos, n, st, cur);
+        case 1: return run_reduce<1, 1>(t, grads, srow, spos, n, sent, st, cur);
+        case 2: return run_reduce<1, 2>(t, grads, srow, spos, n, sent, st, cur);
+        case 4: return run_reduce<1, 4>(t, grads, srow, spos, n, sent, st, cur);
+        default: return run_reduce<1, 8>(t, grads, srow, spos, n, sent, st, cur);
     }
 }
 

@@ -36,7 +36,8 @@ struct CallCounters {
     uint32_t n_valid;    // lookups with a row
     uint32_t n_long;     // runs longer than MLKV_SEQ_SEGMENT_MAX
     uint32_t n_items;    // chunks of the long runs
-    uint32_t pad[2];
+    uint32_t n_short;    // runs of at most MLKV_SEQ_SEGMENT_MAX lookups
+    uint32_t pad;
 };
 
 struct DevState {
@@ -73,11 +74,14 @@ struct Scratch {
     uint32_t* rank;         // [max_batch]
     uint32_t* sk[2];        // sort keys (row ids), ping-pong [max_batch]
     uint32_t* sv[2];        // sort values (positions), ping-pong [max_batch]
-    uint32_t* sort_counts;  // [512][tiles] digit counts of a sort pass, then their output offsets
+    uint32_t* sort_counts;  // [512][tiles] digit counts of a sort pass
+    uint32_t* sort_offsets; // [tiles][512] output position of each tile's first element of each digit
+    uint32_t* sort_dtot;    // [kSortMaxPasses][512] digit totals of each pass
     uint32_t* tile_sums;    // [scan tiles]
-    uint32_t* seg_start;    // [max_batch + 1] run starts in sorted order
-    uint32_t* run_row;      // [max_batch] row of each run
-    uint32_t* run_p0;       // [max_batch] first lookup position of each run
+    uint32_t* seg_start;    // [max_batch + 1] run starts in sorted order (dedup)
+    uint32_t* run_row;      // [max_batch] row of each run (dedup)
+    uint32_t* run_p0;       // [max_batch] first lookup position of each run (dedup)
+    uint4* short_runs;      // [max_batch] the apply's runs of <= MLKV_SEQ_SEGMENT_MAX lookups
     uint32_t* long_s;       // [max_long] long runs: first sorted position
     uint32_t* long_e;       // [max_long] one past the last
     uint32_t* long_row;     // [max_long]
@@ -325,7 +329,7 @@ cudaError_t launch_gather_lines(mlkv_table* t, const uint32_t* rows, int64_t n, 
 int64_t long_runs_bound(int64_t max_batch);   // runs longer than MLKV_SEQ_SEGMENT_MAX, worst case
 int64_t long_items_bound(int64_t max_batch);  // chunks of those runs, worst case
 cudaError_t launch_reduce_apply(mlkv_table* t, const float* grads, const uint32_t* srow,
-                                const uint32_t* spos, int64_t n, cudaStream_t st,
+                                const uint32_t* spos, int64_t n, uint32_t sent, cudaStream_t st,
                                 CallCounters* cur);
 
 // mlkv_table.cu: launch bookkeeping and optional per-kernel timing.

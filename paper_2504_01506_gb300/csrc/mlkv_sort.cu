@@ -7,11 +7,11 @@
 // lookup is given the all-ones digit pattern and sorts last.
 //
 // Each pass is a reduce-then-scan pass over 4096-element tiles: one kernel
-// counts the digits of every tile into a digit-major matrix counts[d][tile];
-// one exclusive scan of that matrix, read in digit-major order, gives every
-// (digit, tile) the output position of its first element; a second kernel
-// ranks each tile's elements stably (warp match over rounds of 32, in order)
-// and scatters them.  No block waits on another, so a pass costs the same when
+// counts the digits of every tile (and the pass's digit totals); one kernel
+// gives every (tile, digit) the output position of its first element (the
+// elements of lower digits plus those of the digit in earlier tiles); a third
+// ranks each tile's elements stably (over rounds of 32, in order) and
+// scatters them.  No block waits on another, so a pass costs the same when
 // the sort shares the GPU with other kernels.  (A single-pass decoupled
 // look-back sort was slower here: a batch is about one wave of tiles, and
 // the chain of tiles that know their prefix grows one window per round trip.)
@@ -147,26 +147,94 @@ __device__ __forceinline__ uint32_t digit_peers(uint32_t dig, bool valid, int bi
 #endif
 }
 
-// Digit counts of one tile, written to column `tile` of the digit-major
-// matrix counts[d * ntiles + tile].
+// Digit counts of one tile, written to column `tile` of counts[d][tile], and
+// added to the pass's digit totals dtot[d].  A thread counts 16 consecutive
+// elements and adds a run of equal digits with one atomic: after the first
+// pass a hot key's lookups are consecutive, and 32 lanes adding to one counter
+// would queue.
 __global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restrict__ kin, uint32_t n,
-                                                        uint32_t* __restrict__ counts, uint32_t ntiles, int shift,
-                                                        int radix, uint32_t sent, int first) {
+                                                        uint32_t* __restrict__ counts, uint32_t* __restrict__ dtot,
+                                                        uint32_t ntiles, int shift, int radix, uint32_t sent,
+                                                        int first) {
     __shared__ uint32_t hist[kMaxRadix];
     for (int d = threadIdx.x; d < radix; d += kThreads) hist[d] = 0;
     __syncthreads();
-    const uint32_t base = blockIdx.x * kTile;
+    const uint32_t i0 = blockIdx.x * kTile + threadIdx.x * kItems;
     uint32_t key[kItems];
+    if (i0 + kItems <= n) {  // 16 consecutive keys, 16-byte aligned
+        const uint4* src = reinterpret_cast<const uint4*>(kin + i0);
+#pragma unroll
+        for (int q = 0; q < kItems / 4; ++q) {
+            const uint4 v = __ldg(src + q);
+            key[4 * q] = v.x;
+            key[4 * q + 1] = v.y;
+            key[4 * q + 2] = v.z;
+            key[4 * q + 3] = v.w;
+        }
+    } else {
+#pragma unroll
+        for (int r = 0; r < kItems; ++r) key[r] = i0 + r < n ? kin[i0 + r] : 0u;
+    }
+    uint32_t cur = 0xFFFFFFFFu, cnt = 0;
 #pragma unroll
     for (int r = 0; r < kItems; ++r) {
-        const uint32_t i = base + r * kThreads + threadIdx.x;
-        key[r] = i < n ? sort_key(kin[i], sent, first) : 0xFFFFFFFFu;
+        if (i0 + r >= n) break;
+        const uint32_t dig = (sort_key(key[r], sent, first) >> shift) & (radix - 1);
+        if (dig != cur) {
+            if (cnt) atomicAdd(&hist[cur], cnt);
+            cur = dig;
+            cnt = 0;
+        }
+        ++cnt;
     }
-#pragma unroll
-    for (int r = 0; r < kItems; ++r)
-        if (base + r * kThreads + threadIdx.x < n) atomicAdd(&hist[(key[r] >> shift) & (radix - 1)], 1u);
+    if (cnt) atomicAdd(&hist[cur], cnt);
     __syncthreads();
-    for (int d = threadIdx.x; d < radix; d += kThreads) counts[(size_t)d * ntiles + blockIdx.x] = hist[d];
+    for (int d = threadIdx.x; d < radix; d += kThreads) {
+        const uint32_t c = hist[d];
+        counts[(size_t)d * ntiles + blockIdx.x] = c;
+        if (c) atomicAdd(dtot + d, c);
+    }
+}
+
+// Output position of the first element of every (tile, digit): the elements
+// of all lower digits, plus those of digit d in earlier tiles; written to
+// offsets[tile][d].  A warp per digit: a warp-wide sum of the lower digits'
+// totals, then a scan of the digit's counts over the tiles, 32 tiles a round,
+// with the loads of 8 rounds issued together.
+__global__ void __launch_bounds__(kThreads) k_sort_offsets(const uint32_t* __restrict__ counts,
+                                                           const uint32_t* __restrict__ dtot,
+                                                           uint32_t* __restrict__ offsets, uint32_t ntiles,
+                                                           int radix) {
+    constexpr int kRounds = 8;
+    const int lane = threadIdx.x & 31;
+    const int d = blockIdx.x * kWarps + (threadIdx.x >> 5);
+    if (d >= radix) return;  // warp-uniform
+    uint32_t below = 0;
+    for (int i = lane; i < d; i += 32) below += __ldg(dtot + i);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) below += __shfl_xor_sync(0xffffffffu, below, o);
+    const uint32_t* row = counts + (size_t)d * ntiles;
+    uint32_t run = below;
+    for (uint32_t t0 = 0; t0 < ntiles; t0 += 32 * kRounds) {
+        uint32_t c[kRounds];
+#pragma unroll
+        for (int k = 0; k < kRounds; ++k) {
+            const uint32_t t = t0 + 32 * k + lane;
+            c[k] = t < ntiles ? __ldg(row + t) : 0u;
+        }
+#pragma unroll
+        for (int k = 0; k < kRounds; ++k) {
+            const uint32_t t = t0 + 32 * k + lane;
+            uint32_t x = c[k];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+                if (lane >= o) x += y;
+            }
+            if (t < ntiles) offsets[(size_t)t * radix + d] = run + x - c[k];
+            run += __shfl_sync(0xffffffffu, x, 31);
+        }
+    }
 }
 
 // Stable rank of each element of the tile among equal digits; the tile is
@@ -174,8 +242,8 @@ __global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restri
 // consecutive threads write consecutive addresses of a digit's run (a direct
 // scatter from registers costs one L2 sector per element).  Warp w owns
 // elements w*512 .. w*512+511 of the tile, in rounds of 32 consecutive
-// elements.  An element of digit d goes to offsets[d * ntiles + tile] plus its
-// rank among the tile's elements of digit d.
+// elements.  An element of digit d goes to offsets[tile][d] plus its rank
+// among the tile's elements of digit d.
 __global__ void __launch_bounds__(kThreads, 3) k_sort_scatter(const uint32_t* __restrict__ kin,
                                                               const uint32_t* __restrict__ vin,
                                                               uint32_t* __restrict__ kout,
@@ -193,7 +261,7 @@ __global__ void __launch_bounds__(kThreads, 3) k_sort_scatter(const uint32_t* __
     __shared__ uint32_t lbase[kMaxRadix];   // position in the sorted tile of its first element of each digit
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     for (int i = threadIdx.x; i < kWarps * kMaxRadix; i += kThreads) (&wcnt[0][0])[i] = 0;
-    for (int d = threadIdx.x; d < radix; d += kThreads) gbase[d] = offsets[(size_t)d * ntiles + blockIdx.x];
+    for (int d = threadIdx.x; d < radix; d += kThreads) gbase[d] = offsets[(size_t)blockIdx.x * radix + d];
     __syncthreads();
     const uint32_t tile0 = blockIdx.x * kTile;
     const uint32_t base = tile0 + w * (kItems * 32);
@@ -361,17 +429,22 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
     const uint32_t sent = (uint32_t)((1ull << bits) - 1);
     const unsigned nt = tiles(n);
     uint32_t* counts = t->s.sort_counts;
+    uint32_t* offsets = t->s.sort_offsets;
+    // digit totals of every pass start at zero
+    cudaError_t e = cudaMemsetAsync(t->s.sort_dtot, 0, (size_t)kSortMaxPasses * kMaxRadix * 4, st);
+    if (e != cudaSuccess) return e;
     const uint32_t* kin = t->s.row_of_pos;
     const uint32_t* vin = nullptr;
     int out = 0;
     for (int p = 0; p < passes; ++p) {
         const int first = p == 0;
-        MLKV_LAUNCH(t, 0, k_sort_hist, nt, kThreads, 0, st, kin, (uint32_t)n, counts, nt, p * D,
-                    radix, sent, first);
-        cudaError_t e = launch_exclusive_scan(t, counts, counts, (int64_t)radix * nt, nullptr, nullptr, st);
-        if (e != cudaSuccess) return e;
+        uint32_t* dtot = t->s.sort_dtot + p * kMaxRadix;
+        MLKV_LAUNCH(t, 0, k_sort_hist, nt, kThreads, 0, st, kin, (uint32_t)n, counts, dtot, nt, p * D, radix,
+                    sent, first);
+        MLKV_LAUNCH(t, 0, k_sort_offsets, (unsigned)((radix + kWarps - 1) / kWarps), kThreads, 0, st, counts, dtot,
+                    offsets, nt, radix);
         MLKV_LAUNCH(t, MLKV_K_SORT_SCATTER, k_sort_scatter, nt, kThreads, 0, st, kin, vin, t->s.sk[out],
-                    t->s.sv[out], (uint32_t)n, counts, nt, p * D, radix, sent, first);
+                    t->s.sv[out], (uint32_t)n, offsets, nt, p * D, radix, sent, first);
         kin = t->s.sk[out];
         vin = t->s.sv[out];
         out ^= 1;

@@ -397,8 +397,7 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     Scratch& s = t->s;
     s.max_long = long_runs_bound(B);
     s.max_items = long_items_bound(B);
-    // the scans run over B lookups and over a sort pass's 512 x tiles_of(B) counts
-    s.tile_sums_len = std::max(tiles_of(B), tiles_of(512 * tiles_of(B))) + 1;
+    s.tile_sums_len = tiles_of(B) + 1;
     struct Piece {
         void** ptr;
         int64_t bytes;
@@ -412,10 +411,13 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
         {(void**)&s.sv[0], B * 4},          {(void**)&s.sv[1], B * 4},
         {(void**)&s.tile_sums, s.tile_sums_len * 4},
         {(void**)&s.sort_counts, 512 * tiles_of(B) * 4},
+        {(void**)&s.sort_offsets, 512 * tiles_of(B) * 4},
+        {(void**)&s.sort_dtot, kSortMaxPasses * 512 * 4},
         {(void**)&s.seg_start, (B + 1) * 4},  {(void**)&s.long_s, s.max_long * 4},
         {(void**)&s.long_e, s.max_long * 4},   {(void**)&s.long_row, s.max_long * 4},
         {(void**)&s.long_base, s.max_long * 4}, {(void**)&s.item_s, s.max_items * 4},
         {(void**)&s.item_e, s.max_items * 4},   {(void**)&s.run_row, B * 4},
+        {(void**)&s.short_runs, B * 16},
         {(void**)&s.run_p0, B * 4},
         {(void**)&s.partial, s.max_items * t->geom.dpad * 4},
     };
@@ -528,9 +530,9 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
         t->sort_bits = t->bits_lines;
     }
     const uint32_t *srow, *spos;
+    const uint32_t sent = (uint32_t)((1ull << t->sort_bits) - 1);  // the sort's key of a lookup without a row
     cudaError_t err = launch_sort_rows(t, n, st, &srow, &spos);
-    if (err == cudaSuccess) err = launch_segments(t, srow, spos, n, st, cs.cur);
-    if (err == cudaSuccess) err = launch_reduce_apply(t, d_grads, srow, spos, n, st, cs.cur);
+    if (err == cudaSuccess) err = launch_reduce_apply(t, d_grads, srow, spos, n, sent, st, cs.cur);
     t->sort_bits = t->bits_rows;
     if (err != cudaSuccess) return cuda_error(t, err, "apply_grad launches");
     return MLKV_OK;
