@@ -106,6 +106,16 @@ typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
  * where splitmix64(z) is the output of a SplitMix64 generator (Steele, Lea &
  * Flood 2014) whose state is z.  State starts at state_init. */
 
+/* Streams and graphs.  Every call that takes a stream enqueues its work on
+ * that stream and returns without waiting for it (the *_host calls, sync,
+ * size, last_unique, tier_stats and kernel_time wait).  Calls on one table must
+ * be ordered by the caller (one stream, or events between streams).  On an
+ * HBM-resident table a sequence of calls can be captured into a CUDA graph and
+ * the graph replayed (the same pointers and sizes each replay; the work of
+ * each call is device-driven: counts, misses and runs are found on the GPU).
+ * Capturing a tiered table's calls returns MLKV_ERR_UNSUPPORTED (its
+ * look-ahead runs on the table's own stream). */
+
 /* Creates a table on the current CUDA device.  Allocates rows + state
  * (capacity x 2 x dim fp32, rows padded to 32 bytes), the index (a power of
  * two >= 2 x capacity slots of 16 bytes) and scratch for max_batch.  With

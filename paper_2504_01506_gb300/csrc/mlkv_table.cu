@@ -185,11 +185,26 @@ struct CallScope {
     CallCounters* nxt;
 };
 
+bool capturing(cudaStream_t st) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return cs == cudaStreamCaptureStatusActive;
+}
+
+// A call's counters: one of two copies, taken in turn; each call zeroes the
+// other copy for the next one in its first kernel, so no memset is enqueued.
+// A captured graph replays a fixed sequence of calls, which may be odd in
+// number: there every call zeroes its own copy first.
 CallScope begin_call(mlkv_table* t, cudaStream_t st) {
     const int p = t->parity;
     t->parity ^= 1;
     t->last_stream = st;
-    return CallScope{&t->dstate->cc[p], &t->dstate->cc[p ^ 1]};
+    CallScope cs{&t->dstate->cc[p], &t->dstate->cc[p ^ 1]};
+    if (capturing(st)) cudaMemsetAsync(cs.cur, 0, sizeof(CallCounters), st);
+    return cs;
 }
 
 // Common argument checks.  Returns MLKV_OK, an error, or -1 for "n == 0: done".
@@ -445,6 +460,8 @@ namespace {
 // On a tiered table every call first waits for a look-ahead in flight, except
 // an apply_grad, which may run beside it (see mlkv_lookahead).
 int wait_lookahead(mlkv_table* t, cudaStream_t st) {
+    if (t->tiered && capturing(st))
+        return set_error(t, MLKV_ERR_UNSUPPORTED, "a tiered table's calls cannot be captured into a graph");
     if (t->tiered && t->tier.la_pending) {
         CK(t, cudaStreamWaitEvent(st, t->tier.ev_la, 0));
         t->tier.la_pending = 0;
@@ -519,6 +536,8 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
     cudaStream_t st = (cudaStream_t)stream;
     // A tiered apply issued while a look-ahead is in flight runs beside it: it
     // may only use cache lines of the preceding Get (no insert, no fetch).
+    if (t->tiered && capturing(st))
+        return set_error(t, MLKV_ERR_UNSUPPORTED, "a tiered table's calls cannot be captured into a graph");
     const bool beside = t->tiered && t->tier.la_pending;
     CallScope cs = begin_call(t, st);
     const bool ins = t->cfg.insert_on_miss != 0 && !beside;
@@ -543,6 +562,8 @@ int mlkv_lookahead(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if (!t->tiered) return MLKV_OK;  // every row is resident already
     cudaStream_t st = (cudaStream_t)stream;
+    if (capturing(st))
+        return set_error(t, MLKV_ERR_UNSUPPORTED, "a tiered table's calls cannot be captured into a graph");
     Tier& tr = t->tier;
     // the look-ahead starts after everything the caller issued before it, and
     // runs on the table's side stream; it is stamped with the next call's epoch

@@ -37,6 +37,14 @@ namespace mlkv {
 namespace {
 
 constexpr uint32_t LINE_NONE = 0xFFFFFFFFu;
+
+// Blocks of the fetch kernel (8 warps each; set at build time).  The host link
+// needs a few hundred rows in flight, not the whole GPU: more warps only queue
+// on it, and a small grid leaves the SMs to the apply that runs beside a
+// look-ahead.
+#ifndef MLKV_TIER_FETCH_BLOCKS
+#define MLKV_TIER_FETCH_BLOCKS 38
+#endif
 constexpr int kSweepLimit = 1 << 16;  // bounded clock sweep per group of rows (32 lines a round)
 
 __device__ __forceinline__ uint32_t ld_relaxed_u32(const uint32_t* p) {
@@ -262,7 +270,7 @@ cudaError_t launch_tier_resolve(mlkv_table* t, const TierArgs& ta, uint32_t* row
     if (!ta.strict) {
         // a warp per fetched row; at most one row per lookup
         int64_t fg = (n + 7) / 8;
-        const int64_t cap = (int64_t)t->num_sms * 8;
+        const int64_t cap = MLKV_TIER_FETCH_BLOCKS;
         if (fg > cap) fg = cap;
         if (fg < 1) fg = 1;
         const int kv = (t->geom.stride / 4 + 31) / 32;
