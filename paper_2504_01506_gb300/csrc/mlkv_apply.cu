@@ -45,10 +45,10 @@ constexpr int kChunk = 64;
 #define MLKV_SHORT_MIN_BLOCKS 4
 #endif
 #ifndef MLKV_LONG_ROWS_IN_FLIGHT
-#define MLKV_LONG_ROWS_IN_FLIGHT 4
+#define MLKV_LONG_ROWS_IN_FLIGHT 8
 #endif
 #ifndef MLKV_LONG_MIN_BLOCKS
-#define MLKV_LONG_MIN_BLOCKS 5
+#define MLKV_LONG_MIN_BLOCKS 3
 #endif
 
 struct RowArgs {
@@ -549,11 +549,16 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     MLKV_LAUNCH(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, st, ra, a);
     const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);
     MLKV_LAUNCH(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, st, ra, a);
-    // small blocks, many of them: every long run can be combined at once
-    const int cthreads = 64;
+    // small blocks, many of them: a block combines about one long run (wider
+    // blocks split a run's chunk sums over more lane groups but take several
+    // runs each, which measured slower)
+#ifndef MLKV_COMBINE_THREADS
+#define MLKV_COMBINE_THREADS 64
+#endif
+    const int cthreads = MLKV_COMBINE_THREADS;
     const size_t smem = (size_t)(cthreads / t->geom.G) * t->geom.dpad * sizeof(float);
-    MLKV_LAUNCH(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), t->num_sms * 16, cthreads, smem, st, ra, a,
-                t->dstate);
+    MLKV_LAUNCH(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), t->num_sms * (1024 / cthreads), cthreads, smem,
+                st, ra, a, t->dstate);
     return cudaGetLastError();
 }
 
