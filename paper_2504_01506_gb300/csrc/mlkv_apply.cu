@@ -32,6 +32,9 @@ namespace mlkv {
 namespace {
 
 constexpr int kChunk = 64;
+// Long runs of more than kBigRun chunk sums (the hottest rows) are combined by
+// a second launch with blocks of 1024 threads; the rest by many small blocks.
+constexpr uint32_t kBigRun = 32;
 
 // Tuning (set at build time): gradient rows in flight per lane group, and the
 // minimum resident blocks per SM the register allocation must allow.
@@ -75,6 +78,7 @@ struct RunArgs {
     uint32_t* long_base;   // [max_long] first chunk item
     uint32_t* item_s;      // [max_items] first sorted position of each chunk
     uint32_t* item_e;      // [max_items] one past its last
+    uint32_t* big_runs;    // [max_long] long runs of more than kBigRun chunks
     float* partial;        // [max_items][dpad]
     uint32_t max_long;
     uint32_t max_items;
@@ -240,6 +244,7 @@ __device__ __forceinline__ void write_long_runs(const RunArgs& a, const uint32_t
         a.long_e[h0 + lane] = qe[lane];
         a.long_row[h0 + lane] = qr[lane];
         a.long_base[h0 + lane] = ib0 + excl;
+        if ((qe[lane] - qs[lane] + kChunk - 1) / kChunk > kBigRun) a.big_runs[atomicAdd(&a.cur->n_big, 1u)] = h0 + lane;
     }
     for (int k = 0; k < nq; ++k) {
         const uint32_t s = qs[k], e = qe[k];
@@ -472,16 +477,48 @@ __global__ void __launch_bounds__(256, MLKV_LONG_MIN_BLOCKS) k_long_sum(RowArgs 
     }
 }
 
+
+// acc += chunk sums base + k0 .. base + k1 - 1, in that order, with eight
+// vectors per lane in flight.
 template <int V, int KV>
-__global__ void __launch_bounds__(256) k_long_combine(RowArgs ra, RunArgs a, DevState* ds) {
+__device__ __forceinline__ void sum_partials(typename Vec<V>::T (&acc)[KV], const RowArgs& ra, const float* partial,
+                                             uint32_t base, uint32_t k0, uint32_t k1, int glane) {
+    using VT = typename Vec<V>::T;
+    constexpr int UNR = KV >= 8 ? 1 : 8 / KV;
+    for (uint32_t x = k0; x < k1; x += UNR) {
+        VT g[UNR][KV];
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+            const VT* src = reinterpret_cast<const VT*>(partial + (size_t)(base + x + u) * ra.dpad);
+#pragma unroll
+            for (int k = 0; k < KV; ++k) {
+                const int j = glane + ra.G * k;
+                if (x + u < k1 && j < ra.NV) g[u][k] = __ldcg(src + j);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < UNR; ++u)
+#pragma unroll
+            for (int k = 0; k < KV; ++k)
+                if (x + u < k1 && glane + ra.G * k < ra.NV) Vec<V>::add(acc[k], g[u][k]);
+    }
+}
+
+// One launch for every long run.  A run of more than kBigRun chunk sums (the
+// hottest rows) takes a whole block: its lane groups split the sums in a fixed
+// way, then group 0 adds the groups' results in order.  Every other long run
+// takes one lane group, which adds its sums in order.  Then the Adagrad step.
+template <int V, int KV>
+__global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, DevState* ds) {
     using VT = typename Vec<V>::T;
     extern __shared__ float sh[];  // [groups][dpad]
-    const uint32_t nl = min(a.cur->n_long, a.max_long);
+    const uint32_t nl = min(a.cur->n_long, a.max_long), nb = a.cur->n_big;
     if (blockIdx.x == 0 && threadIdx.x == 0) ds->last_unique = a.cur->n_short + a.cur->n_long;  // one run per row
     const int G = ra.G, glane = threadIdx.x & (G - 1);
     const int group = threadIdx.x / G;
     const int ngroups = blockDim.x / G;
-    for (uint32_t h = blockIdx.x; h < nl; h += gridDim.x) {  // block-uniform
+    for (uint32_t i = blockIdx.x; i < nb; i += gridDim.x) {  // block-uniform
+        const uint32_t h = a.big_runs[i];
         const uint32_t base = a.long_base[h];
         const uint32_t m = (a.long_e[h] - a.long_s[h] + kChunk - 1) / kChunk;
         const uint32_t per = (m + ngroups - 1) / ngroups;
@@ -489,24 +526,7 @@ __global__ void __launch_bounds__(256) k_long_combine(RowArgs ra, RunArgs a, Dev
         VT acc[KV];
 #pragma unroll
         for (int k = 0; k < KV; ++k) acc[k] = Vec<V>::zero();
-        constexpr int UNR = KV >= 8 ? 1 : 8 / KV;
-        for (uint32_t x = k0; x < k1; x += UNR) {
-            VT g[UNR][KV];
-#pragma unroll
-            for (int u = 0; u < UNR; ++u) {
-                const VT* src = reinterpret_cast<const VT*>(a.partial + (size_t)(base + x + u) * ra.dpad);
-#pragma unroll
-                for (int k = 0; k < KV; ++k) {
-                    const int j = glane + G * k;
-                    if (x + u < k1 && j < ra.NV) g[u][k] = __ldcg(src + j);
-                }
-            }
-#pragma unroll
-            for (int u = 0; u < UNR; ++u)
-#pragma unroll
-                for (int k = 0; k < KV; ++k)
-                    if (x + u < k1 && glane + G * k < ra.NV) Vec<V>::add(acc[k], g[u][k]);
-        }
+        sum_partials<V, KV>(acc, ra, a.partial, base, k0, k1, glane);
         VT* mine = reinterpret_cast<VT*>(sh + (size_t)group * ra.dpad);
 #pragma unroll
         for (int k = 0; k < KV; ++k) {
@@ -532,6 +552,18 @@ __global__ void __launch_bounds__(256) k_long_combine(RowArgs ra, RunArgs a, Dev
         }
         __syncthreads();
     }
+    const uint32_t gg = blockIdx.x * ngroups + group, ngg = gridDim.x * ngroups;
+    for (uint32_t h = gg; h < nl; h += ngg) {  // uniform within the group
+        const uint32_t m = (a.long_e[h] - a.long_s[h] + kChunk - 1) / kChunk;
+        if (m > kBigRun) continue;
+        VT acc[KV], w[KV], Gs[KV];
+#pragma unroll
+        for (int k = 0; k < KV; ++k) acc[k] = Vec<V>::zero();
+        const uint32_t row = a.long_row[h];
+        load_row_state<V, KV>(ra, row, w, Gs, glane);
+        sum_partials<V, KV>(acc, ra, a.partial, a.long_base[h], 0u, m, glane);
+        adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
+    }
 }
 
 template <int V, int KV>
@@ -539,7 +571,8 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
                        int64_t n, uint32_t sent, cudaStream_t st, CallCounters* cur) {
     RowArgs ra{t->slots, t->geom.stride, t->geom.dpad, t->geom.NV, t->geom.G, t->geom.d};
     RunArgs a{grads, srow, spos, (uint32_t)n, sent, cur, t->s.short_runs, t->s.long_s, t->s.long_e,
-              t->s.long_row, t->s.long_base, t->s.item_s, t->s.item_e, t->s.partial, (uint32_t)t->s.max_long,
+              t->s.long_row, t->s.long_base, t->s.item_s, t->s.item_e, t->s.big_runs, t->s.partial,
+              (uint32_t)t->s.max_long,
               (uint32_t)t->s.max_items, ErrSink{&t->dstate->status, t->status_dev_alias}, t->cfg.lr, t->cfg.eps};
     int64_t gh = (n + 255) / 256;  // a warp per 32 positions, at most 8 blocks per SM
     if (gh > (int64_t)t->num_sms * 8) gh = (int64_t)t->num_sms * 8;
@@ -549,16 +582,13 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     MLKV_LAUNCH(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, st, ra, a);
     const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);
     MLKV_LAUNCH(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, st, ra, a);
-    // small blocks, many of them: a block combines about one long run (wider
-    // blocks split a run's chunk sums over more lane groups but take several
-    // runs each, which measured slower)
-#ifndef MLKV_COMBINE_THREADS
-#define MLKV_COMBINE_THREADS 64
-#endif
-    const int cthreads = MLKV_COMBINE_THREADS;
-    const size_t smem = (size_t)(cthreads / t->geom.G) * t->geom.dpad * sizeof(float);
-    MLKV_LAUNCH(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), t->num_sms * (1024 / cthreads), cthreads, smem,
-                st, ra, a, t->dstate);
+    int big = 1024;  // the groups' sums must fit the default 48 KB of shared memory
+    while (big > 64 && (size_t)(big / t->geom.G) * t->geom.dpad * sizeof(float) > 48 * 1024) big /= 2;
+    const size_t smem = (size_t)(big / t->geom.G) * t->geom.dpad * sizeof(float);
+    // one block per SM (a 1024-thread block fills the register file): 4,864
+    // lane groups of 32 for the ordinary long runs, 152 blocks for the big ones
+    MLKV_LAUNCH(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), t->num_sms * (1024 / big), big, smem, st, ra, a,
+                t->dstate);
     return cudaGetLastError();
 }
 

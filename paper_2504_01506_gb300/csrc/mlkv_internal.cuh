@@ -37,7 +37,7 @@ struct CallCounters {
     uint32_t n_long;     // runs longer than MLKV_SEQ_SEGMENT_MAX
     uint32_t n_items;    // chunks of the long runs
     uint32_t n_short;    // runs of at most MLKV_SEQ_SEGMENT_MAX lookups
-    uint32_t pad;
+    uint32_t n_big;      // long runs whose chunk sums are combined by the wide blocks
 };
 
 struct DevState {
@@ -88,6 +88,7 @@ struct Scratch {
     uint32_t* long_base;    // [max_long] first chunk item
     uint32_t* item_s;       // [max_items] first sorted position of each chunk
     uint32_t* item_e;       // [max_items] one past its last
+    uint32_t* big_runs;     // [max_long] long runs with many chunks (combined by wide blocks)
     float* partial;         // [max_items][dpad] chunk sums
     int64_t max_long;
     int64_t max_items;
