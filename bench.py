@@ -215,18 +215,27 @@ def dist_setup(n_gpus: int):
     return None, 0, 0, 1
 
 
-def barrier(dist, torch):
+def barrier(dist, torch, sync_cuda: bool = True):
     if dist is not None:
         dist.barrier()
-    torch.cuda.synchronize()
+    if sync_cuda:
+        torch.cuda.synchronize()
 
 
-def max_over_ranks(dist, torch, x: float) -> float:
+def max_over_ranks(dist, torch, x: float, device: str = "cuda") -> float:
     if dist is None:
         return x
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    t = torch.tensor([x], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_throughput(dist, torch, elapsed_ms: float, units_per_rank: float, device: str = "cuda"):
+    """Whole-job rate of N replicas: all ranks' units over the slowest rank's time.
+    Returns (slowest ms, units/s)."""
+    world = dist.get_world_size() if dist is not None else 1
+    worst = max_over_ranks(dist, torch, elapsed_ms, device)
+    return worst, units_per_rank * world / (worst / 1e3)
 
 
 # --- the oracle arms -------------------------------------------------------------------
@@ -420,8 +429,7 @@ def run_ours(args, cfg):
     launches = launches_per_graph * args.steps if use_graphs else store.launch_count() - launches0
     tier1 = store.tier_stats()
     assert store.sync() == 0, "device status set during the timed region"
-    elapsed_ms = ev0.elapsed_time(ev1)
-    elapsed_ms = max_over_ranks(dist, torch, elapsed_ms)
+    elapsed_ms, value = job_throughput(dist, torch, ev0.elapsed_time(ev1), cfg.batch * args.steps)
     roof_region_ms = elapsed_ms
     if use_graphs:
         # event timings inside a graph are overwritten at every replay: the
@@ -437,8 +445,6 @@ def run_ours(args, cfg):
     dom_ms, dom_n = store.kernel_time()
     store.time_kernel(0)
     assert store.sync() == 0, "device status set during the roofline region"
-    lookups = cfg.batch * args.steps * world
-    value = lookups / (elapsed_ms / 1e3)
     step_bytes = np.mean([s["step"] for s in stats])
     achieved_step = step_bytes * args.steps / (elapsed_ms / 1e3) / 1e9
 

@@ -467,11 +467,18 @@ struct GetRun {
     }
 };
 
+// Blocks per SM of the miss path's kernels (grid-stride loops over the device's
+// miss count; set at build time).  In steady-state training nothing misses and
+// they return at once, at a cost that grows with the blocks launched.
+#ifndef MLKV_MISS_BLOCKS_PER_SM
+#define MLKV_MISS_BLOCKS_PER_SM 8
+#endif
+
 template <int V, int KV>
 struct MissRun {
     static cudaError_t run(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode, float* out,
                            cudaStream_t st, CallCounters* cur) {
-        const unsigned g = capped_grid(t, n * (int64_t)t->geom.G, 256, 8);
+        const unsigned g = capped_grid(t, n * (int64_t)t->geom.G, 256, MLKV_MISS_BLOCKS_PER_SM);
         const float span = t->cfg.init_hi - t->cfg.init_lo;
         RowArgs init_ra = row_args(t);  // new rows live in the host tier when tiered
         if (t->tiered) init_ra.slots = t->tier.host_dev;
@@ -537,7 +544,8 @@ cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out
 
 cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode,
                                   float* out, cudaStream_t st, CallCounters* cur) {
-    MLKV_LAUNCH(t, 0, k_miss_flag, capped_grid(t, n, 256, 8), 256, 0, st, t->index, t->s.miss_pos,
+    MLKV_LAUNCH(t, 0, k_miss_flag, capped_grid(t, n, 256, MLKV_MISS_BLOCKS_PER_SM), 256, 0, st, t->index,
+                t->s.miss_pos,
                 t->s.miss_slot, t->s.first_flag, cur);
     cudaError_t e = launch_exclusive_scan(t, t->s.first_flag, t->s.rank, n, &cur->n_new,
                                           &cur->n_miss, st);
