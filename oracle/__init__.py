@@ -20,6 +20,9 @@ Parity status of each function (what pins it, in ``tests/test_oracle_pins.py``):
     exactly rounded sums with math.fsum).
   * get / put / insert / find / export: hand-built batches with hand-written
     row ids (tests/golden), Get-after-Put and the key-to-row invariants.
+  * keys / import (checkpoints): import-then-export returns what was
+    imported, the later duplicate wins, a missing state keeps the current
+    one, and a table restored from keys + export continues bit-identically.
 """
 import ctypes
 import os
@@ -61,6 +64,10 @@ def load(mutant: int = 0, out_dir: str | None = None) -> ctypes.CDLL:
         getattr(lib, name).argtypes = [vp, vp, i64, vp]
     lib.oracle_insert.restype = i32
     lib.oracle_insert.argtypes = [vp, vp, i64]
+    lib.oracle_import.restype = i32
+    lib.oracle_import.argtypes = [vp, vp, i64, vp, vp]
+    lib.oracle_keys.restype = i64
+    lib.oracle_keys.argtypes = [vp, vp]
     lib.oracle_find.restype = i32
     lib.oracle_find.argtypes = [vp, vp, i64, vp]
     lib.oracle_export.restype = i64
@@ -153,6 +160,17 @@ class Table:
         k = _keys(keys)
         g = _f32(grads, (len(k), self.dim))
         return self.lib.oracle_apply_grad(self.h, _p(k), len(k), _p(g))
+
+    def import_(self, keys, rows, state=None):
+        k = _keys(keys)
+        w = _f32(rows, (len(k), self.dim))
+        G = None if state is None else _f32(state, (len(k), self.dim))
+        return self.lib.oracle_import(self.h, _p(k), len(k), _p(w), None if G is None else _p(G))
+
+    def keys(self) -> np.ndarray:
+        out = np.empty(self.size(), np.int64)
+        self.lib.oracle_keys(self.h, _p(out))
+        return out
 
     def find(self, keys) -> np.ndarray:
         k = _keys(keys)

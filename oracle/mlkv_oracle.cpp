@@ -26,6 +26,10 @@
 //   * a Get (or gradient apply) of an absent key inserts it when
 //     insert_on_miss is set, otherwise the Get writes NaN and reports
 //     ORACLE_NOT_FOUND and the apply skips the key.
+//   * checkpoints (Section 2.2 keeps a store's data by periodic checkpoints):
+//     a checkpoint is every key in row order with its row and state; a
+//     restore upserts them in that order (oracle_keys, oracle_export,
+//     oracle_import), so the restored table has the same row ids.
 //
 // Arithmetic modes.  Rows and state are stored in fp32 (the table's storage
 // type).  precision == 32 evaluates every operation as its own correctly
@@ -193,6 +197,36 @@ int32_t oracle_put(void* h, const int64_t* keys, int64_t n, const float* vals) {
         std::memcpy(t->w.data() + r * d, vals + i * d, sizeof(float) * d);
     }
     return ORACLE_OK;
+}
+
+// Import(keys, rows, state): sequential upsert of the row and, when state is
+// not null, the state of each key (a new key without state gets state_init,
+// a present one keeps its state).  Duplicates: the later occurrence
+// overwrites.  With the keys of a checkpoint in row order, a fresh table gets
+// the checkpoint's row ids.
+int32_t oracle_import(void* h, const int64_t* keys, int64_t n, const float* rows, const float* state) {
+    Table* t = static_cast<Table*>(h);
+    if (n < 0) return ORACLE_ERR_INVALID;
+    const int32_t d = t->dim;
+    for (int64_t i = 0; i < n; ++i) {
+        uint64_t k = (uint64_t)keys[i];
+        int64_t r = t->find(k);
+        if (r < 0) r = t->insert_init(k);
+        std::memcpy(t->w.data() + r * d, rows + i * d, sizeof(float) * d);
+#if ORACLE_MUTANT == 11
+        (void)state;  // planted: the state is not restored
+#else
+        if (state) std::memcpy(t->G.data() + r * d, state + i * d, sizeof(float) * d);
+#endif
+    }
+    return ORACLE_OK;
+}
+
+// Every key in row order (out has oracle_size entries).
+int64_t oracle_keys(const void* h, int64_t* out) {
+    const Table* t = static_cast<const Table*>(h);
+    for (size_t r = 0; r < t->key_of_row.size(); ++r) out[r] = (int64_t)t->key_of_row[r];
+    return (int64_t)t->key_of_row.size();
 }
 
 // Insert-if-absent with the init row (preloading a key set).

@@ -313,4 +313,55 @@ def check_precisions_agree(lib):
     assert np.all(np.abs(Ga - Gb) <= 1e-5 * (1 + np.abs(Gb)))
 
 
+def check_import_semantics(lib):
+    """Import is an upsert of row and state: what was imported comes back out,
+    the later duplicate wins, no state keeps the current one (state_init for a
+    new key), and new keys get the next row ids in order."""
+    d = 5
+    t = _table(lib, d, seed=3, state_init=0.5)
+    t.insert([40, 41])
+    rng = np.random.default_rng(15)
+    rows = rng.standard_normal((4, d)).astype(np.float32)
+    state = np.abs(rng.standard_normal((4, d))).astype(np.float32)
+    assert t.import_([41, 50, 41, 60], rows, state) == oracle.OK
+    w, G = t.export([41, 50, 60])
+    for got, want in ((w[0], rows[2]), (w[1], rows[1]), (w[2], rows[3]),
+                      (G[0], state[2]), (G[1], state[1]), (G[2], state[3])):
+        assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
+    assert t.keys().tolist() == [40, 41, 50, 60] and t.find([50, 60]).tolist() == [2, 3]
+    _, G40 = t.export([40])
+    t.import_([40, 70], rows[:2])  # no state
+    _, G2 = t.export([40, 70])
+    assert np.array_equal(G2[0], G40[0]) and np.all(G2[1] == np.float32(0.5))
+
+
+def check_checkpoint_resume(lib):
+    """A table restored from its keys (row order), rows and state has the same
+    row ids and continues bit-identically with the original."""
+    d = 4
+    kw = dict(lr=0.1, seed=8, state_init=0.0)
+    a = _table(lib, d, **kw)
+    rng = np.random.default_rng(16)
+    batches = [(rng.integers(0, 300, 200), (rng.standard_normal((200, d)) * 0.1).astype(np.float32))
+               for _ in range(6)]
+    for k, g in batches[:3]:
+        a.get(k)
+        a.apply_grad(k, g)
+    keys = a.keys()
+    w, G = a.export(keys)
+    b = _table(lib, d, **kw)
+    b.import_(keys, w, G)
+    assert np.array_equal(b.find(keys), np.arange(len(keys)))
+    for k, g in batches[3:]:
+        oa, _, _ = a.get(k)
+        ob, _, _ = b.get(k)
+        assert np.array_equal(oa.view(np.uint32), ob.view(np.uint32))
+        a.apply_grad(k, g)
+        b.apply_grad(k, g)
+    wa, Ga = a.export(a.keys())
+    wb, Gb = b.export(a.keys())
+    assert np.array_equal(wa.view(np.uint32), wb.view(np.uint32))
+    assert np.array_equal(Ga.view(np.uint32), Gb.view(np.uint32))
+
+
 ALL_CHECKS = [v for k, v in sorted(globals().items()) if k.startswith("check_")]

@@ -5,14 +5,14 @@ The mistakes are planted in the oracle, on the CPU, at compile time:
 3 wrong sign of the step, 4 one step per occurrence, 5 earlier occurrences
 dropped from the sum, 6 first Put occurrence wins, 7 init drops lo,
 8 dedup reports last positions, 9 state_init ignored, 10 a new key is
-inserted once per occurrence.
+inserted once per occurrence, 11 import drops the state.
 """
 import pytest
 
 import oracle
 import oracle_pins
 
-MUTANTS = list(range(1, 11))
+MUTANTS = list(range(1, 12))
 
 
 @pytest.mark.parametrize("mutant", MUTANTS)
