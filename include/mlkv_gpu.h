@@ -173,6 +173,23 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
  * (dest = the application's cache is a Get into a buffer ahead of use.) */
 int mlkv_lookahead(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream);
 
+/* Checkpoints.  MLKV keeps a store's data by periodic checkpoints (Section
+ * 2.2); a checkpoint here is every key in row order (mlkv_dump_keys) with its
+ * row and state (mlkv_export), and a restore imports them in that order
+ * (mlkv_import), which gives the restored table the same row ids, so training
+ * continues bit-identically.
+ *
+ * mlkv_import: upsert of row and state.  d_rows: fp32 [n][dim]; d_state: fp32
+ * [n][dim] or null (a present key keeps its state, a new key gets
+ * state_init).  Duplicate keys: the last occurrence wins.  New keys get rows
+ * in first-occurrence order, as with insert. */
+int mlkv_import(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_rows, const float* d_state,
+                void* stream);
+
+/* d_keys_out[r] = the key of row r for r < n_rows (n_rows <= mlkv_size(t)):
+ * the table's keys in row order.  d_keys_out: device int64 [n_rows]. */
+int mlkv_dump_keys(mlkv_table* t, int64_t* d_keys_out, int64_t n_rows, void* stream);
+
 /* Key -> row id (int64, -1 when absent); never inserts. */
 int mlkv_find(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_rows, void* stream);
 

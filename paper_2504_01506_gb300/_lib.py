@@ -37,7 +37,7 @@ EXPORTED = [
     "mlkv_lookahead", "mlkv_find", "mlkv_export", "mlkv_dedup", "mlkv_get_host",
     "mlkv_apply_grad_host", "mlkv_sync", "mlkv_clear_status", "mlkv_size", "mlkv_launch_count",
     "mlkv_time_kernel", "mlkv_kernel_time", "mlkv_last_unique", "mlkv_last_error",
-    "mlkv_status_string", "mlkv_dedup_keys_static", "mlkv_tier_stats",
+    "mlkv_status_string", "mlkv_dedup_keys_static", "mlkv_tier_stats", "mlkv_import", "mlkv_dump_keys",
 ]
 STATIC_MAX_KEYS = 65536
 
@@ -95,6 +95,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.mlkv_time_kernel.argtypes = [vp, i32]
     lib.mlkv_kernel_time.argtypes = [vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(i64)]
     lib.mlkv_tier_stats.argtypes = [vp, ctypes.POINTER(i64), ctypes.POINTER(i64), ctypes.POINTER(i64)]
+    lib.mlkv_import.argtypes = [vp, vp, i64, vp, vp, vp]
+    lib.mlkv_dump_keys.argtypes = [vp, vp, i64, vp]
     lib.mlkv_last_unique.argtypes = [vp]
     lib.mlkv_last_unique.restype = i64
     lib.mlkv_last_error.argtypes = [vp]
@@ -104,7 +106,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     for name in ("mlkv_open", "mlkv_close", "mlkv_get", "mlkv_put", "mlkv_insert", "mlkv_apply_grad",
                  "mlkv_lookahead", "mlkv_find", "mlkv_export", "mlkv_dedup", "mlkv_get_host",
                  "mlkv_apply_grad_host", "mlkv_sync", "mlkv_clear_status", "mlkv_time_kernel",
-                 "mlkv_kernel_time", "mlkv_dedup_keys_static", "mlkv_tier_stats"):
+                 "mlkv_kernel_time", "mlkv_dedup_keys_static", "mlkv_tier_stats", "mlkv_import",
+                 "mlkv_dump_keys"):
         getattr(lib, name).restype = i32
     _lib = lib
     return lib

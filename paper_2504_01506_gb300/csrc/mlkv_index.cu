@@ -340,7 +340,8 @@ template <int V, int KV>
 __global__ void __launch_bounds__(256) k_put_scatter(Slot* __restrict__ index, RowArgs ra,
                                                      const uint32_t* __restrict__ row_of_pos,
                                                      const uint32_t* __restrict__ slot_of_pos,
-                                                     const float* __restrict__ vals, uint32_t n) {
+                                                     const float* __restrict__ vals,
+                                                     const float* __restrict__ state, uint32_t n) {
     using VT = typename Vec<V>::T;
     const int lane = threadIdx.x & 31, G = ra.G, R = 32 / G, glane = lane & (G - 1), gid = lane / G;
     const uint32_t warp = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -362,6 +363,15 @@ __global__ void __launch_bounds__(256) k_put_scatter(Slot* __restrict__ index, R
             for (int k = 0; k < KV; ++k) {
                 const int j = glane + G * k;
                 if (j < ra.NV) dst[j] = __ldg(src + j);
+            }
+            if (state) {  // import: the state too
+                const VT* ssrc = reinterpret_cast<const VT*>(state + (size_t)p * ra.d);
+                VT* sdst = reinterpret_cast<VT*>(ra.slots + (size_t)r * ra.stride + ra.dpad);
+#pragma unroll
+                for (int k = 0; k < KV; ++k) {
+                    const int j = glane + G * k;
+                    if (j < ra.NV) sdst[j] = __ldg(ssrc + j);
+                }
             }
             if (glane == 0) index[s].aux = AUX_IDLE;
         }
@@ -496,15 +506,27 @@ struct MissRun {
 
 template <int V, int KV>
 struct PutRun {
-    static cudaError_t run(mlkv_table* t, const float* vals, int64_t n, cudaStream_t st) {
+    static cudaError_t run(mlkv_table* t, const float* vals, const float* state, int64_t n, cudaStream_t st) {
         MLKV_LAUNCH(t, 0, k_put_mark, grid_for(n, 256), 256, 0, st, t->index, t->s.row_of_pos,
                     t->s.slot_of_pos, (uint32_t)n);
         const unsigned g = capped_grid(t, n * (int64_t)t->geom.G, 256, 8);
         MLKV_LAUNCH(t, 0, (k_put_scatter<V, KV>), g, 256, 0, st, t->index, row_args(t),
-                    t->s.row_of_pos, t->s.slot_of_pos, vals, (uint32_t)n);
+                    t->s.row_of_pos, t->s.slot_of_pos, vals, state, (uint32_t)n);
         return cudaGetLastError();
     }
 };
+
+// The key of every row below n_rows, at its row: a checkpoint's keys in row
+// order (rows are dense, handed out in first-occurrence order).
+__global__ void __launch_bounds__(256) k_dump_keys(const Slot* __restrict__ index, unsigned long long nslots,
+                                                   int64_t* __restrict__ out, uint32_t n_rows) {
+    for (unsigned long long s = blockIdx.x * (unsigned long long)blockDim.x + threadIdx.x; s < nslots;
+         s += (unsigned long long)gridDim.x * blockDim.x) {
+        const unsigned long long key = index[s].key;
+        const uint32_t row = index[s].row;
+        if (key != EMPTY_KEY && row < n_rows) out[row] = (int64_t)key;
+    }
+}
 
 template <int V, int KV>
 struct ExportRun {
@@ -553,8 +575,14 @@ cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n,
     return dispatch_row<MissRun>(t->geom, t, keys, n, mode, out, st, cur);
 }
 
-cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, int64_t n, cudaStream_t st) {
-    return dispatch_row<PutRun>(t->geom, t, vals, n, st);
+cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, const float* state, int64_t n, cudaStream_t st) {
+    return dispatch_row<PutRun>(t->geom, t, vals, state, n, st);
+}
+
+cudaError_t launch_dump_keys(mlkv_table* t, int64_t* out, int64_t n_rows, cudaStream_t st) {
+    const unsigned long long nslots = t->index_mask + 1;
+    MLKV_LAUNCH(t, 0, k_dump_keys, (unsigned)t->num_sms * 8, 256, 0, st, t->index, nslots, out, (uint32_t)n_rows);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_find(mlkv_table* t, const int64_t* keys, int64_t n, int64_t* rows,

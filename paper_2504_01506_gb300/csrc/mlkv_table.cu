@@ -516,17 +516,38 @@ int mlkv_insert(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream) {
     return MLKV_OK;
 }
 
-int mlkv_put(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_vals, void* stream) {
+// Put, and import (the state too): upsert, the last occurrence of a key wins.
+static int put_rows(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_vals, const float* d_state,
+                    void* stream) {
     int rc = check_call(t, d_keys, n, d_vals, true);
     if (rc) return rc < 0 ? MLKV_OK : rc;
-    if ((rc = choose_geom(t, d_vals, d_vals))) return rc;
+    if ((rc = choose_geom(t, d_vals, d_state ? d_state : d_vals))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
     if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
     CK(t, launch_probe(t, d_keys, n, true, MemoUse::None, true, false, st, cs.cur, cs.nxt));
     CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Put, nullptr, st, cs.cur));
     if (t->tiered && (rc = tier_map(t, ++t->tier.epoch, 0, n, st))) return rc;
-    CK(t, launch_put_scatter(t, d_vals, n, st));
+    CK(t, launch_put_scatter(t, d_vals, d_state, n, st));
+    return MLKV_OK;
+}
+
+int mlkv_put(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_vals, void* stream) {
+    return put_rows(t, d_keys, n, d_vals, nullptr, stream);
+}
+
+int mlkv_import(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_rows, const float* d_state,
+                void* stream) {
+    return put_rows(t, d_keys, n, d_rows, d_state, stream);
+}
+
+int mlkv_dump_keys(mlkv_table* t, int64_t* d_keys_out, int64_t n_rows, void* stream) {
+    if (!t || n_rows < 0 || (n_rows > 0 && !d_keys_out)) return MLKV_ERR_INVALID;
+    if (n_rows == 0) return MLKV_OK;
+    cudaStream_t st = (cudaStream_t)stream;
+    int rc;
+    if ((rc = wait_lookahead(t, st))) return rc;
+    CK(t, launch_dump_keys(t, d_keys_out, n_rows, st));
     return MLKV_OK;
 }
 

@@ -134,6 +134,49 @@ class EmbeddingStore:
         u = int(num.item())
         return uniq[:u], counts[:u]
 
+    # -- checkpoints (keys in row order, rows, state) -----------------------------
+    def import_(self, keys: torch.Tensor, rows: torch.Tensor, state: torch.Tensor | None = None):
+        """Upsert rows (and state, when given) of keys; the later duplicate wins."""
+        keys = self._keys(keys)
+        rows = self._rows(rows, keys.numel())
+        st = None if state is None else self._rows(state, keys.numel())
+        self._check(self.lib.mlkv_import(self.h, keys.data_ptr(), keys.numel(), rows.data_ptr(),
+                                         None if st is None else st.data_ptr(), _stream(self.device)))
+
+    def keys(self) -> torch.Tensor:
+        """Every key of the table, in row order."""
+        n = self.size()
+        out = torch.empty(n, dtype=torch.int64, device=self.device)
+        self._check(self.lib.mlkv_dump_keys(self.h, out.data_ptr(), n, _stream(self.device)))
+        return out
+
+    def save(self, path: str):
+        """Writes a checkpoint (keys in row order, rows, state) to an .npz file."""
+        import numpy as np
+
+        keys = self.keys()
+        rows, state = [], []
+        for s in range(0, keys.numel(), self.max_batch):
+            w, G = self.export(keys[s:s + self.max_batch])
+            rows.append(w.cpu())
+            state.append(G.cpu())
+        cat = (lambda xs: torch.cat(xs).numpy()) if rows else (lambda xs: np.zeros((0, self.dim), np.float32))
+        np.savez(path, keys=keys.cpu().numpy(), rows=cat(rows), state=cat(state), dim=self.dim)
+
+    def load(self, path: str):
+        """Imports a checkpoint written by save() (into an empty table: the same row ids)."""
+        import numpy as np
+
+        ck = np.load(path)
+        if int(ck["dim"]) != self.dim:
+            raise ValueError(f"checkpoint dim {int(ck['dim'])} != table dim {self.dim}")
+        keys = torch.from_numpy(ck["keys"]).to(self.device)
+        rows = torch.from_numpy(ck["rows"]).to(self.device)
+        state = torch.from_numpy(ck["state"]).to(self.device)
+        for s in range(0, keys.numel(), self.max_batch):
+            e = s + self.max_batch
+            self.import_(keys[s:e], rows[s:e].contiguous(), state[s:e].contiguous())
+
     # -- host-buffer forms (copies inside the call) -----------------------------
     def get_host(self, keys: torch.Tensor, out: torch.Tensor):
         assert keys.device.type == "cpu" and out.device.type == "cpu"
