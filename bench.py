@@ -36,6 +36,8 @@ import workloads as W  # noqa: E402
 
 METRIC = "embedding rows/s (Get + grad-apply) and achieved HBM GB/s vs ~8 TB/s peak"
 UNIT = "rows/s"
+METRIC_YCSB = "key-value operations/s (YCSB-shaped batches of Gets and Puts)"
+UNIT_YCSB = "ops/s"
 NOMINAL_HBM_GBS = 8000.0
 SEQ_SEGMENT_MAX = 32
 CHUNK = 64
@@ -159,7 +161,23 @@ def batch_stats(keys: np.ndarray, d: int) -> dict:
     }
 
 
+def ycsb_stats(read: np.ndarray, write: np.ndarray, d: int) -> dict:
+    """Algorithmic bytes of one Get + Put batch."""
+    R, W = len(read), len(write)
+    Ur, Uw = len(np.unique(read)), len(np.unique(write))
+    row = 4 * d
+    return {
+        "B": R + W, "U": Ur + Uw,
+        "get_gather": R * (8 + row) + Ur * (32 + row),     # keys + output; index sector + row per key
+        "probe": W * 12 + Uw * 32,                         # the Put's keys and rows; index sector per key
+        "put_scatter": W * (8 + row + 4) + Uw * row,       # value + row id + slot per write; row per key
+        "step": R * (8 + row) + Ur * (32 + row) + W * (8 + row) + Uw * (32 + row),
+    }
+
+
 def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
+    if "put_scatter" in stats:  # a key-value batch
+        return {1: stats["get_gather"], 2: stats["probe"], 9: stats["put_scatter"]}[kid]
     if kid == 1:
         return stats["get_gather"]
     if kid == 4:
@@ -180,9 +198,10 @@ def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
 KERNEL_NAMES = {1: "k_get (probe + row gather)", 2: "k_probe", 3: "k_sort_scatter",
                 4: "k_short (run sum + Adagrad)", 5: "k_long_sum (chunk sums of long runs)",
                 6: "k_heads (runs found in the sorted ids)", 7: "k_long_combine (chunk sums + Adagrad)",
-                8: "k_tier_fetch (host <-> HBM row swap)"}
+                8: "k_tier_fetch (host <-> HBM row swap)", 9: "k_put_scatter (Put: last occurrence writes)"}
 KERNEL_SOURCES = {1: "mlkv_index.cu", 2: "mlkv_index.cu", 3: "mlkv_sort.cu", 4: "mlkv_apply.cu",
-                  5: "mlkv_apply.cu", 6: "mlkv_sort.cu", 7: "mlkv_apply.cu", 8: "mlkv_tier.cu"}
+                  5: "mlkv_apply.cu", 6: "mlkv_apply.cu", 7: "mlkv_apply.cu", 8: "mlkv_tier.cu",
+                  9: "mlkv_index.cu"}
 
 
 def traffic_for(kid: int):
@@ -259,20 +278,45 @@ def oracle_steps(cfg, steps: int, sample: int, warmup: int = 0):
     return steps * sample / dt, dt
 
 
+def oracle_ycsb_steps(cfg, steps: int, sample: int, warmup: int = 0):
+    """Times the oracle (one host thread) on `steps` Get + Put batches, each on
+    the first `sample` operations of that step's batch.  Returns (ops/s, seconds)."""
+    import oracle
+
+    ref = oracle.Table(cfg.dim, precision=32, seed=cfg.seed, init_lo=cfg.init_lo, init_hi=cfg.init_hi)
+    batches = []
+    for s in range(warmup + steps):
+        r, w, v = cfg.ops(s)
+        nr = int(round(sample * len(r) / cfg.batch))
+        batches.append((r[:nr], w[:sample - nr], v[:sample - nr]))
+    for r, w, v in batches[:warmup]:
+        ref.get(r)
+        ref.put(w, v)
+    t0 = time.perf_counter()
+    for r, w, v in batches[warmup:]:
+        ref.get(r)
+        ref.put(w, v)
+    dt = time.perf_counter() - t0
+    return steps * sample / dt, dt
+
+
 def run_reference(args, cfg):
     dist, rank, _, world = None, int(os.environ.get("RANK", "0")), 0, int(os.environ.get("WORLD_SIZE", "1"))
     if rank != 0:
         return 0
     sample = max(1, cfg.batch // 8)
-    value, dt = oracle_steps(cfg, args.steps, sample, args.warmup)
+    kv = isinstance(cfg, W.YcsbConfig)
+    value, dt = (oracle_ycsb_steps if kv else oracle_steps)(cfg, args.steps, sample, args.warmup)
     line = {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "impl": "reference", "metric": METRIC_YCSB if kv else METRIC, "value": value,
+        "unit": UNIT_YCSB if kv else UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic", "config": workload_config(cfg),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": f"first {sample} of {cfg.batch} lookups of each step (Get + apply)"},
-        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "cpu_baseline": {"value": value, "unit": UNIT_YCSB if kv else UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"first {sample} of {cfg.batch} operations of each step"},
+        "e2e": {"value": value, "unit": UNIT_YCSB if kv else UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
@@ -306,6 +350,12 @@ def workload_config(cfg) -> dict:
          "l2": "inputs larger than L2 every step (gradients and Get output 4*dim B per lookup)"}
     if isinstance(cfg, W.configs.DlrmConfig):
         c.update({"tables": cfg.tables, "zipf_alpha": cfg.alpha})
+    if isinstance(cfg, W.YcsbConfig):
+        keys = f"Zipf({cfg.alpha})" if cfg.alpha else "uniform"
+        c = {"workload": f"{cfg.name}: {cfg.n_keys:,} records of {cfg.dim} fp32 in HBM, batches of "
+                         f"{cfg.batch:,} operations ({cfg.read_fraction:.0%} Get, the rest Put), {keys} keys",
+             "records": cfg.n_keys, "dim": cfg.dim, "batch_ops": cfg.batch, "read_fraction": cfg.read_fraction,
+             "keys": keys, "l2": "inputs larger than L2 every step (written values and Get output 1 KiB per op)"}
     return c
 
 
@@ -321,6 +371,7 @@ def run_ours(args, cfg):
     hbm_peak, peak_kind = peaks()
 
     tiered = cfg.hbm_cache_rows > 0
+    kv = isinstance(cfg, W.YcsbConfig)
     store = EmbeddingStore(dim=cfg.dim, capacity=cfg.n_keys, max_batch=cfg.batch, lr=cfg.lr, eps=cfg.eps,
                            state_init=cfg.state_init, init_lo=cfg.init_lo, init_hi=cfg.init_hi,
                            seed=cfg.seed, hbm_cache_rows=cfg.hbm_cache_rows, device=dev)
@@ -345,23 +396,37 @@ def run_ours(args, cfg):
     # The HBM store cycles a pool of batches.  The tiered store gets a fresh batch
     # every step (a cycled pool would end up resident in its cache): one per
     # kernel-class prepass step, warm-up step, timed step, and the last look-ahead.
-    kinds = (1, 2, 3, 4, 5, 6, 7) + ((8,) if tiered else ())
+    kinds = (1, 2, 9) if kv else (1, 2, 3, 4, 5, 6, 7) + ((8,) if tiered else ())
     base = len(kinds) if tiered else 0
     pool = base + args.warmup + args.steps + 1 if tiered else max(1, min(args.pool, args.steps + args.warmup))
     ngrad = max(1, min(args.pool, pool))
-    keys_h = [cfg.batch_keys(s) for s in range(pool)]
-    keys_d = [torch.from_numpy(k).to(dev) for k in keys_h]
-    gen = torch.Generator(device=dev)
-    grads_d = []
-    for s in range(ngrad):
-        gen.manual_seed(cfg.seed * 1000 + s)
-        grads_d.append(torch.randn((cfg.batch, cfg.dim), generator=gen, device=dev) * cfg.grad_sigma)
     out = torch.empty((cfg.batch, cfg.dim), dtype=torch.float32, device=dev)
-    stats = [batch_stats(k, cfg.dim) for k in keys_h]
     passes = (int(cfg.n_keys).bit_length() + 7) // 8
+    if kv:  # batches of Gets, then Puts
+        ops_d = []
+        stats = []
+        for s in range(pool):
+            r, w, v = cfg.ops(s)
+            ops_d.append((torch.from_numpy(r).to(dev), torch.from_numpy(w).to(dev), torch.from_numpy(v).to(dev)))
+            stats.append(ycsb_stats(r, w, cfg.dim))
+        keys_h = None
+    else:
+        keys_h = [cfg.batch_keys(s) for s in range(pool)]
+        keys_d = [torch.from_numpy(k).to(dev) for k in keys_h]
+        gen = torch.Generator(device=dev)
+        grads_d = []
+        for s in range(ngrad):
+            gen.manual_seed(cfg.seed * 1000 + s)
+            grads_d.append(torch.randn((cfg.batch, cfg.dim), generator=gen, device=dev) * cfg.grad_sigma)
+        stats = [batch_stats(k, cfg.dim) for k in keys_h]
 
     def step(i):
         j = i % pool
+        if kv:
+            r, w, v = ops_d[j]
+            store.get(r, out=out[:r.numel()])
+            store.put(w, v)
+            return
         store.get(keys_d[j], out=out)
         if tiered and args.lookahead:  # Lookahead(next keys) runs beside this step's apply
             store.lookahead(keys_d[(i + 1) % pool])
@@ -485,7 +550,40 @@ def run_ours(args, cfg):
 
     # end to end through the host-buffer calls (copies inside the timed region)
     e2e = None
-    if not args.no_e2e and not tiered:
+    if not args.no_e2e and kv:
+        # keys and written values from pinned host memory, the Get's output back,
+        # around the store's calls
+        r, w, v = ops_d[0]
+        hr, hw, hv = r.cpu().pin_memory(), w.cpu().pin_memory(), v.cpu().pin_memory()
+        hout = torch.empty((r.numel(), cfg.dim), dtype=torch.float32).pin_memory()
+        dr, dw, dv = torch.empty_like(r), torch.empty_like(w), torch.empty_like(v)
+        e2e_steps = max(1, min(args.steps, 20))
+
+        def kv_e2e():
+            dr.copy_(hr, non_blocking=True)
+            dw.copy_(hw, non_blocking=True)
+            dv.copy_(hv, non_blocking=True)
+            store.get(dr, out=out[:dr.numel()])
+            store.put(dw, dv)
+            hout.copy_(out[:dr.numel()], non_blocking=True)
+
+        for _ in range(2):
+            kv_e2e()
+        barrier(dist, torch)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(e2e_steps):
+            kv_e2e()
+        e1.record(stream)
+        barrier(dist, torch)
+        e_ms = max_over_ranks(dist, torch, e0.elapsed_time(e1))
+        assert store.sync() == 0
+        h2d = (r.numel() + w.numel()) * 8 + v.numel() * 4
+        d2h = r.numel() * cfg.dim * 4
+        e2e = {"value": cfg.batch * e2e_steps * world / (e_ms / 1e3), "unit": UNIT_YCSB, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+               "link_gbs": (h2d + d2h) * e2e_steps / (e_ms / 1e3) / 1e9}
+    if not args.no_e2e and not tiered and not kv:
         e2e_pool = min(pool, 2)
         hk = [torch.from_numpy(keys_h[j]).pin_memory() for j in range(e2e_pool)]
         hg = [grads_d[j % ngrad].cpu().pin_memory() for j in range(e2e_pool)]
@@ -514,14 +612,16 @@ def run_ours(args, cfg):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         sample = max(1, cfg.batch // 8)
         steps = max(1, args.cpu_steps)
-        v, dt = oracle_steps(cfg, steps, sample)
-        cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
-               "sample": f"{steps} steps x first {sample} of {cfg.batch} lookups (Get + apply), "
+        v, dt = (oracle_ycsb_steps if kv else oracle_steps)(cfg, steps, sample)
+        cpu = {"value": v, "unit": UNIT_YCSB if kv else UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"{steps} steps x first {sample} of {cfg.batch} "
+                         f"{'operations (Get + Put)' if kv else 'lookups (Get + apply)'}, "
                          f"{dt:.1f} s on one host thread"}
 
     if rank == 0:
         line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "metric": METRIC_YCSB if kv else METRIC, "value": value, "unit": UNIT_YCSB if kv else UNIT,
+            "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": dict(workload_config(cfg), parallelism=f"replicas{world}", distinct_batches=pool),
@@ -530,8 +630,8 @@ def run_ours(args, cfg):
             "distinct_per_step": float(np.mean([s["U"] for s in stats])),
             "roofline": roofline, "kernel_ms_one_step": {KERNEL_NAMES[k]: v for k, v in kernel_ms.items()},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clocks.summary(),
-            "step_launch": ("one CUDA graph replay per step (the Get and the apply of the batch, captured)"
-                            if use_graphs else "each call launched from the host"),
+            "step_launch": (f"one CUDA graph replay per step (the Get and the {'Put' if kv else 'apply'} of the "
+                            f"batch, captured)" if use_graphs else "each call launched from the host"),
         }
         if tier is not None:
             line["tier"] = tier

@@ -31,6 +31,7 @@ K_REDUCE_LONG = 5
 K_SEGMENTS = 6
 K_LONG_COMBINE = 7
 K_TIER_FETCH = 8
+K_PUT_SCATTER = 9
 
 EXPORTED = [
     "mlkv_open", "mlkv_close", "mlkv_get", "mlkv_put", "mlkv_insert", "mlkv_apply_grad",

@@ -510,7 +510,7 @@ struct PutRun {
         MLKV_LAUNCH(t, 0, k_put_mark, grid_for(n, 256), 256, 0, st, t->index, t->s.row_of_pos,
                     t->s.slot_of_pos, (uint32_t)n);
         const unsigned g = capped_grid(t, n * (int64_t)t->geom.G, 256, 8);
-        MLKV_LAUNCH(t, 0, (k_put_scatter<V, KV>), g, 256, 0, st, t->index, row_args(t),
+        MLKV_LAUNCH(t, MLKV_K_PUT_SCATTER, (k_put_scatter<V, KV>), g, 256, 0, st, t->index, row_args(t),
                     t->s.row_of_pos, t->s.slot_of_pos, vals, state, (uint32_t)n);
         return cudaGetLastError();
     }

@@ -19,6 +19,11 @@ dataset is available):
          2-hop fanout 10 then 25 over a Chung-Lu power-law graph, grads
          N(0, 1e-3), lr 0.05.
   tiered 400,000,000 rows, dim 128, 1,048,576 Zipf(1.1) lookups, grads N(0, 1e-3).
+  ycsb   a YCSB-shaped key-value mix (MLKV Section 4.5: 50% reads, 50% writes,
+         uniform or skewed keys): 50,000,000 records of 256 fp32 (1 KiB),
+         batches of 1,048,576 operations, each a Get or a Put by a seeded coin,
+         keys Zipf(0.99) ("ycsb") or uniform ("ycsb-uniform"), written values
+         N(0, 0.01).
 The second parameter of N(., .) is the standard deviation.
 """
 from dataclasses import dataclass, field
@@ -191,6 +196,36 @@ class TieredConfig(StoreConfig):
         return self._cache["map"](self._cache["zipf"].sample(_rng(self.index, step, 3), self.batch))
 
 
+@dataclass
+class YcsbConfig(StoreConfig):
+    """Batches of Get and Put operations over the preloaded records.  A batch's
+    Gets read the records as they were before the batch; its Puts then write
+    (the later of two Puts of a key wins)."""
+    read_fraction: float = 0.5
+    alpha: float = 0.99  # 0: uniform keys
+
+    def _keys(self, step: int) -> np.ndarray:
+        rng = _rng(self.index, step, 3)
+        if self.alpha == 0.0:
+            return rng.integers(0, self.n_keys, self.batch, dtype=np.int64)
+        if "map" not in self._cache:
+            self._cache["map"] = scatter_bijection(self.n_keys, _rng(self.index, 100))
+            self._cache["zipf"] = ZipfSampler(self.n_keys, self.alpha)
+        return self._cache["map"](self._cache["zipf"].sample(rng, self.batch))
+
+    def ops(self, step: int):
+        """(keys read, keys written, values written [n, dim] float32), in batch order."""
+        keys = self._keys(step)
+        read = _rng(self.index, step, 9).random(self.batch) < self.read_fraction
+        w = keys[~read]
+        vals = _rng(self.index, step, 11).standard_normal((len(w), self.dim), dtype=np.float32)
+        vals *= np.float32(self.grad_sigma)
+        return keys[read], w, vals
+
+    def batch_keys(self, step: int) -> np.ndarray:
+        return self._keys(step)
+
+
 def tiny():
     return TinyConfig("tiny", 0, dim=16, n_keys=100_000, batch=4_096, steps=10, lr=0.1,
                       grad_sigma=0.01)
@@ -216,7 +251,18 @@ def tiered():
                         lr=0.01, grad_sigma=1e-3, hbm_cache_rows=120 * 10**9 // 1024)
 
 
-ALL = {"tiny": tiny, "dlrm": dlrm, "kg": kg, "gnn": gnn, "tiered": tiered}
+def ycsb():
+    return YcsbConfig("ycsb", 5, dim=256, n_keys=50_000_000, batch=1_048_576, steps=20, lr=0.0,
+                      grad_sigma=0.01, alpha=0.99)
+
+
+def ycsb_uniform():
+    return YcsbConfig("ycsb-uniform", 6, dim=256, n_keys=50_000_000, batch=1_048_576, steps=20, lr=0.0,
+                      grad_sigma=0.01, alpha=0.0)
+
+
+ALL = {"tiny": tiny, "dlrm": dlrm, "kg": kg, "gnn": gnn, "tiered": tiered, "ycsb": ycsb,
+       "ycsb-uniform": ycsb_uniform}
 
 
 def scaled(cfg: StoreConfig, key_scale: int, batch_scale: int) -> StoreConfig:
