@@ -288,6 +288,7 @@ __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, u
 // with one atomic each and the warps copy their runs out.  (Counters that
 // every warp bumps queue up at the end of the kernel.)
 __global__ void __launch_bounds__(256) k_heads(RunArgs a) {
+    pdl_enter();
     constexpr int kList = 128, kQueue = 16;
     __shared__ uint4 lst[8][kList];  // (start, end, row, first lookup) of short runs
     __shared__ uint32_t qs[8][kQueue], qr[8][kQueue], qe[8][kQueue];  // long runs: start, row, end (0: unknown)
@@ -440,6 +441,7 @@ __device__ __forceinline__ uint4 run_meta(const RunArgs& a, uint32_t u, uint32_t
 
 template <int V, int KV>
 __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra, RunArgs a) {
+    pdl_enter();
     const uint32_t U = a.cur->n_short;
     const int lane = threadIdx.x & 31, G = ra.G, glane = lane & (G - 1), gid = lane / G;
     const unsigned gmask = group_mask(G, gid);
@@ -455,6 +457,7 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
 
 template <int V, int KV>
 __global__ void __launch_bounds__(256, MLKV_LONG_MIN_BLOCKS) k_long_sum(RowArgs ra, RunArgs a) {
+    pdl_enter();
     using VT = typename Vec<V>::T;
     const uint32_t NI = min(a.cur->n_items, a.max_items);
     const int lane = threadIdx.x & 31, G = ra.G, glane = lane & (G - 1), gid = lane / G;
@@ -510,6 +513,7 @@ __device__ __forceinline__ void sum_partials(typename Vec<V>::T (&acc)[KV], cons
 // takes one lane group, which adds its sums in order.  Then the Adagrad step.
 template <int V, int KV>
 __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, DevState* ds) {
+    pdl_enter();
     using VT = typename Vec<V>::T;
     extern __shared__ float sh[];  // [groups][dpad]
     const uint32_t nl = min(a.cur->n_long, a.max_long), nb = a.cur->n_big;
@@ -579,15 +583,15 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     if (gh < 1) gh = 1;
     MLKV_LAUNCH(t, MLKV_K_SEGMENTS, k_heads, (unsigned)gh, 256, 0, st, a);
     const int gs = persistent_blocks(t, (const void*)k_short<V, KV>, 256);
-    MLKV_LAUNCH(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, st, ra, a);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, st, ra, a);
     const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);
-    MLKV_LAUNCH(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, st, ra, a);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, st, ra, a);
     int big = 1024;  // the groups' sums must fit the default 48 KB of shared memory
     while (big > 64 && (size_t)(big / t->geom.G) * t->geom.dpad * sizeof(float) > 48 * 1024) big /= 2;
     const size_t smem = (size_t)(big / t->geom.G) * t->geom.dpad * sizeof(float);
     // one block per SM (a 1024-thread block fills the register file): 4,864
     // lane groups of 32 for the ordinary long runs, 152 blocks for the big ones
-    MLKV_LAUNCH(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), t->num_sms * (1024 / big), big, smem, st, ra, a,
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), t->num_sms * (1024 / big), big, smem, st, ra, a,
                 t->dstate);
     return cudaGetLastError();
 }

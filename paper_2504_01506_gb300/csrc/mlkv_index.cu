@@ -122,6 +122,7 @@ __global__ void __launch_bounds__(256) k_probe(IndexArgs ia, const int64_t* __re
                                                uint32_t* miss_pos, uint32_t* miss_slot,
                                                CallCounters* cur, CallCounters* nxt,
                                                int report_absent, Memo memo, int memo_use) {
+    pdl_enter();
     zero_counters(nxt);
     const uint32_t base = blockIdx.x * (blockDim.x * kProbeKeys) + threadIdx.x;
     unsigned long long k[kProbeKeys];
@@ -186,6 +187,7 @@ __global__ void __launch_bounds__(256, MLKV_GET_MIN_BLOCKS) k_get(IndexArgs ia, 
                                              float* __restrict__ out, uint32_t* miss_pos,
                                              uint32_t* miss_slot, CallCounters* cur,
                                              CallCounters* nxt, Memo memo) {
+    pdl_enter();
     using VT = typename Vec<V>::T;
     zero_counters(nxt);
     const int lane = threadIdx.x & 31;
@@ -239,6 +241,7 @@ __global__ void __launch_bounds__(256, MLKV_GET_MIN_BLOCKS) k_get(IndexArgs ia, 
 __global__ void k_miss_flag(const Slot* __restrict__ index, const uint32_t* __restrict__ miss_pos,
                             const uint32_t* __restrict__ miss_slot, uint32_t* __restrict__ flag,
                             const CallCounters* cur) {
+    pdl_enter();
     const uint32_t m = cur->n_miss;
     for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < m; i += gridDim.x * blockDim.x) {
         const uint32_t p = miss_pos[i];
@@ -258,6 +261,7 @@ __global__ void __launch_bounds__(256) k_miss_assign(IndexArgs ia, RowArgs ra,
                                                      unsigned long long capacity, int init_row,
                                                      unsigned long long seed, float lo, float span,
                                                      float state_init) {
+    pdl_enter();
     using VT = typename Vec<V>::T;
     const uint32_t m = cur->n_miss;
     const int G = ra.G, glane = threadIdx.x & (G - 1);
@@ -303,6 +307,7 @@ __global__ void __launch_bounds__(256) k_miss_finish(IndexArgs ia, RowArgs ra,
                                                      float* __restrict__ out,
                                                      const CallCounters* cur, DevState* ds,
                                                      unsigned long long capacity) {
+    pdl_enter();
     const uint32_t m = cur->n_miss;
     if (blockIdx.x == 0 && threadIdx.x == 0 && m) {
         const unsigned long long nr = ds->next_row + cur->n_new;
@@ -330,6 +335,7 @@ __global__ void __launch_bounds__(256) k_miss_finish(IndexArgs ia, RowArgs ra,
 // occurrences of (0xFFFFFFFE - p).
 __global__ void k_put_mark(Slot* __restrict__ index, const uint32_t* __restrict__ row_of_pos,
                            const uint32_t* __restrict__ slot_of_pos, uint32_t n) {
+    pdl_enter();
     const uint32_t p = blockIdx.x * blockDim.x + threadIdx.x;
     if (p >= n || row_of_pos[p] >= ROW_ABSENT) return;
     atomicMin(&index[slot_of_pos[p]].aux, 0xFFFFFFFEu - p);
@@ -342,6 +348,7 @@ __global__ void __launch_bounds__(256) k_put_scatter(Slot* __restrict__ index, R
                                                      const uint32_t* __restrict__ slot_of_pos,
                                                      const float* __restrict__ vals,
                                                      const float* __restrict__ state, uint32_t n) {
+    pdl_enter();
     using VT = typename Vec<V>::T;
     const int lane = threadIdx.x & 31, G = ra.G, R = 32 / G, glane = lane & (G - 1), gid = lane / G;
     const uint32_t warp = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -381,6 +388,7 @@ __global__ void __launch_bounds__(256) k_put_scatter(Slot* __restrict__ index, R
 __global__ void __launch_bounds__(256) k_find(IndexArgs ia, const int64_t* __restrict__ keys,
                                               uint32_t n, int64_t* __restrict__ rows,
                                               CallCounters* nxt) {
+    pdl_enter();
     zero_counters(nxt);
     const uint32_t p = blockIdx.x * blockDim.x + threadIdx.x;
     if (p >= n) return;
@@ -404,6 +412,7 @@ __global__ void __launch_bounds__(256) k_export(IndexArgs ia, RowArgs ra,
                                                 float* __restrict__ rows_out,
                                                 float* __restrict__ state_out, CallCounters* nxt,
                                                 ExportTier et) {
+    pdl_enter();
     zero_counters(nxt);
     const int lane = threadIdx.x & 31;
     const uint32_t base = (blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * 32u;
@@ -520,6 +529,7 @@ struct PutRun {
 // order (rows are dense, handed out in first-occurrence order).
 __global__ void __launch_bounds__(256) k_dump_keys(const Slot* __restrict__ index, unsigned long long nslots,
                                                    int64_t* __restrict__ out, uint32_t n_rows) {
+    pdl_enter();
     for (unsigned long long s = blockIdx.x * (unsigned long long)blockDim.x + threadIdx.x; s < nslots;
          s += (unsigned long long)gridDim.x * blockDim.x) {
         const unsigned long long key = index[s].key;

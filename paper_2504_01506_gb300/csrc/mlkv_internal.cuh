@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "../../include/mlkv_gpu.h"
 
 namespace mlkv {
@@ -265,6 +267,27 @@ template <> struct Vec<1> {
     }
 };
 
+// Programmatic dependent launch.  MLKV_LAUNCH lets a kernel start while the
+// kernel before it on the stream drains, which hides the launch and ramp-up
+// of the ~25 kernels of a step.  Every kernel begins with pdl_enter():
+//   - griddepcontrol.wait returns once the grid this launch depends on has
+//     completed and its writes are visible (at once when the launch has no
+//     such dependency).  Every kernel waits, on every path, before touching
+//     memory, so the completion of a kernel implies the completion of all the
+//     kernels before it;
+//   - griddepcontrol.launch_dependents lets the next kernel's blocks be
+//     scheduled (once every block of this grid has issued it or exited);
+//     they in turn wait for this grid.  Issued after the wait, it keeps at
+//     most one grid waiting ahead of the running one.
+#ifndef MLKV_PDL_TRIGGER_FIRST
+#define MLKV_PDL_TRIGGER_FIRST 0
+#endif
+__device__ __forceinline__ void pdl_enter() {
+    if (MLKV_PDL_TRIGGER_FIRST) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (!MLKV_PDL_TRIGGER_FIRST) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ uint32_t lanemask_lt() {
     uint32_t m;
     asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
@@ -312,6 +335,9 @@ cudaError_t launch_export(mlkv_table* t, const int64_t* keys, int64_t n, float* 
 // mlkv_sort.cu
 cudaError_t launch_exclusive_scan(mlkv_table* t, const uint32_t* in, uint32_t* out, int64_t n,
                                   uint32_t* total, const uint32_t* enable, cudaStream_t st);
+// The sort's digit totals start at zero: a call that sorts zeroes them before
+// its first kernel (a memset between two kernels would end their overlap).
+cudaError_t zero_sort_totals(mlkv_table* t, cudaStream_t st);
 cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow,
                              const uint32_t** spos);
 cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, const uint32_t* spos, int64_t n,
@@ -341,11 +367,43 @@ int persistent_blocks(mlkv_table* t, const void* kernel, int threads);
 
 }  // namespace mlkv
 
+// Programmatic dependent launch of every kernel (off with -DMLKV_PDL=0: plain
+// stream order; the kernels' pdl_wait() then returns at once).
+#ifndef MLKV_PDL
+#define MLKV_PDL 1
+#endif
+
+namespace mlkv {
+template <typename... Params, typename... Args>
+inline void launch_kernel(bool pdl, void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+                          cudaStream_t st, Args&&... args) {
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = MLKV_PDL && pdl ? 1 : 0;
+    cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);  // an error stays in cudaGetLastError()
+}
+}  // namespace mlkv
+
 // Launch helper: counts the launch and records timing events when asked.
-#define MLKV_LAUNCH(t, kid, kernel, grid, block, smem, stream, ...)        \
-    do {                                                                   \
-        mlkv::timer_before((t), (kid), (stream));                          \
-        kernel<<<(grid), (block), (smem), (stream)>>>(__VA_ARGS__);        \
-        mlkv::timer_after((t), (kid), (stream));                           \
-        (t)->launches++;                                                   \
+#define MLKV_LAUNCH_PDL(pdl, t, kid, kernel, grid, block, smem, stream, ...)                      \
+    do {                                                                                          \
+        mlkv::timer_before((t), (kid), (stream));                                                 \
+        mlkv::launch_kernel((pdl), kernel, dim3(grid), dim3(block), (smem), (stream), __VA_ARGS__); \
+        mlkv::timer_after((t), (kid), (stream));                                                  \
+        (t)->launches++;                                                                          \
     } while (0)
+#define MLKV_LAUNCH(...) MLKV_LAUNCH_PDL(true, __VA_ARGS__)
+// A persistent grid (one wave, each block a fixed share of the work) starts
+// once the kernel before it has finished, with every SM free: blocks placed
+// early on the SMs that drain first would leave the others short of work.
+#ifndef MLKV_PDL_PERSISTENT
+#define MLKV_PDL_PERSISTENT 0
+#endif
+#define MLKV_LAUNCH_PERSISTENT(...) MLKV_LAUNCH_PDL(MLKV_PDL_PERSISTENT != 0, __VA_ARGS__)

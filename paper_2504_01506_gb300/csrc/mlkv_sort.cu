@@ -69,6 +69,7 @@ __device__ __forceinline__ uint32_t tiles_before(const uint32_t* __restrict__ ti
 __global__ void __launch_bounds__(kThreads) k_scan_reduce(const uint32_t* __restrict__ in, uint32_t n,
                                                           uint32_t* __restrict__ tile_sums,
                                                           const uint32_t* enable) {
+    pdl_enter();
     if (enable && *enable == 0u) return;
     const uint32_t base = blockIdx.x * kTile;
     uint32_t s = 0;
@@ -85,6 +86,7 @@ __global__ void __launch_bounds__(kThreads) k_scan_reduce(const uint32_t* __rest
 __global__ void __launch_bounds__(kThreads) k_scan_down(const uint32_t* in, uint32_t* out, uint32_t n,
                                                         const uint32_t* __restrict__ tile_sums,
                                                         uint32_t* total_out, const uint32_t* enable) {
+    pdl_enter();
     if (enable && *enable == 0u) return;
     __shared__ uint32_t tile[kTile + kTile / 32];
     const uint32_t base = blockIdx.x * kTile;
@@ -156,6 +158,7 @@ __global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restri
                                                         uint32_t* __restrict__ counts, uint32_t* __restrict__ dtot,
                                                         uint32_t ntiles, int shift, int radix, uint32_t sent,
                                                         int first) {
+    pdl_enter();
     __shared__ uint32_t hist[kMaxRadix];
     for (int d = threadIdx.x; d < radix; d += kThreads) hist[d] = 0;
     __syncthreads();
@@ -205,6 +208,7 @@ __global__ void __launch_bounds__(kThreads) k_sort_offsets(const uint32_t* __res
                                                            const uint32_t* __restrict__ dtot,
                                                            uint32_t* __restrict__ offsets, uint32_t ntiles,
                                                            int radix) {
+    pdl_enter();
     constexpr int kRounds = 8;
     const int lane = threadIdx.x & 31;
     const int d = blockIdx.x * kWarps + (threadIdx.x >> 5);
@@ -251,6 +255,7 @@ __global__ void __launch_bounds__(kThreads, 3) k_sort_scatter(const uint32_t* __
                                                               const uint32_t* __restrict__ offsets,
                                                               uint32_t ntiles, int shift, int radix, uint32_t sent,
                                                               int first) {
+    pdl_enter();
     // the per-warp digit counts, then (once every position is known) the sorted tile
     __shared__ uint32_t pool[2 * kTile];
     static_assert(kWarps * kMaxRadix <= 2 * kTile, "counts fit the tile buffer");
@@ -348,6 +353,7 @@ __device__ __forceinline__ bool is_head(const uint32_t* srow, uint32_t p, uint32
 
 __global__ void __launch_bounds__(kThreads) k_seg_reduce(const uint32_t* __restrict__ srow, uint32_t n,
                                                          uint32_t sent, uint32_t* __restrict__ tile_sums) {
+    pdl_enter();
     const uint32_t base = blockIdx.x * kTile;
     uint32_t s = 0;
 #pragma unroll 4
@@ -364,6 +370,7 @@ __global__ void __launch_bounds__(kThreads) k_seg_down(const uint32_t* __restric
                                                        uint32_t* __restrict__ run_row,
                                                        uint32_t* __restrict__ run_p0, CallCounters* cur,
                                                        DevState* ds) {
+    pdl_enter();
     const uint32_t base = blockIdx.x * kTile;
     const uint32_t prefix = tiles_before(tile_sums, blockIdx.x);
     // thread t owns items base + t*16 .. +15 (consecutive, for an in-order compaction)
@@ -398,6 +405,7 @@ __global__ void __launch_bounds__(kThreads) k_seg_down(const uint32_t* __restric
 __global__ void k_dedup_out(const int64_t* __restrict__ keys, const uint32_t* __restrict__ spos,
                             const uint32_t* __restrict__ seg_start, const CallCounters* cur,
                             int64_t* __restrict__ uniq, int32_t* __restrict__ counts, int64_t* num) {
+    pdl_enter();
     const uint32_t U = cur->n_unique, nv = cur->n_valid;
     if (blockIdx.x == 0 && threadIdx.x == 0) *num = (int64_t)U;
     for (uint32_t u = blockIdx.x * blockDim.x + threadIdx.x; u < U; u += gridDim.x * blockDim.x) {
@@ -430,9 +438,7 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
     const unsigned nt = tiles(n);
     uint32_t* counts = t->s.sort_counts;
     uint32_t* offsets = t->s.sort_offsets;
-    // digit totals of every pass start at zero
-    cudaError_t e = cudaMemsetAsync(t->s.sort_dtot, 0, (size_t)kSortMaxPasses * kMaxRadix * 4, st);
-    if (e != cudaSuccess) return e;
+    // the digit totals of every pass were zeroed at the start of the call (zero_sort_totals)
     const uint32_t* kin = t->s.row_of_pos;
     const uint32_t* vin = nullptr;
     int out = 0;
@@ -452,6 +458,10 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
     *srow = kin;
     *spos = vin;
     return cudaGetLastError();
+}
+
+cudaError_t zero_sort_totals(mlkv_table* t, cudaStream_t st) {
+    return cudaMemsetAsync(t->s.sort_dtot, 0, (size_t)kSortMaxPasses * kMaxRadix * 4, st);
 }
 
 cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, const uint32_t* spos, int64_t n,

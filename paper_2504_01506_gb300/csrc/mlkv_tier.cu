@@ -66,6 +66,7 @@ __global__ void __launch_bounds__(256) k_tier_init(uint32_t* __restrict__ row_lo
 
 __global__ void __launch_bounds__(256) k_tier_resolve(TierArgs ta, const uint32_t* __restrict__ row_of_pos,
                                                       uint32_t n, uint2* fetch, uint32_t* n_fetch) {
+    pdl_enter();
     const uint32_t p = blockIdx.x * blockDim.x + threadIdx.x;
     if (p >= n) return;
     const uint32_t r = row_of_pos[p];
@@ -104,6 +105,7 @@ __global__ void __launch_bounds__(256) k_tier_resolve(TierArgs ta, const uint32_
 template <int KV>
 __global__ void __launch_bounds__(256) k_tier_fetch(TierArgs ta, const uint2* __restrict__ fetch,
                                                     const uint32_t* n_fetch) {
+    pdl_enter();
     __shared__ uint32_t s_line[8][32];
     const uint32_t nf = *n_fetch;
     const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
@@ -191,6 +193,7 @@ __global__ void __launch_bounds__(256) k_tier_fetch(TierArgs ta, const uint2* __
 }
 
 __global__ void __launch_bounds__(256) k_tier_remap(TierArgs ta, uint32_t* __restrict__ row_of_pos, uint32_t n) {
+    pdl_enter();
     const uint32_t p = blockIdx.x * blockDim.x + threadIdx.x;
     if (p >= n) return;
     const uint32_t r = row_of_pos[p];
@@ -204,6 +207,7 @@ template <int V, int KV>
 __global__ void __launch_bounds__(256) k_gather_lines(const float* __restrict__ slots, int stride, int d, int NV,
                                                       int G, const uint32_t* __restrict__ row_of_pos, uint32_t n,
                                                       float* __restrict__ out) {
+    pdl_enter();
     using VT = typename Vec<V>::T;
     const int lane = threadIdx.x & 31;
     const uint32_t base = (blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * 32u;
