@@ -111,47 +111,79 @@ IndexArgs index_args(mlkv_table* t) {
 
 // ---------------------------------------------------------------------------
 // row_of_pos[p] (and the slot) for every position.  Each thread takes
-// kProbeKeys lookups spaced a block apart, so their loads are in flight
+// kProbeKeys lookups spaced a block apart, so that their loads are in flight
 // together (the probe is latency-bound: a key load, then a random slot load).
+// With COUNT (the gradient apply on an HBM-resident table) a block of 1024
+// threads covers one 4096-lookup tile of the sort and also counts the first
+// sort pass's digits of its rows (see FirstCounts).
 constexpr int kProbeKeys = 4;
 
-template <bool INSERT>
-__global__ void __launch_bounds__(256) k_probe(IndexArgs ia, const int64_t* __restrict__ keys,
+template <bool INSERT, bool COUNT>
+__global__ void __launch_bounds__(COUNT ? 1024 : 256) k_probe(IndexArgs ia, const int64_t* __restrict__ keys,
                                                uint32_t n, uint32_t* __restrict__ row_of_pos,
                                                uint32_t* __restrict__ slot_of_pos,
                                                uint32_t* miss_pos, uint32_t* miss_slot,
                                                CallCounters* cur, CallCounters* nxt,
-                                               int report_absent, Memo memo, int memo_use) {
+                                               int report_absent, Memo memo, int memo_use, FirstCounts fc) {
+    constexpr int KEYS = kProbeKeys;
+    static_assert(KEYS * 1024 == kSortTile, "a counting block covers one sort tile");
     pdl_enter();
     zero_counters(nxt);
-    const uint32_t base = blockIdx.x * (blockDim.x * kProbeKeys) + threadIdx.x;
-    unsigned long long k[kProbeKeys];
-    uint32_t known[kProbeKeys];
-#pragma unroll
-    for (int j = 0; j < kProbeKeys; ++j) {
-        const uint32_t p = base + j * blockDim.x;
-        k[j] = p < n ? (unsigned long long)__ldg(keys + p) : 0ull;
-        known[j] = ROW_PENDING;
-        if (memo_use == (int)MemoUse::Read && p < n && (unsigned long long)memo.key[p] == k[j]) known[j] = memo.row[p];
+    __shared__ uint32_t hist[COUNT ? kSortMaxRadix : 1];
+    if (COUNT) {
+        for (int d = threadIdx.x; d < fc.radix; d += blockDim.x) hist[d] = 0u;
+        __syncthreads();
     }
+    bool missed = false;  // a lookup of this thread waits for the miss path for its row
+    const uint32_t base = blockIdx.x * (blockDim.x * KEYS) + threadIdx.x;
+#pragma unroll 1
+    for (int j0 = 0; j0 < KEYS; j0 += kProbeKeys) {
+        unsigned long long k[kProbeKeys];
+        uint32_t known[kProbeKeys];
 #pragma unroll
-    for (int j = 0; j < kProbeKeys; ++j) {
-        const uint32_t p = base + j * blockDim.x;
-        if (p >= n) continue;
-        if (known[j] < ROW_ABSENT) {  // the row the last Get found for this key here
-            row_of_pos[p] = known[j];
-            continue;
+        for (int j = 0; j < kProbeKeys; ++j) {
+            const uint32_t p = base + (j0 + j) * blockDim.x;
+            k[j] = p < n ? (unsigned long long)__ldg(keys + p) : 0ull;
+            known[j] = ROW_PENDING;
+            if (memo_use == (int)MemoUse::Read && p < n) {
+                const uint32_t r = memo.row[p];  // loaded beside the key it belongs to
+                if ((unsigned long long)memo.key[p] == k[j]) known[j] = r;
+            }
         }
-        uint32_t slot = 0;
-        const uint32_t row = probe_key<INSERT>(ia, k[j], p, slot);
-        if (!INSERT && report_absent && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
-        row_of_pos[p] = row;
-        if (slot_of_pos) slot_of_pos[p] = slot;
-        if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
-        if (memo_use == (int)MemoUse::Save) {
-            memo.key[p] = (int64_t)k[j];
-            memo.row[p] = row;
+#pragma unroll
+        for (int j = 0; j < kProbeKeys; ++j) {
+            const uint32_t p = base + (j0 + j) * blockDim.x;
+            if (p >= n) continue;
+            uint32_t row = known[j];
+            if (row >= ROW_ABSENT) {  // not the row the last Get found for this key here: probe
+                uint32_t slot = 0;
+                row = probe_key<INSERT>(ia, k[j], p, slot);
+                if (!INSERT && report_absent && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
+                if (slot_of_pos) slot_of_pos[p] = slot;
+                if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
+                if (memo_use == (int)MemoUse::Save) {
+                    memo.key[p] = (int64_t)k[j];
+                    memo.row[p] = row;
+                }
+            }
+            row_of_pos[p] = row;
+            if (COUNT) {
+                if (row == ROW_PENDING) missed = true;
+                else atomicAdd(&hist[(row >= ROW_ABSENT ? fc.sent : row) & (uint32_t)(fc.radix - 1)], 1u);
+            }
         }
+    }
+    if (COUNT) {
+        // a tile with a miss is counted after the miss path has given its rows
+        const int dirty = __syncthreads_or(missed);
+        if (!dirty) {
+            for (int d = threadIdx.x; d < fc.radix; d += blockDim.x) {
+                const uint32_t c = hist[d];
+                fc.counts[(size_t)d * fc.ntiles + blockIdx.x] = c;
+                if (c) atomicAdd(fc.dtot + d, c);
+            }
+        }
+        if (threadIdx.x == 0) fc.dirty[blockIdx.x] = dirty ? 1u : 0u;
     }
 }
 
@@ -554,18 +586,30 @@ struct ExportRun {
 
 cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool insert, MemoUse memo,
                          bool want_slot, bool report_absent, cudaStream_t st, CallCounters* cur,
-                         CallCounters* nxt, uint32_t* rows_out) {
+                         CallCounters* nxt, uint32_t* rows_out, const FirstCounts* fc) {
     uint32_t* slot_of_pos = want_slot ? t->s.slot_of_pos : nullptr;
     uint32_t* rows = rows_out ? rows_out : t->s.row_of_pos;
     if (want_slot && memo == MemoUse::Read) memo = MemoUse::None;  // the memo holds no slots
     const Memo m{t->s.memo_key, t->s.memo_row};
+    const int ra = report_absent ? 1 : 0;
+    if (fc) {  // one block per sort tile, counting the first pass
+        const unsigned g = grid_for(n, kSortTile);
+        if (insert)
+            MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<true, true>), g, 1024, 0, st, index_args(t), keys, (uint32_t)n,
+                        rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0, m, (int)memo, *fc);
+        else
+            MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<false, true>), g, 1024, 0, st, index_args(t), keys, (uint32_t)n,
+                        rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, ra, m, (int)memo, *fc);
+        return cudaGetLastError();
+    }
+    const FirstCounts none{};
+    const unsigned g = grid_for(n, 256 * kProbeKeys);
     if (insert)
-        MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<true>, grid_for(n, 256 * kProbeKeys), 256, 0, st, index_args(t), keys,
-                    (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0, m, (int)memo);
+        MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<true, false>), g, 256, 0, st, index_args(t), keys,
+                    (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0, m, (int)memo, none);
     else
-        MLKV_LAUNCH(t, MLKV_K_PROBE, k_probe<false>, grid_for(n, 256 * kProbeKeys), 256, 0, st, index_args(t), keys,
-                    (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt,
-                    report_absent ? 1 : 0, m, (int)memo);
+        MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<false, false>), g, 256, 0, st, index_args(t), keys,
+                    (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, ra, m, (int)memo, none);
     return cudaGetLastError();
 }
 

@@ -28,6 +28,8 @@ constexpr uint32_t AUX_IDLE = 0xFFFFFFFFu;
 constexpr int PROBE_LIMIT = MLKV_PROBE_LIMIT;
 constexpr int kSortMaxPasses = 4;      // row ids have at most 31 bits
 constexpr int kSortMaxDigitBits = 9;   // radix <= 512
+constexpr int kSortMaxRadix = 1 << kSortMaxDigitBits;
+constexpr int kSortTile = 4096;        // lookups per tile of a sort pass
 
 // Per-call counters.  Two copies: a call uses cc[p] and its first kernel
 // zeroes cc[p ^ 1] for the next call, so no memset is enqueued.
@@ -79,6 +81,7 @@ struct Scratch {
     uint32_t* sort_counts;  // [512][tiles] digit counts of a sort pass
     uint32_t* sort_offsets; // [tiles][512] output position of each tile's first element of each digit
     uint32_t* sort_dtot;    // [kSortMaxPasses][512] digit totals of each pass
+    uint32_t* sort_dirty;   // [tiles] 1: the first pass's counts of the tile are left to the histogram kernel
     uint32_t* tile_sums;    // [scan tiles]
     uint32_t* seg_start;    // [max_batch + 1] run starts in sorted order (dedup)
     uint32_t* run_row;      // [max_batch] row of each run (dedup)
@@ -313,6 +316,20 @@ struct Memo {
 };
 enum class MemoUse { None, Read, Save };
 
+// The first sort pass's digit counts, made by the apply's probe: a tile of
+// kSortTile lookups whose rows are all known after the probe (no miss) has its
+// column of counts[digit][tile] written and its counts added to the pass's
+// totals there, and dirty[tile] = 0; a tile with a miss gets dirty[tile] = 1
+// and is counted by the histogram kernel once the miss path has given rows.
+struct FirstCounts {
+    uint32_t* counts;
+    uint32_t* dtot;
+    uint32_t* dirty;
+    uint32_t ntiles;
+    int radix;       // digits of the first pass
+    uint32_t sent;   // sort key of a lookup without a row
+};
+
 // ---------------------------------------------------------------------------
 // Host-side launchers (each returns cudaGetLastError() of its launches).
 enum class MissMode : int { Init = 0, Put = 1, Get = 2 };
@@ -320,7 +337,7 @@ enum class MissMode : int { Init = 0, Put = 1, Get = 2 };
 // mlkv_index.cu
 cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool insert, MemoUse memo,
                          bool want_slot, bool report_absent, cudaStream_t st, CallCounters* cur,
-                         CallCounters* nxt, uint32_t* rows_out = nullptr);
+                         CallCounters* nxt, uint32_t* rows_out = nullptr, const FirstCounts* fc = nullptr);
 cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out, cudaStream_t st,
                        CallCounters* cur, CallCounters* nxt);
 cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode,
@@ -338,8 +355,11 @@ cudaError_t launch_exclusive_scan(mlkv_table* t, const uint32_t* in, uint32_t* o
 // The sort's digit totals start at zero: a call that sorts zeroes them before
 // its first kernel (a memset between two kernels would end their overlap).
 cudaError_t zero_sort_totals(mlkv_table* t, cudaStream_t st);
+// The first pass's counts for the probe to make (t->sort_bits rows, n lookups).
+FirstCounts first_counts(mlkv_table* t, int64_t n);
+// first_dirty: null, or FirstCounts::dirty of a probe that counted the first pass.
 cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow,
-                             const uint32_t** spos);
+                             const uint32_t** spos, const uint32_t* first_dirty = nullptr);
 cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, const uint32_t* spos, int64_t n,
                             cudaStream_t st, CallCounters* cur);
 cudaError_t launch_dedup_out(mlkv_table* t, const int64_t* keys, const uint32_t* spos, int64_t n,

@@ -24,6 +24,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kItems = 16;
 constexpr int kTile = kThreads * kItems;  // 4096
+static_assert(kTile == kSortTile, "the probe counts tiles of the sort's size");
 constexpr int kWarps = kThreads / 32;
 
 __device__ __forceinline__ int spad(int i) { return i + (i >> 5); }
@@ -125,7 +126,7 @@ __device__ __forceinline__ uint32_t sort_key(uint32_t r, uint32_t sent, bool fir
     return first ? (r >= ROW_ABSENT ? sent : r) : r;
 }
 
-constexpr int kMaxRadix = 1 << kSortMaxDigitBits;
+constexpr int kMaxRadix = kSortMaxRadix;
 
 #ifndef MLKV_SORT_RANK_BALLOT
 #define MLKV_SORT_RANK_BALLOT 1
@@ -153,12 +154,14 @@ __device__ __forceinline__ uint32_t digit_peers(uint32_t dig, bool valid, int bi
 // added to the pass's digit totals dtot[d].  A thread counts 16 consecutive
 // elements and adds a run of equal digits with one atomic: after the first
 // pass a hot key's lookups are consecutive, and 32 lanes adding to one counter
-// would queue.
+// would queue.  In the first pass, a tile the probe has counted already
+// (dirty[tile] == 0) is skipped.
 __global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restrict__ kin, uint32_t n,
                                                         uint32_t* __restrict__ counts, uint32_t* __restrict__ dtot,
                                                         uint32_t ntiles, int shift, int radix, uint32_t sent,
-                                                        int first) {
+                                                        int first, const uint32_t* __restrict__ dirty) {
     pdl_enter();
+    if (dirty && dirty[blockIdx.x] == 0u) return;  // block-uniform
     __shared__ uint32_t hist[kMaxRadix];
     for (int d = threadIdx.x; d < radix; d += kThreads) hist[d] = 0;
     __syncthreads();
@@ -201,24 +204,34 @@ __global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restri
 
 // Output position of the first element of every (tile, digit): the elements
 // of all lower digits, plus those of digit d in earlier tiles; written to
-// offsets[tile][d].  A warp per digit: a warp-wide sum of the lower digits'
-// totals, then a scan of the digit's counts over the tiles, 32 tiles a round,
-// with the loads of 8 rounds issued together.
+// offsets[tile][d].  Each block first scans the pass's digit totals (all of
+// them, two per thread) for the elements of the lower digits; then a warp per
+// digit scans the digit's counts over the tiles, 32 tiles a round, with the
+// loads of 16 rounds issued together (every tile of a batch of up to 2M
+// lookups in one round trip).
 __global__ void __launch_bounds__(kThreads) k_sort_offsets(const uint32_t* __restrict__ counts,
                                                            const uint32_t* __restrict__ dtot,
                                                            uint32_t* __restrict__ offsets, uint32_t ntiles,
                                                            int radix) {
     pdl_enter();
-    constexpr int kRounds = 8;
+    static_assert(2 * kThreads == kMaxRadix, "two digit totals per thread");
+    constexpr int kRounds = 16;
+    __shared__ uint32_t lower[kMaxRadix];  // elements of the digits below each digit
+    {
+        const int i = 2 * threadIdx.x;
+        const uint32_t a = i < radix ? __ldg(dtot + i) : 0u;
+        const uint32_t b = i + 1 < radix ? __ldg(dtot + i + 1) : 0u;
+        uint32_t total;
+        const uint32_t ex = block_exclusive_scan(a + b, total);
+        lower[i] = ex;
+        lower[i + 1] = ex + a;
+    }
+    __syncthreads();
     const int lane = threadIdx.x & 31;
     const int d = blockIdx.x * kWarps + (threadIdx.x >> 5);
     if (d >= radix) return;  // warp-uniform
-    uint32_t below = 0;
-    for (int i = lane; i < d; i += 32) below += __ldg(dtot + i);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) below += __shfl_xor_sync(0xffffffffu, below, o);
     const uint32_t* row = counts + (size_t)d * ntiles;
-    uint32_t run = below;
+    uint32_t run = lower[d];
     for (uint32_t t0 = 0; t0 < ntiles; t0 += 32 * kRounds) {
         uint32_t c[kRounds];
 #pragma unroll
@@ -228,6 +241,7 @@ __global__ void __launch_bounds__(kThreads) k_sort_offsets(const uint32_t* __res
         }
 #pragma unroll
         for (int k = 0; k < kRounds; ++k) {
+            if (t0 + 32 * k >= ntiles) break;  // warp-uniform
             const uint32_t t = t0 + 32 * k + lane;
             uint32_t x = c[k];
 #pragma unroll
@@ -428,11 +442,27 @@ cudaError_t launch_exclusive_scan(mlkv_table* t, const uint32_t* in, uint32_t* o
     return cudaGetLastError();
 }
 
+namespace {
+// Passes and digit width for ids of `bits` bits: the fewest passes of at most
+// kSortMaxDigitBits bits, the bits spread evenly over them.
+void sort_geometry(int bits, int& passes, int& D) {
+    passes = (bits + kSortMaxDigitBits - 1) / kSortMaxDigitBits;
+    D = (bits + passes - 1) / passes;
+}
+}  // namespace
+
+FirstCounts first_counts(mlkv_table* t, int64_t n) {
+    int passes, D;
+    sort_geometry(t->sort_bits, passes, D);
+    return FirstCounts{t->s.sort_counts, t->s.sort_dtot, t->s.sort_dirty, tiles(n), 1 << D,
+                       (uint32_t)((1ull << t->sort_bits) - 1)};
+}
+
 cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow,
-                             const uint32_t** spos) {
+                             const uint32_t** spos, const uint32_t* first_dirty) {
     const int bits = t->sort_bits;
-    const int passes = (bits + kSortMaxDigitBits - 1) / kSortMaxDigitBits;
-    const int D = (bits + passes - 1) / passes;
+    int passes, D;
+    sort_geometry(bits, passes, D);
     const int radix = 1 << D;
     const uint32_t sent = (uint32_t)((1ull << bits) - 1);
     const unsigned nt = tiles(n);
@@ -446,7 +476,7 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
         const int first = p == 0;
         uint32_t* dtot = t->s.sort_dtot + p * kMaxRadix;
         MLKV_LAUNCH(t, 0, k_sort_hist, nt, kThreads, 0, st, kin, (uint32_t)n, counts, dtot, nt, p * D, radix,
-                    sent, first);
+                    sent, first, first ? first_dirty : nullptr);
         MLKV_LAUNCH(t, 0, k_sort_offsets, (unsigned)((radix + kWarps - 1) / kWarps), kThreads, 0, st, counts, dtot,
                     offsets, nt, radix);
         MLKV_LAUNCH(t, MLKV_K_SORT_SCATTER, k_sort_scatter, nt, kThreads, 0, st, kin, vin, t->s.sk[out],
