@@ -29,8 +29,10 @@ constexpr int kWarps = kThreads / 32;
 
 __device__ __forceinline__ int spad(int i) { return i + (i >> 5); }
 
-// Exclusive scan of one value per thread over a 256-thread block.
-__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t& total) {
+// Exclusive scan of one value per thread over a block of THREADS threads.
+template <int THREADS>
+__device__ __forceinline__ uint32_t block_exclusive_scan_n(uint32_t v, uint32_t& total) {
+    constexpr int kWarps = THREADS / 32;
     __shared__ uint32_t warp_sums[kWarps];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     uint32_t x = v;
@@ -55,6 +57,10 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t& t
     total = warp_sums[kWarps - 1];
     __syncthreads();
     return wprefix + x - v;
+}
+
+__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t& total) {
+    return block_exclusive_scan_n<kThreads>(v, total);
 }
 
 // Sum of tile_sums[0..b) by the whole block.
@@ -258,11 +264,20 @@ __global__ void __launch_bounds__(kThreads) k_sort_offsets(const uint32_t* __res
 // Stable rank of each element of the tile among equal digits; the tile is
 // then laid out in shared memory in sorted order and written out so that
 // consecutive threads write consecutive addresses of a digit's run (a direct
-// scatter from registers costs one L2 sector per element).  Warp w owns
-// elements w*512 .. w*512+511 of the tile, in rounds of 32 consecutive
-// elements.  An element of digit d goes to offsets[tile][d] plus its rank
+// scatter from registers costs one L2 sector per element).  The block has
+// kSThreads threads; warp w owns elements w*kSItems*32 .. of the tile, in
+// rounds of 32 consecutive elements (more warps a tile: fewer rounds each).  An element of digit d goes to offsets[tile][d] plus its rank
 // among the tile's elements of digit d.
-__global__ void __launch_bounds__(kThreads, 3) k_sort_scatter(const uint32_t* __restrict__ kin,
+#ifndef MLKV_SCATTER_THREADS
+#define MLKV_SCATTER_THREADS 512
+#endif
+#ifndef MLKV_SCATTER_MIN_BLOCKS
+#define MLKV_SCATTER_MIN_BLOCKS 3
+#endif
+constexpr int kSThreads = MLKV_SCATTER_THREADS;
+constexpr int kSWarps = kSThreads / 32;
+constexpr int kSItems = kTile / kSThreads;
+__global__ void __launch_bounds__(kSThreads, kSThreads == 256 ? 3 : MLKV_SCATTER_MIN_BLOCKS) k_sort_scatter(const uint32_t* __restrict__ kin,
                                                               const uint32_t* __restrict__ vin,
                                                               uint32_t* __restrict__ kout,
                                                               uint32_t* __restrict__ vout, uint32_t n,
@@ -272,30 +287,30 @@ __global__ void __launch_bounds__(kThreads, 3) k_sort_scatter(const uint32_t* __
     pdl_enter();
     // the per-warp digit counts, then (once every position is known) the sorted tile
     __shared__ uint32_t pool[2 * kTile];
-    static_assert(kWarps * kMaxRadix <= 2 * kTile, "counts fit the tile buffer");
+    static_assert(kSWarps * kMaxRadix <= 2 * kTile, "counts fit the tile buffer");
     uint32_t (*wcnt)[kMaxRadix] = reinterpret_cast<uint32_t (*)[kMaxRadix]>(pool);
     uint32_t* skey = pool;
     uint32_t* sval = pool + kTile;
     __shared__ uint32_t gbase[kMaxRadix];   // output position of the tile's first element of each digit
     __shared__ uint32_t lbase[kMaxRadix];   // position in the sorted tile of its first element of each digit
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    for (int i = threadIdx.x; i < kWarps * kMaxRadix; i += kThreads) (&wcnt[0][0])[i] = 0;
-    for (int d = threadIdx.x; d < radix; d += kThreads) gbase[d] = offsets[(size_t)blockIdx.x * radix + d];
+    for (int i = threadIdx.x; i < kSWarps * kMaxRadix; i += kSThreads) (&wcnt[0][0])[i] = 0;
+    for (int d = threadIdx.x; d < radix; d += kSThreads) gbase[d] = offsets[(size_t)blockIdx.x * radix + d];
     __syncthreads();
     const uint32_t tile0 = blockIdx.x * kTile;
-    const uint32_t base = tile0 + w * (kItems * 32);
+    const uint32_t base = tile0 + w * (kSItems * 32);
     const int digit_bits = __ffs(radix) - 1;
     const uint32_t lt = lanemask_lt();
-    uint32_t key[kItems], val[kItems], rnk[kItems];
+    uint32_t key[kSItems], val[kSItems], rnk[kSItems];
     // all loads first, so they are in flight together
 #pragma unroll
-    for (int r = 0; r < kItems; ++r) {
+    for (int r = 0; r < kSItems; ++r) {
         const uint32_t i = base + r * 32 + lane;
         key[r] = i < n ? sort_key(kin[i], sent, first) : 0u;
         val[r] = i < n ? (first ? i : vin[i]) : 0u;
     }
 #pragma unroll
-    for (int r = 0; r < kItems; ++r) {
+    for (int r = 0; r < kSItems; ++r) {
         const bool valid = base + r * 32 + lane < n;
         const uint32_t dig = (key[r] >> shift) & (radix - 1);
         const uint32_t peers = digit_peers(dig, valid, digit_bits);
@@ -309,15 +324,15 @@ __global__ void __launch_bounds__(kThreads, 3) k_sort_scatter(const uint32_t* __
     __syncthreads();
     // per digit: exclusive prefix over the warps; per tile: exclusive prefix
     // over the digits (thread t owns digits t*dpt .. t*dpt+dpt-1, in order)
-    const int dpt = radix > kThreads ? radix / kThreads : 1;
-    uint32_t tot[kMaxRadix / kThreads], mine = 0;
+    const int dpt = radix > kSThreads ? radix / kSThreads : 1;
+    uint32_t tot[kMaxRadix / kSThreads], mine = 0;
 #pragma unroll
-    for (int j = 0; j < kMaxRadix / kThreads; ++j) {
+    for (int j = 0; j < kMaxRadix / kSThreads; ++j) {
         const int d = threadIdx.x * dpt + j;
         tot[j] = 0;
         if (j >= dpt || d >= radix) continue;
 #pragma unroll
-        for (int ww = 0; ww < kWarps; ++ww) {
+        for (int ww = 0; ww < kSWarps; ++ww) {
             const uint32_t c = wcnt[ww][d];
             wcnt[ww][d] = tot[j];
             tot[j] += c;
@@ -325,9 +340,9 @@ __global__ void __launch_bounds__(kThreads, 3) k_sort_scatter(const uint32_t* __
         mine += tot[j];
     }
     uint32_t all;
-    uint32_t run = block_exclusive_scan(mine, all);
+    uint32_t run = block_exclusive_scan_n<kSThreads>(mine, all);
 #pragma unroll
-    for (int j = 0; j < kMaxRadix / kThreads; ++j) {
+    for (int j = 0; j < kMaxRadix / kSThreads; ++j) {
         const int d = threadIdx.x * dpt + j;
         if (j >= dpt || d >= radix) continue;
         lbase[d] = run;
@@ -335,21 +350,21 @@ __global__ void __launch_bounds__(kThreads, 3) k_sort_scatter(const uint32_t* __
     }
     __syncthreads();
 #pragma unroll
-    for (int r = 0; r < kItems; ++r) {
+    for (int r = 0; r < kSItems; ++r) {
         if (rnk[r] == 0xFFFFFFFFu) continue;
         const uint32_t dig = (key[r] >> shift) & (radix - 1);
         rnk[r] += lbase[dig] + wcnt[w][dig];  // position in the sorted tile
     }
     __syncthreads();  // the counts are dead: the buffer takes the sorted tile
 #pragma unroll
-    for (int r = 0; r < kItems; ++r) {
+    for (int r = 0; r < kSItems; ++r) {
         if (rnk[r] == 0xFFFFFFFFu) continue;
         skey[rnk[r]] = key[r];
         sval[rnk[r]] = val[r];
     }
     __syncthreads();
     const uint32_t cnt = n - tile0 < (uint32_t)kTile ? n - tile0 : (uint32_t)kTile;
-    for (uint32_t l = threadIdx.x; l < cnt; l += kThreads) {
+    for (uint32_t l = threadIdx.x; l < cnt; l += kSThreads) {
         const uint32_t k = skey[l];
         const uint32_t dig = (k >> shift) & (radix - 1);
         const uint32_t dst = gbase[dig] + (l - lbase[dig]);
@@ -479,7 +494,7 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
                     sent, first, first ? first_dirty : nullptr);
         MLKV_LAUNCH(t, 0, k_sort_offsets, (unsigned)((radix + kWarps - 1) / kWarps), kThreads, 0, st, counts, dtot,
                     offsets, nt, radix);
-        MLKV_LAUNCH(t, MLKV_K_SORT_SCATTER, k_sort_scatter, nt, kThreads, 0, st, kin, vin, t->s.sk[out],
+        MLKV_LAUNCH(t, MLKV_K_SORT_SCATTER, k_sort_scatter, nt, kSThreads, 0, st, kin, vin, t->s.sk[out],
                     t->s.sv[out], (uint32_t)n, offsets, nt, p * D, radix, sent, first);
         kin = t->s.sk[out];
         vin = t->s.sv[out];
