@@ -92,16 +92,18 @@ __device__ __forceinline__ unsigned group_mask(int G, int gid) {
 
 // acc += the gradient rows of sorted positions s .. s+len-1, in that order.
 // The group loads up to G positions at a time (one per lane) and hands them
-// round with group shuffles.
-template <int V, int KV, int ROWS = MLKV_REDUCE_ROWS_IN_FLIGHT>
+// round with group shuffles.  With PRE the first G positions were loaded by
+// the caller (pl_first, one per lane).
+template <int V, int KV, int ROWS = MLKV_REDUCE_ROWS_IN_FLIGHT, bool PRE = false>
 __device__ __forceinline__ void sum_rows(typename Vec<V>::T (&acc)[KV], const float* __restrict__ grads,
                                          const uint32_t* __restrict__ spos, uint32_t s, uint32_t len, int d,
-                                         int NV, int G, int glane, unsigned gmask) {
+                                         int NV, int G, int glane, unsigned gmask, uint32_t pl_first = 0u) {
     using VT = typename Vec<V>::T;
     constexpr int UNR = KV >= ROWS ? 1 : ROWS / KV;
     for (uint32_t base = 0; base < len; base += G) {
         const uint32_t cnt = min((uint32_t)G, len - base);
-        const uint32_t pl = (uint32_t)glane < cnt ? __ldg(spos + s + base + glane) : 0u;
+        const uint32_t pl = (PRE && base == 0) ? pl_first
+                            : (uint32_t)glane < cnt ? __ldg(spos + s + base + glane) : 0u;
         for (uint32_t x = 0; x < cnt; x += UNR) {
             VT g[UNR][KV];
 #pragma unroll
@@ -265,6 +267,10 @@ __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, u
                                           uint32_t row, uint32_t p0, int glane, unsigned gmask) {
     using VT = typename Vec<V>::T;
     VT w[KV], Gs[KV], acc[KV];
+    // the positions of the run's other lookups load beside its row, state and
+    // first gradient row, so a run of a few lookups costs two round trips
+    const uint32_t rest = len - 1;
+    const uint32_t pl0 = (uint32_t)glane < min(rest, (uint32_t)ra.G) ? __ldg(a.spos + s + 1 + glane) : 0u;
     load_row_state<V, KV>(ra, row, w, Gs, glane);
     const VT* g0 = reinterpret_cast<const VT*>(a.grads + (size_t)p0 * ra.d);
 #pragma unroll
@@ -273,7 +279,9 @@ __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, u
         const int j = glane + ra.G * k;
         if (j < ra.NV) Vec<V>::add(acc[k], __ldcs(g0 + j));  // 0 + g: first term, in order
     }
-    if (len > 1) sum_rows<V, KV>(acc, a.grads, a.spos, s + 1, len - 1, ra.d, ra.NV, ra.G, glane, gmask);
+    if (len > 1)
+        sum_rows<V, KV, MLKV_REDUCE_ROWS_IN_FLIGHT, true>(acc, a.grads, a.spos, s + 1, rest, ra.d, ra.NV, ra.G,
+                                                          glane, gmask, pl0);
     adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
 }
 
