@@ -142,15 +142,20 @@ def batch_stats(keys: np.ndarray, d: int) -> dict:
     long_ = counts > SEQ_SEGMENT_MAX
     Bl, Ul = int(counts[long_].sum()), int(long_.sum())
     Bs, Us = B - Bl, U - Ul
+    U1 = int((counts == 1).sum())  # runs of one lookup (k_single)
+    Bm, Um = Bs - U1, Us - U1      # the other short runs (k_short)
     items = int(np.ceil(counts[long_] / CHUNK).sum())
     row = 4 * d
     return {
-        "B": B, "U": U, "Bs": Bs, "Us": Us, "Bl": Bl, "Ul": Ul, "items": items,
+        "B": B, "U": U, "Bs": Bs, "Us": Us, "Bl": Bl, "Ul": Ul, "items": items, "U1": U1, "Um": Um,
         # Get: keys + output per lookup; index sector + row per distinct key
         "get_gather": B * (8 + row) + U * (32 + row),
-        # short runs: gradient rows + sorted position per lookup; row and state
-        # read and written once plus the run's bounds, row and first position
-        "reduce_short": Bs * (row + 4) + Us * (4 * row + 16),
+        # short runs of 2+ lookups: gradient rows + sorted position per lookup;
+        # row and state read and written once plus the run's 16-byte record
+        "reduce_short": Bm * (row + 4) + Um * (4 * row + 16),
+        # runs of one lookup: the gradient row, row and state read and written
+        # once, the 8-byte record
+        "reduce_single": U1 * (row + 4 * row + 8),
         # long runs: gradient rows + sorted positions, chunk sums written
         "reduce_long": Bl * (row + 4) + items * row,
         # chunk sums read, row and state read and written once per long run
@@ -182,6 +187,8 @@ def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
         return stats["get_gather"]
     if kid == 4:
         return stats["reduce_short"]
+    if kid == 10:
+        return stats["reduce_single"]
     if kid == 5:
         return stats["reduce_long"]
     if kid == 7:
@@ -190,18 +197,19 @@ def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
         return stats["B"] * 16.0  # per pass: (row id, position) read and written
     if kid == 2:
         return stats["B"] * 12.0 + stats["U"] * 32.0
-    if kid == 6:  # each sorted row id read twice, short-run records written
-        return stats["B"] * 8.0 + stats["Us"] * 20.0
+    if kid == 6:  # each sorted row id read twice, run records written (with the run's first position)
+        return stats["B"] * 8.0 + stats["Um"] * 20.0 + stats["U1"] * 12.0
     return 0.0
 
 
 KERNEL_NAMES = {1: "k_get (probe + row gather)", 2: "k_probe", 3: "k_sort_scatter",
                 4: "k_short (run sum + Adagrad)", 5: "k_long_sum (chunk sums of long runs)",
                 6: "k_heads (runs found in the sorted ids)", 7: "k_long_combine (chunk sums + Adagrad)",
-                8: "k_tier_fetch (host <-> HBM row swap)", 9: "k_put_scatter (Put: last occurrence writes)"}
+                8: "k_tier_fetch (host <-> HBM row swap)", 9: "k_put_scatter (Put: last occurrence writes)",
+                10: "k_single (runs of one lookup + Adagrad)"}
 KERNEL_SOURCES = {1: "mlkv_index.cu", 2: "mlkv_index.cu", 3: "mlkv_sort.cu", 4: "mlkv_apply.cu",
                   5: "mlkv_apply.cu", 6: "mlkv_apply.cu", 7: "mlkv_apply.cu", 8: "mlkv_tier.cu",
-                  9: "mlkv_index.cu"}
+                  9: "mlkv_index.cu", 10: "mlkv_apply.cu"}
 
 
 def traffic_for(kid: int):
@@ -396,7 +404,7 @@ def run_ours(args, cfg):
     # The HBM store cycles a pool of batches.  The tiered store gets a fresh batch
     # every step (a cycled pool would end up resident in its cache): one per
     # kernel-class prepass step, warm-up step, timed step, and the last look-ahead.
-    kinds = (1, 2, 9) if kv else (1, 2, 3, 4, 5, 6, 7) + ((8,) if tiered else ())
+    kinds = (1, 2, 9) if kv else (1, 2, 3, 4, 5, 6, 7, 10) + ((8,) if tiered else ())
     base = len(kinds) if tiered else 0
     pool = base + args.warmup + args.steps + 1 if tiered else max(1, min(args.pool, args.steps + args.warmup))
     ngrad = max(1, min(args.pool, pool))

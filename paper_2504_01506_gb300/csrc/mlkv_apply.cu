@@ -47,6 +47,13 @@ constexpr uint32_t kBigRun = 32;
 #ifndef MLKV_SHORT_MIN_BLOCKS
 #define MLKV_SHORT_MIN_BLOCKS 4
 #endif
+// k_single: runs of one lookup in flight per lane group, and blocks per SM.
+#ifndef MLKV_SINGLES
+#define MLKV_SINGLES 1
+#endif
+#ifndef MLKV_SINGLE_MIN_BLOCKS
+#define MLKV_SINGLE_MIN_BLOCKS 6
+#endif
 #ifndef MLKV_LONG_ROWS_IN_FLIGHT
 #define MLKV_LONG_ROWS_IN_FLIGHT 8
 #endif
@@ -70,8 +77,9 @@ struct RunArgs {
     uint32_t n;
     uint32_t sent;
     CallCounters* cur;
-    uint4* runs;           // [max_batch] short runs: (first sorted position, one past the last, row,
-                           //   first lookup position)
+    uint4* runs;           // [max_batch] short runs of 2 or more lookups: (first sorted position, one
+                           //   past the last, row, first lookup position)
+    uint2* singles;        // [max_batch] runs of one lookup: (row, lookup position)
     uint32_t* long_s;      // [max_long] first sorted position
     uint32_t* long_e;      // [max_long] one past the last
     uint32_t* long_row;    // [max_long]
@@ -295,28 +303,34 @@ __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, u
 // reserves room in the short-run list, the long-run list and the chunk list
 // with one atomic each and the warps copy their runs out.  (Counters that
 // every warp bumps queue up at the end of the kernel.)
-__global__ void __launch_bounds__(256) k_heads(RunArgs a) {
+__global__ void __launch_bounds__(256, 5) k_heads(RunArgs a) {
     pdl_enter();
     constexpr int kList = 128, kQueue = 16;
     __shared__ uint4 lst[8][kList];  // (start, end, row, first lookup) of short runs
+    __shared__ uint2 sgl[8][kList];  // (row, lookup) of runs of one lookup
     __shared__ uint32_t qs[8][kQueue], qr[8][kQueue], qe[8][kQueue];  // long runs: start, row, end (0: unknown)
-    __shared__ uint32_t wsh[8], wlg[8], wit[8];  // per warp: short runs, long runs, chunks; then their bases
+    __shared__ uint32_t wsh[8], wlg[8], wit[8], ws1[8];  // per warp: short runs, long runs, chunks,
+                                                         // runs of one lookup; then their bases
     const uint32_t n = a.n, sent = a.sent;
     const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
     const uint32_t lt = lanemask_lt();
     const uint32_t warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t nwarps = (gridDim.x * blockDim.x) >> 5;
     const uint32_t nwin = (n + 31) >> 5;
-    int cnt = 0, nq = 0;  // warp-uniform
-    // a full list or queue goes out at once (only batches far above a few
+    int cnt = 0, cnt1 = 0, nq = 0;  // warp-uniform
+    // full lists or a full queue go out at once (only batches far above a few
     // runs per window and warp get here)
     auto flush = [&]() {
         __syncwarp();
-        uint32_t base = 0;
+        uint32_t base = 0, base1 = 0;
         if (lane == 0 && cnt) base = atomicAdd(&a.cur->n_short, (uint32_t)cnt);
+        if (lane == 0 && cnt1) base1 = atomicAdd(&a.cur->n_single, (uint32_t)cnt1);
         base = __shfl_sync(0xffffffffu, base, 0);
+        base1 = __shfl_sync(0xffffffffu, base1, 0);
         for (int k = lane; k < cnt; k += 32) a.runs[base + k] = lst[wib][k];
+        for (int k = lane; k < cnt1; k += 32) a.singles[base1 + k] = sgl[wib][k];
         cnt = 0;
+        cnt1 = 0;
         __syncwarp();
     };
     auto measure = [&]() {  // fills in the unknown ends of the queued long runs
@@ -368,10 +382,14 @@ __global__ void __launch_bounds__(256) k_heads(RunArgs a) {
             else lng = true;
             lng = lng || len > MLKV_SEQ_SEGMENT_MAX;
         }
-        const unsigned sm = __ballot_sync(0xffffffffu, head && !lng);
-        if (cnt + __popc(sm) > kList) flush();
-        if (head && !lng) lst[wib][cnt + __popc(sm & lt)] = make_uint4(p, p + len, r, pos);
+        const bool shrt = head && !lng;  // len >= 1
+        const unsigned sm = __ballot_sync(0xffffffffu, shrt && len > 1);
+        const unsigned s1 = __ballot_sync(0xffffffffu, shrt && len == 1);
+        if (cnt + __popc(sm) > kList || cnt1 + __popc(s1) > kList) flush();
+        if (shrt && len > 1) lst[wib][cnt + __popc(sm & lt)] = make_uint4(p, p + len, r, pos);
+        if (shrt && len == 1) sgl[wib][cnt1 + __popc(s1 & lt)] = make_uint2(r, pos);
         cnt += __popc(sm);
+        cnt1 += __popc(s1);
         for (unsigned lm = __ballot_sync(0xffffffffu, head && lng); lm; lm &= lm - 1) {
             const int i = __ffs(lm) - 1;
             if (nq == kQueue) {
@@ -408,30 +426,36 @@ __global__ void __launch_bounds__(256) k_heads(RunArgs a) {
         wsh[wib] = (uint32_t)cnt;
         wlg[wib] = (uint32_t)nq;
         wit[wib] = items;
+        ws1[wib] = (uint32_t)cnt1;
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-        uint32_t ts = 0, tl = 0, ti = 0;
+        uint32_t ts = 0, tl = 0, ti = 0, t1 = 0;
         for (int k = 0; k < 8; ++k) {
             ts += wsh[k];
             tl += wlg[k];
             ti += wit[k];
+            t1 += ws1[k];
         }
         uint32_t bs = ts ? atomicAdd(&a.cur->n_short, ts) : 0u;
         uint32_t bl = tl ? atomicAdd(&a.cur->n_long, tl) : 0u;
         uint32_t bi = ti ? atomicAdd(&a.cur->n_items, ti) : 0u;
+        uint32_t b1 = t1 ? atomicAdd(&a.cur->n_single, t1) : 0u;
         for (int k = 0; k < 8; ++k) {
-            const uint32_t c0 = wsh[k], c1 = wlg[k], c2 = wit[k];
+            const uint32_t c0 = wsh[k], c1 = wlg[k], c2 = wit[k], c3 = ws1[k];
             wsh[k] = bs;
             wlg[k] = bl;
             wit[k] = bi;
+            ws1[k] = b1;
             bs += c0;
             bl += c1;
             bi += c2;
+            b1 += c3;
         }
     }
     __syncthreads();
     for (int k = lane; k < cnt; k += 32) a.runs[wsh[wib] + k] = lst[wib][k];
+    for (int k = lane; k < cnt1; k += 32) a.singles[ws1[wib] + k] = sgl[wib][k];
     if (wlg[wib] + nq > a.max_long || wit[wib] + items > a.max_items) {
         if (lane == 0 && nq) record_error(a.err, MLKV_ERR_FULL);
         return;
@@ -460,6 +484,58 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
         const uint4 m = next;  // (start, end, row, first lookup)
         next = run_meta(a, u + ngroups, U);
         short_run<V, KV>(ra, a, m.x, m.y - m.x, m.z, m.w, glane, gmask);
+    }
+}
+
+// One lane group per run of one lookup (most runs of a Zipf batch): its row,
+// state and gradient row, SINGLES runs at a time, records loaded one round
+// ahead; the sum is the gradient row itself (0 + g), then the Adagrad step.
+// With no loop over positions it needs few registers, so more warps (and
+// rows) are in flight than in k_short.
+template <int V, int KV>
+__global__ void __launch_bounds__(256, MLKV_SINGLE_MIN_BLOCKS) k_single(RowArgs ra, RunArgs a) {
+    pdl_enter();
+    using VT = typename Vec<V>::T;
+    constexpr int SG = MLKV_SINGLES;
+    const uint32_t U = a.cur->n_single;
+    const int lane = threadIdx.x & 31, G = ra.G, glane = lane & (G - 1);
+    const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
+    const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
+    const uint2 none = make_uint2(0xFFFFFFFFu, 0u);
+    uint2 next[SG];
+#pragma unroll
+    for (int j = 0; j < SG; ++j) next[j] = group * SG + j < U ? __ldg(a.singles + group * SG + j) : none;
+    for (uint32_t u = group * SG; u < U; u += ngroups * SG) {  // uniform within the group
+        uint2 m[SG];
+#pragma unroll
+        for (int j = 0; j < SG; ++j) {
+            m[j] = next[j];
+            const uint32_t v = u + ngroups * SG + j;
+            next[j] = v < U ? __ldg(a.singles + v) : none;
+        }
+        VT w[SG][KV], Gs[SG][KV], g[SG][KV];
+#pragma unroll
+        for (int j = 0; j < SG; ++j) {
+            if (m[j].x == 0xFFFFFFFFu) continue;
+            load_row_state<V, KV>(ra, m[j].x, w[j], Gs[j], glane);
+            const VT* src = reinterpret_cast<const VT*>(a.grads + (size_t)m[j].y * ra.d);
+#pragma unroll
+            for (int k = 0; k < KV; ++k) {
+                const int jj = glane + G * k;
+                if (jj < ra.NV) g[j][k] = __ldcs(src + jj);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < SG; ++j) {
+            if (m[j].x == 0xFFFFFFFFu) continue;
+            VT acc[KV];
+#pragma unroll
+            for (int k = 0; k < KV; ++k) {
+                acc[k] = Vec<V>::zero();
+                if (glane + G * k < ra.NV) Vec<V>::add(acc[k], g[j][k]);  // 0 + g, as in a longer run
+            }
+            adagrad_store<V, KV>(ra, m[j].x, w[j], Gs[j], acc, glane, a.lr, a.eps);
+        }
     }
 }
 
@@ -525,7 +601,8 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
     using VT = typename Vec<V>::T;
     extern __shared__ float sh[];  // [groups][dpad]
     const uint32_t nl = min(a.cur->n_long, a.max_long), nb = a.cur->n_big;
-    if (blockIdx.x == 0 && threadIdx.x == 0) ds->last_unique = a.cur->n_short + a.cur->n_long;  // one run per row
+    if (blockIdx.x == 0 && threadIdx.x == 0)
+        ds->last_unique = a.cur->n_single + a.cur->n_short + a.cur->n_long;  // one run per row
     const int G = ra.G, glane = threadIdx.x & (G - 1);
     const int group = threadIdx.x / G;
     const int ngroups = blockDim.x / G;
@@ -582,7 +659,7 @@ template <int V, int KV>
 cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, const uint32_t* spos,
                        int64_t n, uint32_t sent, cudaStream_t st, CallCounters* cur) {
     RowArgs ra{t->slots, t->geom.stride, t->geom.dpad, t->geom.NV, t->geom.G, t->geom.d};
-    RunArgs a{grads, srow, spos, (uint32_t)n, sent, cur, t->s.short_runs, t->s.long_s, t->s.long_e,
+    RunArgs a{grads, srow, spos, (uint32_t)n, sent, cur, t->s.short_runs, t->s.single_runs, t->s.long_s, t->s.long_e,
               t->s.long_row, t->s.long_base, t->s.item_s, t->s.item_e, t->s.big_runs, t->s.partial,
               (uint32_t)t->s.max_long,
               (uint32_t)t->s.max_items, ErrSink{&t->dstate->status, t->status_dev_alias}, t->cfg.lr, t->cfg.eps};
@@ -590,6 +667,8 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     if (gh > (int64_t)t->num_sms * 8) gh = (int64_t)t->num_sms * 8;
     if (gh < 1) gh = 1;
     MLKV_LAUNCH(t, MLKV_K_SEGMENTS, k_heads, (unsigned)gh, 256, 0, st, a);
+    const int g1 = persistent_blocks(t, (const void*)k_single<V, KV>, 256);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, st, ra, a);
     const int gs = persistent_blocks(t, (const void*)k_short<V, KV>, 256);
     MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, st, ra, a);
     const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);

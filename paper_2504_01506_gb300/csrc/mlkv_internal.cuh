@@ -42,6 +42,7 @@ struct CallCounters {
     uint32_t n_items;    // chunks of the long runs
     uint32_t n_short;    // runs of at most MLKV_SEQ_SEGMENT_MAX lookups
     uint32_t n_big;      // long runs whose chunk sums are combined by the wide blocks
+    uint32_t n_single;   // runs of one lookup
 };
 
 struct DevState {
@@ -86,7 +87,8 @@ struct Scratch {
     uint32_t* seg_start;    // [max_batch + 1] run starts in sorted order (dedup)
     uint32_t* run_row;      // [max_batch] row of each run (dedup)
     uint32_t* run_p0;       // [max_batch] first lookup position of each run (dedup)
-    uint4* short_runs;      // [max_batch] the apply's runs of <= MLKV_SEQ_SEGMENT_MAX lookups
+    uint4* short_runs;      // [max_batch] the apply's runs of 2 .. MLKV_SEQ_SEGMENT_MAX lookups
+    uint2* single_runs;     // [max_batch] its runs of one lookup: (row, lookup position)
     uint32_t* long_s;       // [max_long] long runs: first sorted position
     uint32_t* long_e;       // [max_long] one past the last
     uint32_t* long_row;     // [max_long]
