@@ -39,13 +39,10 @@ constexpr uint32_t kBigRun = 32;
 // Tuning (set at build time): gradient rows in flight per lane group, and the
 // minimum resident blocks per SM the register allocation must allow.
 #ifndef MLKV_REDUCE_ROWS_IN_FLIGHT
-#define MLKV_REDUCE_ROWS_IN_FLIGHT 4
-#endif
-#ifndef MLKV_REDUCE_MIN_BLOCKS
-#define MLKV_REDUCE_MIN_BLOCKS 5
+#define MLKV_REDUCE_ROWS_IN_FLIGHT 8
 #endif
 #ifndef MLKV_SHORT_MIN_BLOCKS
-#define MLKV_SHORT_MIN_BLOCKS 4
+#define MLKV_SHORT_MIN_BLOCKS 2
 #endif
 // k_single: runs of one lookup in flight per lane group, and blocks per SM.
 #ifndef MLKV_SINGLES
