@@ -125,8 +125,7 @@ __global__ void __launch_bounds__(COUNT ? 1024 : 256) k_probe(IndexArgs ia, cons
                                                uint32_t* miss_pos, uint32_t* miss_slot,
                                                CallCounters* cur, CallCounters* nxt,
                                                int report_absent, Memo memo, int memo_use, FirstCounts fc) {
-    constexpr int KEYS = kProbeKeys;
-    static_assert(KEYS * 1024 == kSortTile, "a counting block covers one sort tile");
+    static_assert(kProbeKeys * 1024 == kSortTile, "a counting block covers one sort tile");
     pdl_enter();
     zero_counters(nxt);
     __shared__ uint32_t hist[COUNT ? kSortMaxRadix : 1];
@@ -135,42 +134,39 @@ __global__ void __launch_bounds__(COUNT ? 1024 : 256) k_probe(IndexArgs ia, cons
         __syncthreads();
     }
     bool missed = false;  // a lookup of this thread waits for the miss path for its row
-    const uint32_t base = blockIdx.x * (blockDim.x * KEYS) + threadIdx.x;
-#pragma unroll 1
-    for (int j0 = 0; j0 < KEYS; j0 += kProbeKeys) {
-        unsigned long long k[kProbeKeys];
-        uint32_t known[kProbeKeys];
+    const uint32_t base = blockIdx.x * (blockDim.x * kProbeKeys) + threadIdx.x;
+    unsigned long long k[kProbeKeys];
+    uint32_t known[kProbeKeys];
 #pragma unroll
-        for (int j = 0; j < kProbeKeys; ++j) {
-            const uint32_t p = base + (j0 + j) * blockDim.x;
-            k[j] = p < n ? (unsigned long long)__ldg(keys + p) : 0ull;
-            known[j] = ROW_PENDING;
-            if (memo_use == (int)MemoUse::Read && p < n) {
-                const uint32_t r = memo.row[p];  // loaded beside the key it belongs to
-                if ((unsigned long long)memo.key[p] == k[j]) known[j] = r;
+    for (int j = 0; j < kProbeKeys; ++j) {
+        const uint32_t p = base + j * blockDim.x;
+        k[j] = p < n ? (unsigned long long)__ldg(keys + p) : 0ull;
+        known[j] = ROW_PENDING;
+        if (memo_use == (int)MemoUse::Read && p < n) {
+            const uint32_t r = memo.row[p];  // loaded beside the key it belongs to
+            if ((unsigned long long)memo.key[p] == k[j]) known[j] = r;
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < kProbeKeys; ++j) {
+        const uint32_t p = base + j * blockDim.x;
+        if (p >= n) continue;
+        uint32_t row = known[j];
+        if (row >= ROW_ABSENT) {  // not the row the last Get found for this key here: probe
+            uint32_t slot = 0;
+            row = probe_key<INSERT>(ia, k[j], p, slot);
+            if (!INSERT && report_absent && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
+            if (slot_of_pos) slot_of_pos[p] = slot;
+            if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
+            if (memo_use == (int)MemoUse::Save) {
+                memo.key[p] = (int64_t)k[j];
+                memo.row[p] = row;
             }
         }
-#pragma unroll
-        for (int j = 0; j < kProbeKeys; ++j) {
-            const uint32_t p = base + (j0 + j) * blockDim.x;
-            if (p >= n) continue;
-            uint32_t row = known[j];
-            if (row >= ROW_ABSENT) {  // not the row the last Get found for this key here: probe
-                uint32_t slot = 0;
-                row = probe_key<INSERT>(ia, k[j], p, slot);
-                if (!INSERT && report_absent && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
-                if (slot_of_pos) slot_of_pos[p] = slot;
-                if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
-                if (memo_use == (int)MemoUse::Save) {
-                    memo.key[p] = (int64_t)k[j];
-                    memo.row[p] = row;
-                }
-            }
-            row_of_pos[p] = row;
-            if (COUNT) {
-                if (row == ROW_PENDING) missed = true;
-                else atomicAdd(&hist[(row >= ROW_ABSENT ? fc.sent : row) & (uint32_t)(fc.radix - 1)], 1u);
-            }
+        row_of_pos[p] = row;
+        if (COUNT) {
+            if (row == ROW_PENDING) missed = true;
+            else atomicAdd(&hist[(row >= ROW_ABSENT ? fc.sent : row) & (uint32_t)(fc.radix - 1)], 1u);
         }
     }
     if (COUNT) {

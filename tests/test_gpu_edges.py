@@ -3,6 +3,7 @@ every error is a status the kernels record and the host reads)."""
 import numpy as np
 import pytest
 
+import oracle
 import workloads as W
 from gpu_helpers import assert_bits, dev, host, make_pair, torch_cuda
 
@@ -47,6 +48,47 @@ def test_single_lookup():
     store.apply_grad(dev(k), dev(g))
     ref.apply_grad(k, g)
     assert_bits(host(store.export(dev(k))[0]), ref.export(k)[0], "single apply")
+
+
+@pytest.mark.parametrize("shape", ["all_distinct", "one_key", "every_length", "no_singletons"])
+def test_run_length_mixes(shape):
+    """Batches made only of runs of one lookup, of one long run, of runs of
+    every length 1..40 (singletons, short runs, the 32/33 boundary, long
+    runs) and of no singletons at all: rows and state against the oracle, and
+    the apply's count of distinct rows (last_unique) against the batch's."""
+    cfg = _small(dim=16)
+    store, ref = make_pair(cfg, capacity=8192, max_batch=4096)
+    rng = np.random.default_rng(11)
+    if shape == "all_distinct":
+        keys = rng.permutation(4096).astype(np.int64) * 7 + 3
+    elif shape == "one_key":
+        keys = np.full(4096, 99, np.int64)
+    elif shape == "every_length":
+        keys = np.concatenate([np.full(m, 1000 + m, np.int64) for m in range(1, 41)])
+    else:
+        keys = np.repeat(np.arange(2000, dtype=np.int64) * 5 + 1, 2)
+    keys = keys[rng.permutation(len(keys))]  # occurrences scattered over the batch
+    grads = (rng.standard_normal((len(keys), cfg.dim)) * 0.01).astype(np.float32)
+    store.get(dev(keys))
+    ref.get(keys)
+    store.apply_grad(dev(keys), dev(grads))
+    ref.apply_grad(keys, grads)
+    assert store.sync() == 0
+    u, c = np.unique(keys, return_counts=True)
+    assert store.last_unique() == len(u)
+    w, G = store.export(dev(u))
+    rw, rG = ref.export(u)
+    short = c <= 32  # summed in occurrence order: the oracle's op sequence, bit for bit
+    assert_bits(host(w)[short], rw[short], f"{shape}: rows of short-run keys")
+    assert_bits(host(G)[short], rG[short], f"{shape}: state of short-run keys")
+    if (~short).any():
+        ref64 = oracle.Table(cfg.dim, lr=cfg.lr, eps=cfg.eps, state_init=cfg.state_init, init_lo=cfg.init_lo,
+                             init_hi=cfg.init_hi, seed=cfg.seed, precision=64)
+        ref64.get(keys)
+        ref64.apply_grad(keys, grads)
+        lw, lG = ref64.export(u[~short])
+        tol = lambda got, want: np.abs(got - want) <= 1e-5 * (1 + np.abs(want))
+        assert tol(host(w)[~short], lw).all() and tol(host(G)[~short], lG).all()
 
 
 def test_not_found_without_insert():
