@@ -660,8 +660,14 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
               t->s.long_row, t->s.long_base, t->s.item_s, t->s.item_e, t->s.big_runs, t->s.partial,
               (uint32_t)t->s.max_long,
               (uint32_t)t->s.max_items, ErrSink{&t->dstate->status, t->status_dev_alias}, t->cfg.lr, t->cfg.eps};
-    int64_t gh = (n + 255) / 256;  // a warp per 32 positions, at most 8 blocks per SM
-    if (gh > (int64_t)t->num_sms * 8) gh = (int64_t)t->num_sms * 8;
+    // a warp per 32 positions, the windows dealt out grid-stride over at most
+    // one wave of blocks
+#ifndef MLKV_HEADS_ONE_WAVE
+#define MLKV_HEADS_ONE_WAVE 1
+#endif
+    const int64_t cap = MLKV_HEADS_ONE_WAVE ? persistent_blocks(t, (const void*)k_heads, 256) : (int64_t)t->num_sms * 8;
+    int64_t gh = (n + 255) / 256;
+    if (gh > cap) gh = cap;
     if (gh < 1) gh = 1;
     MLKV_LAUNCH(t, MLKV_K_SEGMENTS, k_heads, (unsigned)gh, 256, 0, st, a);
     const int g1 = persistent_blocks(t, (const void*)k_single<V, KV>, 256);

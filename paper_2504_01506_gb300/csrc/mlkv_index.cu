@@ -518,7 +518,7 @@ struct GetRun {
 // miss count; set at build time).  In steady-state training nothing misses and
 // they return at once, at a cost that grows with the blocks launched.
 #ifndef MLKV_MISS_BLOCKS_PER_SM
-#define MLKV_MISS_BLOCKS_PER_SM 8
+#define MLKV_MISS_BLOCKS_PER_SM 4
 #endif
 
 template <int V, int KV>
