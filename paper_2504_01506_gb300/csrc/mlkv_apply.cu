@@ -10,21 +10,26 @@
 //
 //  k_heads        a warp per window of 32 sorted positions finds the runs
 //                 that start there (a row id unlike its left neighbour) and
-//                 their lengths; runs of <= MLKV_SEQ_SEGMENT_MAX lookups are
-//                 appended to a list with one atomic per warp (any order: every
-//                 run is summed on its own), longer ones are measured (a
-//                 warp-wide search for their end) and listed for k_long_*.
-//  k_short        one lane group per listed run: the row, the state and the
-//                 first gradient row are loaded together, the rest summed in
+//                 their lengths; runs of one lookup and the other runs of
+//                 <= MLKV_SEQ_SEGMENT_MAX lookups go to two lists (one atomic
+//                 per block and list; any order: every run is summed on its
+//                 own), longer ones are measured (a warp-wide search for their
+//                 end) and listed for k_long_*.
+//  k_single       one lane group per run of one lookup: row, state and the
+//                 gradient row loaded together, then the Adagrad step.
+//  k_short        one lane group per run of 2 .. MLKV_SEQ_SEGMENT_MAX
+//                 lookups: the row, the state, the first gradient row and the
+//                 run's other positions are loaded together, the rest summed in
 //                 occurrence order, then the Adagrad step.
 //  k_long_sum     one lane group per chunk of kChunk lookups of a long run
 //                 (Zipf-hot keys reach 10^4-10^5 lookups): chunk sum to scratch.
 //  k_long_combine one block per long run: the chunk sums are split over the
 //                 block's lane groups in a fixed way, added in that order, and
 //                 the row updated.
-// All three keep registers low so that many warps are resident: the access
-// pattern is random 512-byte rows, which HBM serves near its copy bandwidth
-// only with many requests in flight.  Results do not depend on scheduling.
+// Each is tuned for requests in flight (resident warps against rows in flight
+// per warp): the access pattern is random 512-byte rows, which HBM serves near
+// its copy bandwidth only with many requests in flight.  Results do not depend
+// on scheduling.
 #include "mlkv_internal.cuh"
 
 namespace mlkv {
@@ -33,7 +38,7 @@ namespace {
 
 constexpr int kChunk = 64;
 // Long runs of more than kBigRun chunk sums (the hottest rows) are combined by
-// a second launch with blocks of 1024 threads; the rest by many small blocks.
+// a whole 1024-thread block of k_long_combine; the rest by one lane group each.
 constexpr uint32_t kBigRun = 32;
 
 // Tuning (set at build time): gradient rows in flight per lane group, and the
@@ -295,11 +300,12 @@ __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, u
 // next change of value in the window (the next run, or the absent lookups
 // that sort last) or, for the window's last run, where the next window's row
 // ids first differ (past that, it is long and its end is searched for after
-// the windows).  Runs of <= MLKV_SEQ_SEGMENT_MAX lookups are staged in the
-// warp's shared-memory list, long ones in its queue; at the end the block
-// reserves room in the short-run list, the long-run list and the chunk list
-// with one atomic each and the warps copy their runs out.  (Counters that
-// every warp bumps queue up at the end of the kernel.)
+// the windows).  Runs of one lookup and the other runs of <=
+// MLKV_SEQ_SEGMENT_MAX lookups are staged in the warp's two shared-memory
+// lists, long ones in its queue; at the end the block reserves room in the
+// two run lists, the long-run list and the chunk list with one atomic each and
+// the warps copy their runs out.  (Counters that every warp bumps queue up at
+// the end of the kernel.)
 __global__ void __launch_bounds__(256, 5) k_heads(RunArgs a) {
     pdl_enter();
     constexpr int kList = 128, kQueue = 16;
@@ -460,10 +466,10 @@ __global__ void __launch_bounds__(256, 5) k_heads(RunArgs a) {
     emit_long(wlg[wib], wit[wib]);
 }
 
-// One lane group per listed short run.  The run's bounds, row and first lookup
-// position are independent loads, issued one run ahead: while a run's row,
-// state and first gradient row are being loaded, the next run's are already on
-// their way, so a run of one lookup (most of them) costs about one round trip.
+// One lane group per listed run of 2 .. MLKV_SEQ_SEGMENT_MAX lookups.  The
+// run's record (bounds, row, first lookup position) is loaded one run ahead;
+// its row, state, first gradient row and the positions of its other lookups
+// then load together, and the other gradient rows after them.
 __device__ __forceinline__ uint4 run_meta(const RunArgs& a, uint32_t u, uint32_t U) {
     return u < U ? __ldg(a.runs + u) : make_uint4(0u, 0u, 0u, 0u);
 }
