@@ -23,13 +23,24 @@ def _close(got, want):
     return np.abs(np.asarray(got, np.float64) - want) <= TOL * (1 + np.abs(want))
 
 
-@pytest.mark.parametrize("seed,dim", [(1, 32), (2, 16), (3, 100)])
-def test_random_call_sequences(seed, dim):
+@pytest.mark.parametrize("seed,dim,tiered", [(1, 32, False), (2, 16, False), (3, 100, False), (4, 32, True)])
+def test_random_call_sequences(seed, dim, tiered):
+    """The tiered case keeps its rows in host memory behind an HBM cache of
+    two batches and a little more (batches of up to 1,024 lookups, 2,312 lines
+    for 6,000 keys), so rows are evicted and fetched back all along; before some applies of the last Get's keys it issues a look-ahead of
+    another batch (the training order Get, Lookahead, apply)."""
     torch = torch_cuda()
     cfg = W.scaled(W.tiny(), 10, 1)
     cfg.dim = dim
-    n_keys, max_batch = 6_000, 4_096
+    n_keys, max_batch = 6_000, (1_024 if tiered else 4_096)
     store, ref32 = make_pair(cfg, capacity=20_000, max_batch=max_batch)
+    if tiered:
+        from paper_2504_01506_gb300 import EmbeddingStore
+
+        store.close()
+        store = EmbeddingStore(dim=cfg.dim, capacity=20_000, max_batch=max_batch, lr=cfg.lr, eps=cfg.eps,
+                               state_init=cfg.state_init, init_lo=cfg.init_lo, init_hi=cfg.init_hi, seed=cfg.seed,
+                               hbm_cache_rows=2 * max_batch + 64 + 200, device="cuda:0")  # < the 6,000 keys
     ref64 = oracle.Table(cfg.dim, lr=cfg.lr, eps=cfg.eps, state_init=cfg.state_init, init_lo=cfg.init_lo,
                          init_hi=cfg.init_hi, seed=cfg.seed, precision=64)
     rng = np.random.default_rng(seed)
@@ -44,11 +55,19 @@ def test_random_call_sequences(seed, dim):
         n = int(rng.integers(1, max_batch + 1))
         return universe[rng.choice(n_keys, n, p=weights)]
 
+    prev = None
+    la_pending = False  # a look-ahead was issued and no call has waited for it yet
+    n_lookahead = 0
     for step in range(60):
+        if step:
+            prev = op
         op = rng.choice(["get", "apply", "apply_last", "put", "insert", "import", "find", "export", "dedup"],
                         p=[0.2, 0.15, 0.15, 0.1, 0.05, 0.05, 0.1, 0.1, 0.1])
         if op == "apply_last" and last_get is None:
             op = "get"
+        if la_pending and op in ("apply", "apply_last"):
+            op = "get"  # an apply would run beside the pending look-ahead too; every other call waits for it
+        la_pending = la_pending and op in ("apply", "apply_last")
         if op == "get":
             keys = batch()
             out = store.get(dev(keys))
@@ -58,6 +77,10 @@ def test_random_call_sequences(seed, dim):
             last_get = keys
         elif op in ("apply", "apply_last"):
             keys = last_get if op == "apply_last" else batch()  # the training order, or other keys
+            if tiered and op == "apply_last" and prev == "get" and rng.random() < 0.7:
+                store.lookahead(dev(batch()))  # runs beside the apply, right after its Get
+                la_pending = True
+                n_lookahead += 1
             grads = (rng.standard_normal((len(keys), dim)) * 0.01).astype(np.float32)
             store.apply_grad(dev(keys), dev(grads))
             ref32.apply_grad(keys, grads)
@@ -70,12 +93,12 @@ def test_random_call_sequences(seed, dim):
             ref32.put(keys, vals)
             ref64.put(keys, vals)
         elif op == "insert":
-            keys = universe[rng.choice(n_keys, int(rng.integers(1, 2_000)))]
+            keys = universe[rng.choice(n_keys, int(rng.integers(1, max_batch // 2)))]
             store.insert(dev(keys))
             ref32.insert(keys)
             ref64.insert(keys)
         elif op == "import":
-            keys = universe[rng.choice(n_keys, int(rng.integers(1, 2_000)))]
+            keys = universe[rng.choice(n_keys, int(rng.integers(1, max_batch // 2)))]
             rows = (rng.standard_normal((len(keys), dim)) * 0.01).astype(np.float32)
             state = np.abs(rng.standard_normal((len(keys), dim)) * 0.01).astype(np.float32)
             store.import_(dev(keys), dev(rows), dev(state))
@@ -105,6 +128,9 @@ def test_random_call_sequences(seed, dim):
             checks.append(("dedup", (uniq, counts, num, kd), (ou, oc), None))
 
     assert store.sync() == 0
+    if tiered:  # the case did what it is for: look-aheads, and rows evicted and fetched back
+        fetched, written, _ = store.tier_stats()
+        assert n_lookahead >= 2 and fetched > 0 and written > 0, (n_lookahead, fetched, written)
     for i, (kind, got, want, exact) in enumerate(checks):
         what = f"seed {seed}, dim {dim}, check {i} ({kind})"
         if kind == "get":
