@@ -81,7 +81,7 @@ struct Scratch {
     uint32_t* sv[2];        // sort values (positions), ping-pong [max_batch]
     uint32_t* sort_counts;  // [512][tiles] digit counts of a sort pass
     uint32_t* sort_offsets; // [tiles][512] output position of each tile's first element of each digit
-    uint32_t* sort_dtot;    // [kSortMaxPasses][512] digit totals of each pass
+    uint32_t* sort_dtot;    // [kSortMaxPasses][512] digit totals of each pass, zero between sorts
     uint32_t* sort_dirty;   // [tiles] 1: the first pass's counts of the tile are left to the histogram kernel
     uint32_t* tile_sums;    // [scan tiles]
     uint32_t* seg_start;    // [max_batch + 1] run starts in sorted order (dedup)
@@ -354,9 +354,6 @@ cudaError_t launch_export(mlkv_table* t, const int64_t* keys, int64_t n, float* 
 // mlkv_sort.cu
 cudaError_t launch_exclusive_scan(mlkv_table* t, const uint32_t* in, uint32_t* out, int64_t n,
                                   uint32_t* total, const uint32_t* enable, cudaStream_t st);
-// The sort's digit totals start at zero: a call that sorts zeroes them before
-// its first kernel (a memset between two kernels would end their overlap).
-cudaError_t zero_sort_totals(mlkv_table* t, cudaStream_t st);
 // The first pass's counts for the probe to make (t->sort_bits rows, n lookups).
 FirstCounts first_counts(mlkv_table* t, int64_t n);
 // first_dirty: null, or FirstCounts::dirty of a probe that counted the first pass.

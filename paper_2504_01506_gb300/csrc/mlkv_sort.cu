@@ -283,8 +283,12 @@ __global__ void __launch_bounds__(kSThreads, kSThreads == 256 ? 3 : MLKV_SCATTER
                                                               uint32_t* __restrict__ vout, uint32_t n,
                                                               const uint32_t* __restrict__ offsets,
                                                               uint32_t ntiles, int shift, int radix, uint32_t sent,
-                                                              int first) {
+                                                              int first, uint32_t* __restrict__ dtot) {
     pdl_enter();
+    // the pass's digit totals were read by the offsets kernel, which has
+    // finished: zero them for the next sort (the totals are zero between sorts)
+    if (blockIdx.x == 0)
+        for (int d = threadIdx.x; d < radix; d += kSThreads) dtot[d] = 0u;
     // the per-warp digit counts, then (once every position is known) the sorted tile
     __shared__ uint32_t pool[2 * kTile];
     static_assert(kSWarps * kMaxRadix <= 2 * kTile, "counts fit the tile buffer");
@@ -483,7 +487,8 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
     const unsigned nt = tiles(n);
     uint32_t* counts = t->s.sort_counts;
     uint32_t* offsets = t->s.sort_offsets;
-    // the digit totals of every pass were zeroed at the start of the call (zero_sort_totals)
+    // the digit totals of every pass are zero (the arena starts zeroed; each
+    // pass's scatter zeroes its pass's totals once they are read)
     const uint32_t* kin = t->s.row_of_pos;
     const uint32_t* vin = nullptr;
     int out = 0;
@@ -495,7 +500,7 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
         MLKV_LAUNCH(t, 0, k_sort_offsets, (unsigned)((radix + kWarps - 1) / kWarps), kThreads, 0, st, counts, dtot,
                     offsets, nt, radix);
         MLKV_LAUNCH(t, MLKV_K_SORT_SCATTER, k_sort_scatter, nt, kSThreads, 0, st, kin, vin, t->s.sk[out],
-                    t->s.sv[out], (uint32_t)n, offsets, nt, p * D, radix, sent, first);
+                    t->s.sv[out], (uint32_t)n, offsets, nt, p * D, radix, sent, first, dtot);
         kin = t->s.sk[out];
         vin = t->s.sv[out];
         out ^= 1;
@@ -503,10 +508,6 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
     *srow = kin;
     *spos = vin;
     return cudaGetLastError();
-}
-
-cudaError_t zero_sort_totals(mlkv_table* t, cudaStream_t st) {
-    return cudaMemsetAsync(t->s.sort_dtot, 0, (size_t)kSortMaxPasses * kMaxRadix * 4, st);
 }
 
 cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, const uint32_t* spos, int64_t n,

@@ -564,7 +564,6 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
         return set_error(t, MLKV_ERR_UNSUPPORTED, "a tiered table's calls cannot be captured into a graph");
     const bool beside = t->tiered && t->tier.la_pending;
     CallScope cs = begin_call(t, st);
-    CK(t, zero_sort_totals(t, st));
     const bool ins = t->cfg.insert_on_miss != 0 && !beside;
     // On an HBM-resident table the probe also counts the sort's first pass (the
     // tiered apply sorts cache lines, known only after the probe).
@@ -645,7 +644,6 @@ int mlkv_dedup(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_uniqu
     cudaStream_t st = (cudaStream_t)stream;
     if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
-    CK(t, zero_sort_totals(t, st));
     CK(t, launch_probe(t, d_keys, n, false, MemoUse::None, false, false, st, cs.cur, cs.nxt));
     const uint32_t *srow, *spos;
     CK(t, launch_sort_rows(t, n, st, &srow, &spos));
