@@ -553,6 +553,14 @@ struct PutRun {
     }
 };
 
+// Zeroes a call's counters before its first kernel (calls captured into a
+// graph, see begin_call); a kernel rather than a memset keeps the chain of
+// programmatic launches.
+__global__ void k_zero_counters(CallCounters* c) {
+    pdl_enter();
+    if (threadIdx.x < sizeof(CallCounters) / 4) reinterpret_cast<uint32_t*>(c)[threadIdx.x] = 0u;
+}
+
 // The key of every row below n_rows, at its row: a checkpoint's keys in row
 // order (rows are dense, handed out in first-occurrence order).
 __global__ void __launch_bounds__(256) k_dump_keys(const Slot* __restrict__ index, unsigned long long nslots,
@@ -627,6 +635,11 @@ cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n,
 
 cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, const float* state, int64_t n, cudaStream_t st) {
     return dispatch_row<PutRun>(t->geom, t, vals, state, n, st);
+}
+
+cudaError_t launch_zero_counters(mlkv_table* t, CallCounters* c, cudaStream_t st) {
+    MLKV_LAUNCH(t, 0, k_zero_counters, 1, 32, 0, st, c);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_dump_keys(mlkv_table* t, int64_t* out, int64_t n_rows, cudaStream_t st) {

@@ -346,6 +346,7 @@ cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n,
                                   float* out, cudaStream_t st, CallCounters* cur);
 cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, const float* state, int64_t n, cudaStream_t st);
 cudaError_t launch_dump_keys(mlkv_table* t, int64_t* out, int64_t n_rows, cudaStream_t st);
+cudaError_t launch_zero_counters(mlkv_table* t, CallCounters* c, cudaStream_t st);
 cudaError_t launch_find(mlkv_table* t, const int64_t* keys, int64_t n, int64_t* rows,
                         cudaStream_t st, CallCounters* nxt);
 cudaError_t launch_export(mlkv_table* t, const int64_t* keys, int64_t n, float* rows,

@@ -197,13 +197,13 @@ bool capturing(cudaStream_t st) {
 // A call's counters: one of two copies, taken in turn; each call zeroes the
 // other copy for the next one in its first kernel, so no memset is enqueued.
 // A captured graph replays a fixed sequence of calls, which may be odd in
-// number: there every call zeroes its own copy first.
+// number: there every call zeroes its own copy first, with a one-block kernel.
 CallScope begin_call(mlkv_table* t, cudaStream_t st) {
     const int p = t->parity;
     t->parity ^= 1;
     t->last_stream = st;
     CallScope cs{&t->dstate->cc[p], &t->dstate->cc[p ^ 1]};
-    if (capturing(st)) cudaMemsetAsync(cs.cur, 0, sizeof(CallCounters), st);
+    if (capturing(st)) launch_zero_counters(t, cs.cur, st);
     return cs;
 }
 
