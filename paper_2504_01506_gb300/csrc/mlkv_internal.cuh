@@ -420,10 +420,10 @@ inline void launch_kernel(bool pdl, void (*kernel)(Params...), dim3 grid, dim3 b
         (t)->launches++;                                                                          \
     } while (0)
 #define MLKV_LAUNCH(...) MLKV_LAUNCH_PDL(true, __VA_ARGS__)
-// A persistent grid (one wave, each block a fixed share of the work) starts
-// once the kernel before it has finished, with every SM free: blocks placed
-// early on the SMs that drain first would leave the others short of work.
+// The persistent grids (one wave, each block a fixed share of the work) may
+// start as the kernel before them drains too; -DMLKV_PDL_PERSISTENT=0 makes
+// them wait for it in full (every SM free when their blocks are placed).
 #ifndef MLKV_PDL_PERSISTENT
-#define MLKV_PDL_PERSISTENT 0
+#define MLKV_PDL_PERSISTENT 1
 #endif
 #define MLKV_LAUNCH_PERSISTENT(...) MLKV_LAUNCH_PDL(MLKV_PDL_PERSISTENT != 0, __VA_ARGS__)
