@@ -24,6 +24,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import threading
 import time
 
@@ -90,9 +91,10 @@ class ClockSampler:
             time.sleep(0.002)
 
     def start(self):
-        os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
         try:
-            self._smi_path = os.path.join(ROOT, "gpurun_out", "clocks.csv")
+            # nvidia-smi's samples go to a temporary file, read back in stop()
+            fd, self._smi_path = tempfile.mkstemp(prefix="mlkv_clocks_", suffix=".csv")
+            os.close(fd)
             self._smi = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.idx}",
                  "--query-gpu=index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -119,6 +121,10 @@ class ClockSampler:
                     if len(f) >= 5 and f[1].isdigit():
                         mask = int(f[4], 16) if f[4].startswith("0x") else 0
                         self.samples.append((int(f[1]), int(f[2]), mask))
+            except OSError:
+                pass
+            try:
+                os.remove(self._smi_path)
             except OSError:
                 pass
 
