@@ -108,7 +108,10 @@ typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
 
 /* Streams and graphs.  Every call that takes a stream enqueues its work on
  * that stream and returns without waiting for it (the *_host calls, sync,
- * size, last_unique, tier_stats and kernel_time wait).  Calls on one table must
+ * size, last_unique, tier_stats and kernel_time wait).  The library launches
+ * its kernels with programmatic dependent launch, so a kernel may start while
+ * the one before it drains, but each waits for the work before it on entry:
+ * stream order holds as for any launch, for the caller's work too.  Calls on one table must
  * be ordered by the caller (one stream, or events between streams).  On an
  * HBM-resident table a sequence of calls can be captured into a CUDA graph and
  * the graph replayed (the same pointers and sizes each replay; the work of
