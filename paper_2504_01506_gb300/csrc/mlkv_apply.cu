@@ -49,6 +49,10 @@ constexpr uint32_t kBigRun = 32;
 #ifndef MLKV_SHORT_MIN_BLOCKS
 #define MLKV_SHORT_MIN_BLOCKS 2
 #endif
+// k_short: runs a lane group claims at a time.
+#ifndef MLKV_SHORT_GRAB
+#define MLKV_SHORT_GRAB 4
+#endif
 // k_single: runs of one lookup in flight per lane group, and blocks per SM.
 #ifndef MLKV_SINGLES
 #define MLKV_SINGLES 1
@@ -482,11 +486,22 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
     const unsigned gmask = group_mask(G, gid);
     const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
     const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
-    uint4 next = run_meta(a, group, U);
-    for (uint32_t u = group; u < U; u += ngroups) {  // uniform within the group
-        const uint4 m = next;  // (start, end, row, first lookup)
-        next = run_meta(a, u + ngroups, U);
-        short_run<V, KV>(ra, a, m.x, m.y - m.x, m.z, m.w, glane, gmask);
+    // Runs take 2 .. 32 lookups, so fixed shares would leave the kernel to the
+    // group with the most lookups: each group claims chunks of kGrab runs, its
+    // first chunk by its index, the rest from a counter (one atomic a chunk)
+    constexpr uint32_t kGrab = MLKV_SHORT_GRAB;
+    uint32_t base = group * kGrab;
+    while (base < U) {  // uniform within the group
+        const uint32_t end = min(U, base + kGrab);
+        uint4 next = run_meta(a, base, end);
+        for (uint32_t u = base; u < end; ++u) {
+            const uint4 m = next;  // (start, end, row, first lookup)
+            next = run_meta(a, u + 1, end);
+            short_run<V, KV>(ra, a, m.x, m.y - m.x, m.z, m.w, glane, gmask);
+        }
+        uint32_t c = 0;
+        if (glane == 0) c = atomicAdd(&a.cur->short_next, kGrab);
+        base = ngroups * kGrab + __shfl_sync(gmask, c, 0, G);
     }
 }
 

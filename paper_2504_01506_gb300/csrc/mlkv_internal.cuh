@@ -43,6 +43,7 @@ struct CallCounters {
     uint32_t n_short;    // runs of at most MLKV_SEQ_SEGMENT_MAX lookups
     uint32_t n_big;      // long runs whose chunk sums are combined by the wide blocks
     uint32_t n_single;   // runs of one lookup
+    uint32_t short_next; // next chunk of short runs to claim (k_short's dynamic hand-out)
 };
 
 struct DevState {
