@@ -75,3 +75,34 @@ def test_null_and_bad_arguments_without_gpu(lib):
     assert lib.mlkv_get(None, None, 0, None, None) == 1
     assert lib.mlkv_open(None, None) == 1
     assert lib.mlkv_close(None) == 0
+
+
+def test_binding_argument_counts_match_header(lib):
+    """Every declared function takes as many arguments in the ctypes binding as
+    the header declares (a dropped or extra parameter would pass pointers into
+    the wrong places)."""
+    from paper_2504_01506_gb300 import _lib
+
+    src = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    arity = {}
+    for m in re.finditer(r"\b(mlkv_[a-z_]+)\s*\(([^)]*)\)\s*;", src, flags=re.S):
+        params = " ".join(m.group(2).split())
+        arity[m.group(1)] = 0 if params in ("", "void") else params.count(",") + 1
+    assert sorted(arity) == declared_functions()
+    bound = _lib.load()
+    for name, n in arity.items():
+        assert len(getattr(bound, name).argtypes) == n, name
+
+
+def test_binding_constants_match_header():
+    """Status codes, kernel ids, flags and limits in the binding equal the header's."""
+    from paper_2504_01506_gb300 import _lib
+
+    src = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    defines = {m.group(1): int(m.group(2)) for m in re.finditer(r"#define MLKV_(\w+) (\d+)u?\b", src)}
+    checked = 0
+    for name, value in defines.items():
+        if hasattr(_lib, name):
+            assert getattr(_lib, name) == value, name
+            checked += 1
+    assert checked >= 20  # status codes, kernel ids, flags and limits
