@@ -30,15 +30,15 @@
  *     used from one host thread at a time.
  *   - Errors a host check finds are returned at once and nothing is enqueued.
  *     Errors a kernel finds (MLKV_ERR_FULL, MLKV_ERR_PROBE_LIMIT,
- *     MLKV_ERR_NOT_FOUND, MLKV_ERR_TIMEOUT, MLKV_ERR_INVALID for the reserved
- *     key) are sticky:
+ *     MLKV_ERR_NOT_FOUND, MLKV_ERR_INVALID for the reserved key) are sticky:
  *     they are recorded in the table's status word, returned by mlkv_sync and
  *     by later calls once the GPU has reached the failing call, and cleared by
  *     mlkv_clear_status.
  *   - n == 0 is a no-op that returns MLKV_OK (after the argument checks).
  *   - No call allocates device memory except mlkv_open (the table, its index,
  *     its scratch sized for max_batch) and the first *_host call (staging
- *     sized for max_batch).  Every wait inside a kernel is bounded.
+ *     sized for max_batch).  Every loop inside a kernel is bounded (the probe
+ *     limit, the tier's sweep limit); no kernel spins on a flag.
  */
 #ifndef MLKV_GPU_H
 #define MLKV_GPU_H
@@ -58,7 +58,8 @@ extern "C" {
 #define MLKV_ERR_FULL 5        /* more distinct keys than `capacity` */
 #define MLKV_ERR_PROBE_LIMIT 6 /* an index probe exceeded the probe bound */
 #define MLKV_ERR_NOT_FOUND 7   /* absent key and insert_on_miss == 0 */
-#define MLKV_ERR_TIMEOUT 8     /* a bounded wait inside a kernel ran out (the batch is not applied in full) */
+#define MLKV_ERR_TIMEOUT 8     /* reserved for a bounded wait inside a kernel that ran out; no kernel
+                                  of this library waits on a flag or another kernel, so none records it */
 
 /* Largest dimension the row kernels take (8 vectors per lane of a warp). */
 #define MLKV_MAX_DIM 1024  /* dim > 256 needs dim % 4 == 0 */
