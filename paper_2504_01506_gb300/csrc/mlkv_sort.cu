@@ -7,7 +7,9 @@
 // lookup is given the all-ones digit pattern and sorts last.
 //
 // Each pass is a reduce-then-scan pass over 4096-element tiles: one kernel
-// counts the digits of every tile (and the pass's digit totals); one kernel
+// counts the digits of every tile (and the pass's digit totals; in a gradient
+// apply the probe has already counted the first pass's tiles that had no
+// miss, see FirstCounts); one kernel
 // gives every (tile, digit) the output position of its first element (the
 // elements of lower digits plus those of the digit in earlier tiles); a third
 // ranks each tile's elements stably (over rounds of 32, in order) and
