@@ -79,6 +79,8 @@ class EmbeddingStore:
 
     # -- the MLKV interface ----------------------------------------------------
     def get(self, keys: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:
+        """Get: the row of every key ([n, dim], into `out` when given).  Absent keys
+        are inserted with the init row (insert_on_miss), else NaN and NOT_FOUND."""
         keys = self._keys(keys)
         n = keys.numel()
         if out is None:
@@ -88,22 +90,29 @@ class EmbeddingStore:
         return out
 
     def put(self, keys: torch.Tensor, values: torch.Tensor):
+        """Put (upsert): row of each key = its value; the last duplicate wins; a new
+        key starts with state_init, a present one keeps its state."""
         keys = self._keys(keys)
         values = self._rows(values, keys.numel())
         self._check(self.lib.mlkv_put(self.h, keys.data_ptr(), keys.numel(), values.data_ptr(),
                                       _stream(self.device)))
 
     def insert(self, keys: torch.Tensor):
+        """Inserts the absent keys with the init row (row ids in first-occurrence order)."""
         keys = self._keys(keys)
         self._check(self.lib.mlkv_insert(self.h, keys.data_ptr(), keys.numel(), _stream(self.device)))
 
     def apply_grad(self, keys: torch.Tensor, grads: torch.Tensor):
+        """The per-key Rmw: each distinct key's gradients summed, then one Adagrad step
+        on its row and state."""
         keys = self._keys(keys)
         grads = self._rows(grads, keys.numel())
         self._check(self.lib.mlkv_apply_grad(self.h, keys.data_ptr(), keys.numel(), grads.data_ptr(),
                                              _stream(self.device)))
 
     def lookahead(self, keys: torch.Tensor):
+        """Lookahead: brings the rows of the next batch's keys into the HBM cache on
+        the table's side stream (a no-op for an HBM-resident table)."""
         keys = self._keys(keys)
         self._check(self.lib.mlkv_lookahead(self.h, keys.data_ptr(), keys.numel(), _stream(self.device)))
 
@@ -179,12 +188,17 @@ class EmbeddingStore:
 
     # -- host-buffer forms (copies inside the call) -----------------------------
     def get_host(self, keys: torch.Tensor, out: torch.Tensor):
-        assert keys.device.type == "cpu" and out.device.type == "cpu"
+        """Get from and into host tensors (pinned for asynchronous copies); `out` is
+        valid once the stream has synchronised."""
+        if keys.device.type != "cpu" or out.device.type != "cpu":
+            raise TypeError("get_host takes host tensors")
         self._check(self.lib.mlkv_get_host(self.h, keys.data_ptr(), keys.numel(), out.data_ptr(),
                                            _stream(self.device)))
 
     def apply_grad_host(self, keys: torch.Tensor, grads: torch.Tensor):
-        assert keys.device.type == "cpu" and grads.device.type == "cpu"
+        """apply_grad from host tensors (copied to the device inside the call)."""
+        if keys.device.type != "cpu" or grads.device.type != "cpu":
+            raise TypeError("apply_grad_host takes host tensors")
         self._check(self.lib.mlkv_apply_grad_host(self.h, keys.data_ptr(), keys.numel(),
                                                   grads.data_ptr(), _stream(self.device)))
 
