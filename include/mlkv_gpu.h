@@ -91,7 +91,8 @@ typedef struct mlkv_config {
     float state_init;        /* Adagrad state of a new row */
     float init_lo, init_hi;  /* a new row is drawn U[init_lo, init_hi) by the counter-based init */
     uint64_t seed;           /* seed of the counter-based init */
-    int64_t staleness_bound; /* MLKV's consistency bound; 0 (bulk-synchronous) is the only one accepted */
+    int64_t staleness_bound; /* MLKV's consistency bound s (Section 3.3.1): 0 bulk-synchronous;
+                                1..64 stale-synchronous (HBM-resident tables; see below) */
     int64_t hbm_cache_rows;  /* 0: rows + state resident in HBM.  > 0: rows + state live in host
                                 memory (the tier) and this many rows are cached in HBM; it must be
                                 >= 2 * max_batch + 64 (a call and a look-ahead in flight) */
@@ -118,7 +119,20 @@ typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
  * the graph replayed (the same pointers and sizes each replay; the work of
  * each call is device-driven: counts, misses and runs are found on the GPU).
  * Capturing a tiered table's calls returns MLKV_ERR_UNSUPPORTED (its
- * look-ahead runs on the table's own stream). */
+ * look-ahead runs on the table's own stream).
+ *
+ * Stale-synchronous mode (staleness_bound s >= 1, the bounded staleness of
+ * MLKV Section 3.3.1): issue the gradient applies on one stream and every
+ * other call on another.  A Get then waits only for the applies issued more
+ * than s applies before it, so it may run while the last s are in flight, and
+ * each element it returns holds the effect of every earlier apply except, in
+ * any mix, those of the last s (an element is read whole; a row may mix).  An
+ * apply waits for the call issued before it on the other stream (the Get of
+ * its keys) and for the apply before it; it inserts no key (an absent key is
+ * skipped and MLKV_ERR_NOT_FOUND recorded).  Every other call waits for every
+ * apply issued before it.  Rows and state after the applies are what
+ * bulk-synchronous calls give.  Such a table's calls cannot be captured into a
+ * graph (MLKV_ERR_UNSUPPORTED). */
 
 /* Creates a table on the current CUDA device.  Allocates rows + state
  * (capacity x 2 x dim fp32, rows padded to 32 bytes), the index (a power of
@@ -129,7 +143,8 @@ typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
  * slot; a row fetched into the cache hands its host slot to the row it
  * evicts), and a side stream for look-ahead.
  * Returns MLKV_ERR_INVALID (bad field), MLKV_ERR_UNSUPPORTED
- * (staleness_bound != 0), MLKV_ERR_NOMEM or MLKV_ERR_CUDA.  On success *out
+ * (staleness_bound outside 0..64, or non-zero with hbm_cache_rows > 0),
+ * MLKV_ERR_NOMEM or MLKV_ERR_CUDA.  On success *out
  * owns everything; free it with mlkv_close. */
 int mlkv_open(const mlkv_config* cfg, mlkv_table** out);
 

@@ -534,8 +534,8 @@ struct MissRun {
                     (unsigned long long)t->cfg.capacity, mode == MissMode::Put ? 0 : 1,
                     (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init);
         MLKV_LAUNCH(t, 0, (k_miss_finish<V, KV>), g, 256, 0, st, index_args(t), init_ra,
-                    t->s.miss_pos, t->s.miss_slot, t->s.row_of_pos, t->s.first_flag,
-                    mode == MissMode::Get ? out : nullptr, cur, t->dstate,
+                    t->s.miss_pos, t->s.miss_slot, mode == MissMode::Get ? nullptr : t->s.row_of_pos,
+                    t->s.first_flag, mode == MissMode::Get ? out : nullptr, cur, t->dstate,
                     (unsigned long long)t->cfg.capacity);
         return cudaGetLastError();
     }

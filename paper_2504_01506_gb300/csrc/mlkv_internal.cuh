@@ -50,7 +50,8 @@ struct DevState {
     unsigned long long next_row;  // rows handed out so far
     uint32_t status;              // first device-detected error (MLKV_ERR_*), sticky
     uint32_t last_unique;         // distinct rows of the last gradient apply
-    CallCounters cc[2];
+    CallCounters cc[2];           // the counters of every call but the gradient apply, in turn
+    CallCounters cca[2];          // the gradient apply's, in turn
 };
 
 // Row-kernel geometry: a row of d floats is NV vectors of V floats; a group of
@@ -158,6 +159,15 @@ struct mlkv_table {
     float* stage_vals;
     cudaStream_t last_stream;
     int parity;
+    cudaStream_t last_apply_stream;
+    int parity_apply;
+    // Stale-synchronous mode (staleness_bound s >= 1): events order the Get's
+    // stream and the apply's (see mlkv_get).
+    int64_t stale;
+    cudaEvent_t* ev_apply;       // [stale + 1]: apply number j records ev_apply[j % (stale + 1)]
+    cudaEvent_t ev_other;        // after the last call other than an apply
+    int other_recorded;
+    int64_t n_applies;
     int64_t launches;
     mlkv::KernelTimer timer;
     double timed_ms;

@@ -180,9 +180,25 @@ constexpr int kScanTile = 4096;
 
 int64_t tiles_of(int64_t n) { return (n + kScanTile - 1) / kScanTile; }
 
+// A call's counters.  In stale-synchronous mode the scope also records, when
+// the call has enqueued its work, the event the next apply waits for (any
+// call but an apply) or the apply's own event.
 struct CallScope {
     CallCounters* cur;
     CallCounters* nxt;
+    mlkv_table* t = nullptr;
+    cudaStream_t st = nullptr;
+    bool apply = false;
+    ~CallScope() {
+        if (!t) return;
+        if (apply) {
+            ++t->n_applies;
+            cudaEventRecord(t->ev_apply[t->n_applies % (t->stale + 1)], st);
+        } else {
+            cudaEventRecord(t->ev_other, st);
+            t->other_recorded = 1;
+        }
+    }
 };
 
 bool capturing(cudaStream_t st) {
@@ -198,18 +214,53 @@ bool capturing(cudaStream_t st) {
 // other copy for the next one in its first kernel, so no memset is enqueued.
 // A captured graph replays a fixed sequence of calls, which may be odd in
 // number: there every call zeroes its own copy first, with a one-block kernel.
-CallScope begin_call(mlkv_table* t, cudaStream_t st) {
+//
+// Stale-synchronous mode (staleness_bound s >= 1, Gets and applies on two
+// streams): a Get waits for every apply issued more than s applies before it,
+// so it may run beside the last s; any other call waits for every apply; an
+// apply waits for the call before it on the other stream (the Get whose keys
+// it updates) and for the apply before it.  Applies count their own counters,
+// so a Get and an apply in flight together never share them.
+CallScope begin_call(mlkv_table* t, cudaStream_t st, bool get = false) {
     const int p = t->parity;
     t->parity ^= 1;
     t->last_stream = st;
+    if (t->stale > 0) {
+        const int64_t j = get ? t->n_applies - t->stale : t->n_applies;
+        if (j >= 1) cudaStreamWaitEvent(st, t->ev_apply[j % (t->stale + 1)], 0);
+    }
     CallScope cs{&t->dstate->cc[p], &t->dstate->cc[p ^ 1]};
+    if (t->stale > 0) {
+        cs.t = t;
+        cs.st = st;
+    }
+    if (capturing(st)) launch_zero_counters(t, cs.cur, st);
+    return cs;
+}
+
+CallScope begin_apply(mlkv_table* t, cudaStream_t st) {
+    const int p = t->parity_apply;
+    t->parity_apply ^= 1;
+    t->last_apply_stream = st;
+    if (t->stale > 0) {
+        if (t->other_recorded) cudaStreamWaitEvent(st, t->ev_other, 0);
+        if (t->n_applies >= 1) cudaStreamWaitEvent(st, t->ev_apply[t->n_applies % (t->stale + 1)], 0);
+    }
+    CallScope cs{&t->dstate->cca[p], &t->dstate->cca[p ^ 1]};
+    if (t->stale > 0) {
+        cs.t = t;
+        cs.st = st;
+        cs.apply = true;
+    }
     if (capturing(st)) launch_zero_counters(t, cs.cur, st);
     return cs;
 }
 
 // Common argument checks.  Returns MLKV_OK, an error, or -1 for "n == 0: done".
-int check_call(mlkv_table* t, const void* keys, int64_t n, const void* buf, bool need_buf) {
+int check_call(mlkv_table* t, const void* keys, int64_t n, const void* buf, bool need_buf, void* stream = nullptr) {
     if (!t) return MLKV_ERR_INVALID;
+    if (t->stale > 0 && stream && capturing((cudaStream_t)stream))
+        return set_error(t, MLKV_ERR_UNSUPPORTED, "calls of a stale-synchronous table cannot be captured into a graph");
     if (n < 0 || n > t->cfg.max_batch)
         return set_error(t, MLKV_ERR_INVALID, "n = %lld outside [0, max_batch = %lld]", (long long)n,
                          (long long)t->cfg.max_batch);
@@ -301,6 +352,12 @@ int mlkv_close(mlkv_table* t) {
         for (int i = 0; i < 2 * KernelTimer::kMax; ++i) cudaEventDestroy(t->timer.ev[i]);
         delete[] t->timer.ev;
     }
+    if (t->ev_apply) {
+        for (int64_t i = 0; i <= t->stale; ++i)
+            if (t->ev_apply[i]) cudaEventDestroy(t->ev_apply[i]);
+        delete[] t->ev_apply;
+    }
+    if (t->ev_other) cudaEventDestroy(t->ev_other);
     if (t->tiered) {
         Tier& tr = t->tier;
         if (tr.la_stream) cudaStreamDestroy(tr.la_stream);
@@ -339,7 +396,9 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     if (c.max_batch < 1 || c.max_batch >= (1ll << 30)) return MLKV_ERR_INVALID;
     if (c.reserved != 0 || (c.flags & ~MLKV_IDENTITY_HASH)) return MLKV_ERR_INVALID;
     if (!(c.init_hi >= c.init_lo)) return MLKV_ERR_INVALID;
-    if (c.staleness_bound != 0) return MLKV_ERR_UNSUPPORTED;
+    // stale-synchronous mode (MLKV Section 3.3.1): HBM-resident tables, bounds up to 64
+    if (c.staleness_bound < 0 || c.staleness_bound > 64) return MLKV_ERR_UNSUPPORTED;
+    if (c.staleness_bound != 0 && c.hbm_cache_rows > 0) return MLKV_ERR_UNSUPPORTED;
     // a tier needs room for two batches' rows at once (a call and a look-ahead in flight)
     if (c.hbm_cache_rows < 0 || c.hbm_cache_rows >= (1ll << 31) - 2) return MLKV_ERR_INVALID;
     if (c.hbm_cache_rows > 0 && c.hbm_cache_rows < 2 * c.max_batch + 64) return MLKV_ERR_INVALID;
@@ -389,6 +448,15 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
             return fail(MLKV_ERR_CUDA);
         tr.epoch = 1;
         t->slots = tr.cache;
+    }
+    t->stale = c.staleness_bound;
+    if (t->stale > 0) {
+        t->ev_apply = new (std::nothrow) cudaEvent_t[t->stale + 1]();
+        if (!t->ev_apply) return fail(MLKV_ERR_NOMEM);
+        for (int64_t i = 0; i <= t->stale; ++i)
+            if (cudaEventCreateWithFlags(&t->ev_apply[i], cudaEventDisableTiming) != cudaSuccess)
+                return fail(MLKV_ERR_CUDA);
+        if (cudaEventCreateWithFlags(&t->ev_other, cudaEventDisableTiming) != cudaSuccess) return fail(MLKV_ERR_CUDA);
     }
     int64_t nslots = 64;
     while (nslots < 2 * c.capacity) nslots <<= 1;
@@ -485,7 +553,7 @@ int tier_map(mlkv_table* t, uint32_t epoch, int strict, int64_t n, cudaStream_t 
 extern "C" {
 
 int mlkv_get(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_out, void* stream) {
-    int rc = check_call(t, d_keys, n, d_out, true);
+    int rc = check_call(t, d_keys, n, d_out, true, stream);
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if ((rc = choose_geom(t, d_out, d_out))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
@@ -500,14 +568,14 @@ int mlkv_get(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_out, void
         CK(t, launch_gather_lines(t, t->s.row_of_pos, n, d_out, st));
         return MLKV_OK;
     }
-    CallScope cs = begin_call(t, st);
+    CallScope cs = begin_call(t, st, true);
     CK(t, launch_get(t, d_keys, n, d_out, st, cs.cur, cs.nxt));
     if (t->cfg.insert_on_miss) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Get, d_out, st, cs.cur));
     return MLKV_OK;
 }
 
 int mlkv_insert(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream) {
-    int rc = check_call(t, d_keys, n, nullptr, false);
+    int rc = check_call(t, d_keys, n, nullptr, false, stream);
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if ((rc = choose_geom(t, t->slots, t->slots))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
@@ -521,7 +589,7 @@ int mlkv_insert(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream) {
 // Put, and import (the state too): upsert, the last occurrence of a key wins.
 static int put_rows(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_vals, const float* d_state,
                     void* stream) {
-    int rc = check_call(t, d_keys, n, d_vals, true);
+    int rc = check_call(t, d_keys, n, d_vals, true, stream);
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if ((rc = choose_geom(t, d_vals, d_state ? d_state : d_vals))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
@@ -554,7 +622,7 @@ int mlkv_dump_keys(mlkv_table* t, int64_t* d_keys_out, int64_t n_rows, void* str
 }
 
 int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float* d_grads, void* stream) {
-    int rc = check_call(t, d_keys, n, d_grads, true);
+    int rc = check_call(t, d_keys, n, d_grads, true, stream);
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if ((rc = choose_geom(t, d_grads, d_grads))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
@@ -563,12 +631,15 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
     if (t->tiered && capturing(st))
         return set_error(t, MLKV_ERR_UNSUPPORTED, "a tiered table's calls cannot be captured into a graph");
     const bool beside = t->tiered && t->tier.la_pending;
-    CallScope cs = begin_call(t, st);
-    const bool ins = t->cfg.insert_on_miss != 0 && !beside;
+    CallScope cs = begin_apply(t, st);
+    // stale-synchronous: a Get may be inserting beside this apply, and its memo
+    // may be the next Get's; the apply inserts nothing and probes every key
+    const bool ins = t->cfg.insert_on_miss != 0 && !beside && t->stale == 0;
+    const MemoUse memo = t->stale ? MemoUse::None : MemoUse::Read;
     // On an HBM-resident table the probe also counts the sort's first pass (the
     // tiered apply sorts cache lines, known only after the probe).
     const FirstCounts fc = first_counts(t, n);
-    CK(t, launch_probe(t, d_keys, n, ins, MemoUse::Read, false, !ins, st, cs.cur, cs.nxt, nullptr,
+    CK(t, launch_probe(t, d_keys, n, ins, memo, false, !ins, st, cs.cur, cs.nxt, nullptr,
                        t->tiered ? nullptr : &fc));
     if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
     if (t->tiered) {
@@ -586,7 +657,7 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
 }
 
 int mlkv_lookahead(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream) {
-    int rc = check_call(t, d_keys, n, nullptr, false);
+    int rc = check_call(t, d_keys, n, nullptr, false, stream);
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if (!t->tiered) return MLKV_OK;  // every row is resident already
     cudaStream_t st = (cudaStream_t)stream;
@@ -608,7 +679,7 @@ int mlkv_lookahead(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream
 }
 
 int mlkv_find(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_rows, void* stream) {
-    int rc = check_call(t, d_keys, n, d_rows, true);
+    int rc = check_call(t, d_keys, n, d_rows, true, stream);
     if (rc) return rc < 0 ? MLKV_OK : rc;
     cudaStream_t st = (cudaStream_t)stream;
     if ((rc = wait_lookahead(t, st))) return rc;
@@ -619,7 +690,7 @@ int mlkv_find(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_rows, 
 
 int mlkv_export(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_rows, float* d_state,
                 void* stream) {
-    int rc = check_call(t, d_keys, n, d_rows ? (void*)d_rows : (void*)d_state, true);
+    int rc = check_call(t, d_keys, n, d_rows ? (void*)d_rows : (void*)d_state, true, stream);
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if ((rc = choose_geom(t, d_rows ? d_rows : d_state, d_state ? d_state : d_rows))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
@@ -632,13 +703,13 @@ int mlkv_export(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_rows, 
 int mlkv_dedup(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_unique_keys,
                int32_t* d_counts, int64_t* d_num_unique, void* stream) {
     if (t && n == 0) {  // nothing to sort: report zero distinct keys
-        int rc = check_call(t, d_keys, n, nullptr, false);
+        int rc = check_call(t, d_keys, n, nullptr, false, stream);
         if (rc > 0) return rc;
         if (d_num_unique)
             CK(t, cudaMemsetAsync(d_num_unique, 0, sizeof(int64_t), (cudaStream_t)stream));
         return MLKV_OK;
     }
-    int rc = check_call(t, d_keys, n, d_unique_keys, true);
+    int rc = check_call(t, d_keys, n, d_unique_keys, true, stream);
     if (rc) return rc < 0 ? MLKV_OK : rc;
     if (!d_counts || !d_num_unique) return set_error(t, MLKV_ERR_INVALID, "null pointer");
     cudaStream_t st = (cudaStream_t)stream;
@@ -690,6 +761,7 @@ int mlkv_apply_grad_host(mlkv_table* t, const int64_t* h_keys, int64_t n, const 
 int mlkv_sync(mlkv_table* t) {
     if (!t) return MLKV_ERR_INVALID;
     CK(t, cudaStreamSynchronize(t->last_stream));
+    if (t->last_apply_stream != t->last_stream) CK(t, cudaStreamSynchronize(t->last_apply_stream));
     if (t->tiered) CK(t, cudaStreamSynchronize(t->tier.la_stream));
     uint32_t st = 0;
     CK(t, cudaMemcpy(&st, &t->dstate->status, sizeof(st), cudaMemcpyDeviceToHost));
@@ -710,6 +782,8 @@ int mlkv_clear_status(mlkv_table* t) {
 int64_t mlkv_size(mlkv_table* t) {
     if (!t) return -1;
     if (cudaStreamSynchronize(t->last_stream) != cudaSuccess) return -1;
+    if (t->last_apply_stream != t->last_stream && cudaStreamSynchronize(t->last_apply_stream) != cudaSuccess)
+        return -1;
     if (t->tiered && cudaStreamSynchronize(t->tier.la_stream) != cudaSuccess) return -1;
     unsigned long long nr = 0;
     if (cudaMemcpy(&nr, &t->dstate->next_row, sizeof(nr), cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
@@ -719,6 +793,8 @@ int64_t mlkv_size(mlkv_table* t) {
 int64_t mlkv_last_unique(mlkv_table* t) {
     if (!t) return -1;
     if (cudaStreamSynchronize(t->last_stream) != cudaSuccess) return -1;
+    if (t->last_apply_stream != t->last_stream && cudaStreamSynchronize(t->last_apply_stream) != cudaSuccess)
+        return -1;
     uint32_t u = 0;
     if (cudaMemcpy(&u, &t->dstate->last_unique, sizeof(u), cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
     return (int64_t)u;
