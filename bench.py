@@ -388,7 +388,12 @@ def run_ours(args, cfg):
     kv = isinstance(cfg, W.YcsbConfig)
     store = EmbeddingStore(dim=cfg.dim, capacity=cfg.n_keys, max_batch=cfg.batch, lr=cfg.lr, eps=cfg.eps,
                            state_init=cfg.state_init, init_lo=cfg.init_lo, init_hi=cfg.init_hi,
-                           seed=cfg.seed, hbm_cache_rows=cfg.hbm_cache_rows, device=dev)
+                           seed=cfg.seed, hbm_cache_rows=cfg.hbm_cache_rows,
+                           staleness_bound=args.staleness, device=dev)
+    # stale-synchronous steps: each Get on one stream, each apply on another; the
+    # table lets Get(t) run beside the last `staleness` applies before it
+    s_get = torch.cuda.Stream(dev) if args.staleness else None
+    s_apply = torch.cuda.Stream(dev) if args.staleness else None
     # preload every key of the table (untimed), in preload order
     chunk = cfg.batch
     for s in range(0, cfg.n_keys, chunk):
@@ -441,6 +446,12 @@ def run_ours(args, cfg):
             store.get(r, out=out[:r.numel()])
             store.put(w, v)
             return
+        if args.staleness:
+            with torch.cuda.stream(s_get):
+                store.get(keys_d[j], out=out)
+            with torch.cuda.stream(s_apply):
+                store.apply_grad(keys_d[j], grads_d[i % ngrad])
+            return
         store.get(keys_d[j], out=out)
         if tiered and args.lookahead:  # Lookahead(next keys) runs beside this step's apply
             store.lookahead(keys_d[(i + 1) % pool])
@@ -462,7 +473,7 @@ def run_ours(args, cfg):
     # An HBM-resident step is captured into a CUDA graph per batch (the Get and
     # the apply of that batch) and replayed: the calls' work is device-driven,
     # so a replay does all of it with one launch from the host.
-    use_graphs = not tiered and args.graphs
+    use_graphs = not tiered and args.graphs and not args.staleness  # stale-synchronous calls refuse capture
     graphs, launches_per_graph = [], 0
     if use_graphs:
         cap = torch.cuda.Stream(dev)
@@ -498,8 +509,14 @@ def run_ours(args, cfg):
     if args.profile:
         torch.cuda.profiler.start()
     ev0.record(stream)
+    for side in (s_get, s_apply):
+        if side is not None:
+            side.wait_stream(stream)
     for i in range(args.steps):
         timed_step(base + args.warmup + i)
+    for side in (s_get, s_apply):
+        if side is not None:
+            stream.wait_stream(side)
     ev1.record(stream)
     barrier(dist, torch)
     if args.profile:
@@ -638,14 +655,17 @@ def run_ours(args, cfg):
             "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": dict(workload_config(cfg), parallelism=f"replicas{world}", distinct_batches=pool),
+            "config": dict(workload_config(cfg), parallelism=f"replicas{world}", distinct_batches=pool,
+                           **({"staleness_bound": args.staleness} if args.staleness else {})),
             "achieved_gbs": achieved_step, "hbm_frac_measured": achieved_step / hbm_peak,
             "hbm_frac_nominal": achieved_step / NOMINAL_HBM_GBS,
             "distinct_per_step": float(np.mean([s["U"] for s in stats])),
             "roofline": roofline, "kernel_ms_one_step": {KERNEL_NAMES[k]: v for k, v in kernel_ms.items()},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clocks.summary(),
             "step_launch": (f"one CUDA graph replay per step (the Get and the {'Put' if kv else 'apply'} of the "
-                            f"batch, captured)" if use_graphs else "each call launched from the host"),
+                            f"batch, captured)" if use_graphs else
+                            "each call launched from the host" + (", Gets and applies on two streams"
+                                                                  if args.staleness else "")),
         }
         if tier is not None:
             line["tier"] = tier
@@ -682,7 +702,12 @@ def main():
                     help="tiered config: no look-ahead; each Get fetches its own missing rows")
     ap.add_argument("--scale", type=int, default=1,
                     help="divide the table's rows by this (same batch); for small profiling cases")
+    ap.add_argument("--staleness", type=int, default=0,
+                    help="HBM-resident training configs: open the table stale-synchronous with this bound "
+                         "(1..64) and run Gets and applies on two streams")
     args = ap.parse_args()
+    if args.staleness and (args.config in ("tiered", "ycsb", "ycsb-uniform") or not 0 < args.staleness <= 64):
+        ap.error("--staleness takes 1..64 and an HBM-resident training config")
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     cfg = W.ALL[args.config]()
