@@ -109,8 +109,8 @@ typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
  * Flood 2014) whose state is z.  State starts at state_init. */
 
 /* Streams and graphs.  Every call that takes a stream enqueues its work on
- * that stream and returns without waiting for it (the *_host calls, sync,
- * size, last_unique, tier_stats and kernel_time wait).  The library launches
+ * that stream and returns without waiting for it (sync, size, last_unique,
+ * tier_stats and kernel_time wait).  The library launches
  * its kernels with programmatic dependent launch, so a kernel may start while
  * the one before it drains, but each waits for the work before it on entry:
  * stream order holds as for any launch, for the caller's work too.  Calls on one table must
@@ -249,7 +249,9 @@ int mlkv_dedup_keys_static(const int64_t* d_keys, int64_t n, int64_t* d_unique_k
 /* Host-buffer forms of Get and the gradient apply: the keys (and gradients)
  * are copied host -> device into table-owned staging on `stream`, the device
  * call runs, and Get's output is copied back to h_out.  The first call
- * allocates the staging (max_batch keys + max_batch x dim floats).  The call
+ * allocates the staging (max_batch keys + max_batch x dim floats; on a
+ * stale-synchronous table the applies' own second set, so that a Get and an
+ * apply on the two streams do not share it).  The call
  * returns once the work is enqueued; h_out is valid after the stream syncs. */
 int mlkv_get_host(mlkv_table* t, const int64_t* h_keys, int64_t n, float* h_out, void* stream);
 int mlkv_apply_grad_host(mlkv_table* t, const int64_t* h_keys, int64_t n, const float* h_grads,

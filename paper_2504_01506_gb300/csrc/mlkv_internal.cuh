@@ -155,8 +155,10 @@ struct mlkv_table {
     mlkv::Scratch s;
     void* arena;                 // one allocation holding Scratch
     int64_t arena_bytes;
-    int64_t* stage_keys;         // *_host staging, lazily allocated
-    float* stage_vals;
+    // *_host staging, lazily allocated: [0] for every call of a bulk-synchronous
+    // table; on a stale-synchronous one [1] for the applies, which run beside Gets
+    int64_t* stage_keys[2];
+    float* stage_vals[2];
     cudaStream_t last_stream;
     int parity;
     cudaStream_t last_apply_stream;

@@ -380,8 +380,10 @@ int mlkv_close(mlkv_table* t) {
     cudaFree(t->index);
     cudaFree(t->dstate);
     cudaFree(t->arena);
-    cudaFree(t->stage_keys);
-    cudaFree(t->stage_vals);
+    for (int i = 0; i < 2; ++i) {
+        cudaFree(t->stage_keys[i]);
+        cudaFree(t->stage_vals[i]);
+    }
     if (t->status_host) cudaFreeHost(t->status_host);
     delete t;
     return MLKV_OK;
@@ -723,14 +725,17 @@ int mlkv_dedup(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_uniqu
     return MLKV_OK;
 }
 
-static int ensure_staging(mlkv_table* t) {
-    if (t->stage_keys) return MLKV_OK;
+// The staging set of a host-buffer call: the applies of a stale-synchronous
+// table have their own, since a Get may still be reading its keys beside them.
+static int ensure_staging(mlkv_table* t, bool apply, int& set) {
+    set = apply && t->stale > 0 ? 1 : 0;
+    if (t->stage_keys[set]) return MLKV_OK;
     const size_t kb = (size_t)t->cfg.max_batch * sizeof(int64_t);
     const size_t vb = (size_t)t->cfg.max_batch * t->cfg.dim * sizeof(float);
-    if (cudaMalloc(&t->stage_keys, kb) != cudaSuccess) return set_error(t, MLKV_ERR_NOMEM, "staging keys");
-    if (cudaMalloc(&t->stage_vals, vb) != cudaSuccess) {
-        cudaFree(t->stage_keys);
-        t->stage_keys = nullptr;
+    if (cudaMalloc(&t->stage_keys[set], kb) != cudaSuccess) return set_error(t, MLKV_ERR_NOMEM, "staging keys");
+    if (cudaMalloc(&t->stage_vals[set], vb) != cudaSuccess) {
+        cudaFree(t->stage_keys[set]);
+        t->stage_keys[set] = nullptr;
         return set_error(t, MLKV_ERR_NOMEM, "staging values");
     }
     return MLKV_OK;
@@ -739,11 +744,12 @@ static int ensure_staging(mlkv_table* t) {
 int mlkv_get_host(mlkv_table* t, const int64_t* h_keys, int64_t n, float* h_out, void* stream) {
     int rc = check_call(t, h_keys, n, h_out, true);
     if (rc) return rc < 0 ? MLKV_OK : rc;
-    if ((rc = ensure_staging(t))) return rc;
+    int set;
+    if ((rc = ensure_staging(t, false, set))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
-    CK(t, cudaMemcpyAsync(t->stage_keys, h_keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
-    if ((rc = mlkv_get(t, t->stage_keys, n, t->stage_vals, stream))) return rc;
-    CK(t, cudaMemcpyAsync(h_out, t->stage_vals, (size_t)n * t->cfg.dim * 4, cudaMemcpyDeviceToHost, st));
+    CK(t, cudaMemcpyAsync(t->stage_keys[set], h_keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
+    if ((rc = mlkv_get(t, t->stage_keys[set], n, t->stage_vals[set], stream))) return rc;
+    CK(t, cudaMemcpyAsync(h_out, t->stage_vals[set], (size_t)n * t->cfg.dim * 4, cudaMemcpyDeviceToHost, st));
     return MLKV_OK;
 }
 
@@ -751,11 +757,12 @@ int mlkv_apply_grad_host(mlkv_table* t, const int64_t* h_keys, int64_t n, const 
                          void* stream) {
     int rc = check_call(t, h_keys, n, h_grads, true);
     if (rc) return rc < 0 ? MLKV_OK : rc;
-    if ((rc = ensure_staging(t))) return rc;
+    int set;
+    if ((rc = ensure_staging(t, true, set))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
-    CK(t, cudaMemcpyAsync(t->stage_keys, h_keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
-    CK(t, cudaMemcpyAsync(t->stage_vals, h_grads, (size_t)n * t->cfg.dim * 4, cudaMemcpyHostToDevice, st));
-    return mlkv_apply_grad(t, t->stage_keys, n, t->stage_vals, stream);
+    CK(t, cudaMemcpyAsync(t->stage_keys[set], h_keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
+    CK(t, cudaMemcpyAsync(t->stage_vals[set], h_grads, (size_t)n * t->cfg.dim * 4, cudaMemcpyHostToDevice, st));
+    return mlkv_apply_grad(t, t->stage_keys[set], n, t->stage_vals[set], stream);
 }
 
 int mlkv_sync(mlkv_table* t) {

@@ -35,8 +35,10 @@ def _oracle(cfg):
                         init_hi=cfg.init_hi, seed=cfg.seed, precision=32)
 
 
-@pytest.mark.parametrize("s", [1, 2])
-def test_stale_synchronous_training_loop(s):
+@pytest.mark.parametrize("s,host_buffers", [(1, False), (2, False), (1, True)])
+def test_stale_synchronous_training_loop(s, host_buffers):
+    """host_buffers: the host-buffer calls, whose keys and gradients are staged
+    on the device inside the call (a Get's staging must not be an apply's)."""
     torch = torch_cuda()
     cfg = W.tiny()
     rng = np.random.default_rng(40 + s)
@@ -64,16 +66,27 @@ def test_stale_synchronous_training_loop(s):
 
     store = _store(cfg, s)
     store.insert(dev(pre))
-    kd = [dev(k) for k, _ in steps]
-    gd = [dev(g) for _, g in steps]
-    outs = [torch.empty((BATCH, DIM), device="cuda:0") for _ in steps]
+    if host_buffers:
+        kd = [torch.from_numpy(k).pin_memory() for k, _ in steps]
+        gd = [torch.from_numpy(g).pin_memory() for _, g in steps]
+        outs = [torch.empty((BATCH, DIM)).pin_memory() for _ in steps]
+    else:
+        kd = [dev(k) for k, _ in steps]
+        gd = [dev(g) for _, g in steps]
+        outs = [torch.empty((BATCH, DIM), device="cuda:0") for _ in steps]
     torch.cuda.synchronize()
     s_get, s_apply = torch.cuda.Stream(), torch.cuda.Stream()
     for t in range(STEPS):
         with torch.cuda.stream(s_get):
-            store.get(kd[t], out=outs[t])
+            if host_buffers:
+                store.get_host(kd[t], outs[t])
+            else:
+                store.get(kd[t], out=outs[t])
         with torch.cuda.stream(s_apply):
-            store.apply_grad(kd[t], gd[t])
+            if host_buffers:
+                store.apply_grad_host(kd[t], gd[t])
+            else:
+                store.apply_grad(kd[t], gd[t])
     torch.cuda.synchronize()
     assert store.sync() == 0
 
@@ -89,7 +102,7 @@ def test_stale_synchronous_training_loop(s):
         for k, row in snap.items():
             first.setdefault(k, row)
     for t, (keys, _) in enumerate(steps):
-        got = host(outs[t])
+        got = outs[t].numpy() if host_buffers else host(outs[t])
         ok = np.zeros_like(got, dtype=bool)
         for j in range(max(0, t - s), t + 1):
             want = np.stack([snaps[j].get(k, first[k]) for k in keys.tolist()])
