@@ -77,6 +77,13 @@ extern "C" {
 /* Longest probe sequence of the index; a longer one records MLKV_ERR_PROBE_LIMIT. */
 #define MLKV_PROBE_LIMIT 1024
 
+/* staleness_bound values (MLKV Section 3.3.1): 0 is bulk-synchronous, this one
+ * asynchronous (no bound), any other stale-synchronous.  A bound above
+ * MLKV_MAX_STALENESS is kept as MLKV_MAX_STALENESS: a tighter bound, which
+ * meets the one asked for. */
+#define MLKV_STALENESS_ASYNC INT64_MAX
+#define MLKV_MAX_STALENESS 64
+
 /*
  * Open of MLKV Section 3.1: Open(model_id, dim, staleness_bound).  model_id
  * maps to the returned handle; one handle per table.
@@ -91,8 +98,9 @@ typedef struct mlkv_config {
     float state_init;        /* Adagrad state of a new row */
     float init_lo, init_hi;  /* a new row is drawn U[init_lo, init_hi) by the counter-based init */
     uint64_t seed;           /* seed of the counter-based init */
-    int64_t staleness_bound; /* MLKV's consistency bound s (Section 3.3.1): 0 bulk-synchronous;
-                                1..64 stale-synchronous (HBM-resident tables; see below) */
+    int64_t staleness_bound; /* MLKV's consistency bound s (Section 3.3.1), >= 0: 0 bulk-
+                                synchronous; MLKV_STALENESS_ASYNC asynchronous; any other
+                                stale-synchronous (HBM-resident tables; see below) */
     int64_t hbm_cache_rows;  /* 0: rows + state resident in HBM.  > 0: rows + state live in host
                                 memory (the tier) and this many rows are cached in HBM; it must be
                                 >= 2 * max_batch + 64 (a call and a look-ahead in flight) */
@@ -126,7 +134,8 @@ typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
  * other call on another.  A Get then waits only for the applies issued more
  * than s applies before it, so it may run while the last s are in flight, and
  * each element it returns holds the effect of every earlier apply except, in
- * any mix, those of the last s (an element is read whole; a row may mix).  An
+ * any mix, those of the last s (an element is read whole; a row may mix).  In
+ * asynchronous mode (MLKV_STALENESS_ASYNC) a Get waits for no apply.  An
  * apply waits for the call issued before it on the other stream (the Get of
  * its keys) and for the apply before it; it inserts no key (an absent key is
  * skipped and MLKV_ERR_NOT_FOUND recorded).  Every other call waits for every
@@ -143,7 +152,7 @@ typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
  * slot; a row fetched into the cache hands its host slot to the row it
  * evicts), and a side stream for look-ahead.
  * Returns MLKV_ERR_INVALID (bad field), MLKV_ERR_UNSUPPORTED
- * (staleness_bound outside 0..64, or non-zero with hbm_cache_rows > 0),
+ * (staleness_bound non-zero with hbm_cache_rows > 0),
  * MLKV_ERR_NOMEM or MLKV_ERR_CUDA.  On success *out
  * owns everything; free it with mlkv_close. */
 int mlkv_open(const mlkv_config* cfg, mlkv_table** out);

@@ -22,6 +22,8 @@ ERR_TIMEOUT = 8
 SEQ_SEGMENT_MAX = 32
 PROBE_LIMIT = 1024
 IDENTITY_HASH = 2
+MAX_STALENESS = 64
+STALENESS_ASYNC = 2**63 - 1  # staleness_bound of the asynchronous mode (INT64_MAX)
 
 K_GET_GATHER = 1
 K_PROBE = 2

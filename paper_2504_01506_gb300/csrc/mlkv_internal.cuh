@@ -30,6 +30,7 @@ constexpr int kSortMaxPasses = 4;      // row ids have at most 31 bits
 constexpr int kSortMaxDigitBits = 9;   // radix <= 512
 constexpr int kSortMaxRadix = 1 << kSortMaxDigitBits;
 constexpr int kSortTile = 4096;        // lookups per tile of a sort pass
+constexpr int64_t kMaxStaleness = MLKV_MAX_STALENESS;  // largest bound kept below no bound
 
 // Per-call counters.  Two copies: a call uses cc[p] and its first kernel
 // zeroes cc[p ^ 1] for the next call, so no memset is enqueued.
@@ -165,8 +166,9 @@ struct mlkv_table {
     int parity_apply;
     // Stale-synchronous mode (staleness_bound s >= 1): events order the Get's
     // stream and the apply's (see mlkv_get).
-    int64_t stale;
-    cudaEvent_t* ev_apply;       // [stale + 1]: apply number j records ev_apply[j % (stale + 1)]
+    int64_t stale;               // the bound kept: 0, 1..kMaxStaleness, or INT64_MAX (no bound)
+    int64_t ring;                // events in ev_apply
+    cudaEvent_t* ev_apply;       // [ring]: apply number j records ev_apply[j % ring]
     cudaEvent_t ev_other;        // after the last call other than an apply
     int other_recorded;
     int64_t n_applies;

@@ -193,7 +193,7 @@ struct CallScope {
         if (!t) return;
         if (apply) {
             ++t->n_applies;
-            cudaEventRecord(t->ev_apply[t->n_applies % (t->stale + 1)], st);
+            cudaEventRecord(t->ev_apply[t->n_applies % t->ring], st);
         } else {
             cudaEventRecord(t->ev_other, st);
             t->other_recorded = 1;
@@ -217,7 +217,8 @@ bool capturing(cudaStream_t st) {
 //
 // Stale-synchronous mode (staleness_bound s >= 1, Gets and applies on two
 // streams): a Get waits for every apply issued more than s applies before it,
-// so it may run beside the last s; any other call waits for every apply; an
+// so it may run beside the last s (asynchronous mode, s = INT64_MAX: a Get
+// waits for no apply); any other call waits for every apply; an
 // apply waits for the call before it on the other stream (the Get whose keys
 // it updates) and for the apply before it.  Applies count their own counters,
 // so a Get and an apply in flight together never share them.
@@ -225,9 +226,9 @@ CallScope begin_call(mlkv_table* t, cudaStream_t st, bool get = false) {
     const int p = t->parity;
     t->parity ^= 1;
     t->last_stream = st;
-    if (t->stale > 0) {
+    if (t->stale > 0 && !(get && t->stale == INT64_MAX)) {
         const int64_t j = get ? t->n_applies - t->stale : t->n_applies;
-        if (j >= 1) cudaStreamWaitEvent(st, t->ev_apply[j % (t->stale + 1)], 0);
+        if (j >= 1) cudaStreamWaitEvent(st, t->ev_apply[j % t->ring], 0);
     }
     CallScope cs{&t->dstate->cc[p], &t->dstate->cc[p ^ 1]};
     if (t->stale > 0) {
@@ -244,7 +245,7 @@ CallScope begin_apply(mlkv_table* t, cudaStream_t st) {
     t->last_apply_stream = st;
     if (t->stale > 0) {
         if (t->other_recorded) cudaStreamWaitEvent(st, t->ev_other, 0);
-        if (t->n_applies >= 1) cudaStreamWaitEvent(st, t->ev_apply[t->n_applies % (t->stale + 1)], 0);
+        if (t->n_applies >= 1) cudaStreamWaitEvent(st, t->ev_apply[t->n_applies % t->ring], 0);
     }
     CallScope cs{&t->dstate->cca[p], &t->dstate->cca[p ^ 1]};
     if (t->stale > 0) {
@@ -353,7 +354,7 @@ int mlkv_close(mlkv_table* t) {
         delete[] t->timer.ev;
     }
     if (t->ev_apply) {
-        for (int64_t i = 0; i <= t->stale; ++i)
+        for (int64_t i = 0; i < t->ring; ++i)
             if (t->ev_apply[i]) cudaEventDestroy(t->ev_apply[i]);
         delete[] t->ev_apply;
     }
@@ -398,8 +399,8 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     if (c.max_batch < 1 || c.max_batch >= (1ll << 30)) return MLKV_ERR_INVALID;
     if (c.reserved != 0 || (c.flags & ~MLKV_IDENTITY_HASH)) return MLKV_ERR_INVALID;
     if (!(c.init_hi >= c.init_lo)) return MLKV_ERR_INVALID;
-    // stale-synchronous mode (MLKV Section 3.3.1): HBM-resident tables, bounds up to 64
-    if (c.staleness_bound < 0 || c.staleness_bound > 64) return MLKV_ERR_UNSUPPORTED;
+    // stale-synchronous and asynchronous modes (MLKV Section 3.3.1): HBM-resident tables
+    if (c.staleness_bound < 0) return MLKV_ERR_INVALID;
     if (c.staleness_bound != 0 && c.hbm_cache_rows > 0) return MLKV_ERR_UNSUPPORTED;
     // a tier needs room for two batches' rows at once (a call and a look-ahead in flight)
     if (c.hbm_cache_rows < 0 || c.hbm_cache_rows >= (1ll << 31) - 2) return MLKV_ERR_INVALID;
@@ -451,11 +452,16 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
         tr.epoch = 1;
         t->slots = tr.cache;
     }
-    t->stale = c.staleness_bound;
+    // The bound kept: s up to kMaxStaleness, a tighter bound above it (which
+    // meets the one asked for), none at INT64_MAX.  A Get waits for the apply
+    // issued s applies back, so the ring holds the last s + 1 applies' events
+    // (the last one's alone with no bound).
+    t->stale = c.staleness_bound == INT64_MAX ? INT64_MAX : std::min<int64_t>(c.staleness_bound, kMaxStaleness);
+    t->ring = t->stale == INT64_MAX ? 1 : t->stale + 1;
     if (t->stale > 0) {
-        t->ev_apply = new (std::nothrow) cudaEvent_t[t->stale + 1]();
+        t->ev_apply = new (std::nothrow) cudaEvent_t[t->ring]();
         if (!t->ev_apply) return fail(MLKV_ERR_NOMEM);
-        for (int64_t i = 0; i <= t->stale; ++i)
+        for (int64_t i = 0; i < t->ring; ++i)
             if (cudaEventCreateWithFlags(&t->ev_apply[i], cudaEventDisableTiming) != cudaSuccess)
                 return fail(MLKV_ERR_CUDA);
         if (cudaEventCreateWithFlags(&t->ev_other, cudaEventDisableTiming) != cudaSuccess) return fail(MLKV_ERR_CUDA);

@@ -10,6 +10,10 @@ Keys are int64 CUDA tensors; rows, values and gradients float32 [n, dim] CUDA
 tensors.  Every call is enqueued on the current torch stream of the store's
 device and runs in the CUDA library; this class only checks tensor types and
 passes pointers.
+
+staleness_bound (Open's third argument, Section 3.3.1): 0 runs every call in
+order; s >= 1 lets a Get issued on one stream run beside the last s gradient
+applies issued on another; STALENESS_ASYNC (INT64_MAX) lets it run beside any.
 """
 import ctypes
 

@@ -173,8 +173,9 @@ def test_open_rejects_bad_configs():
     from paper_2504_01506_gb300 import EmbeddingStore, MLKVError
 
     for kw, code in ((dict(dim=0), 1), (dict(dim=1025), 1), (dict(dim=257), 1), (dict(capacity=0), 1),
-                     (dict(staleness_bound=65), 2), (dict(staleness_bound=-1), 2),
+                     (dict(staleness_bound=-1), 1),
                      (dict(staleness_bound=1, hbm_cache_rows=100), 2),  # stale-synchronous: HBM-resident only
+                     (dict(staleness_bound=2**63 - 1, hbm_cache_rows=100), 2),
                      (dict(hbm_cache_rows=10), 1), (dict(flags=64), 1)):
         args = dict(dim=8, capacity=100, max_batch=10)
         args.update(kw)

@@ -1,9 +1,11 @@
-"""Stale-synchronous tables (the bounded staleness of MLKV Section 3.3.1): Gets
-on one stream, gradient applies on another, against the oracle.
+"""Stale-synchronous and asynchronous tables (the bounded staleness of MLKV
+Section 3.3.1): Gets on one stream, gradient applies on another, against the
+oracle.
 
 With bound s a Get may run beside the last s applies issued before it: each
 element it returns is the oracle's value after j applies, for some j between
-(t - s) and t at step t, chosen element by element.  The applies themselves run
+(t - s) and t at step t, chosen element by element (any j <= t with no bound,
+the asynchronous mode).  The applies themselves run
 in order, so the table after the last one is exactly the bulk-synchronous
 oracle's.  Batches draw keys uniformly (no run longer than 32 lookups), so every
 comparison is bit for bit against the fp32 oracle."""
@@ -17,6 +19,7 @@ from gpu_helpers import assert_bits, dev, host, torch_cuda
 pytestmark = pytest.mark.gpu
 
 DIM, N_KEYS, BATCH, STEPS = 16, 5_000, 1_024, 10
+ASYNC = 2**63 - 1
 
 
 def _store(cfg, s, **over):
@@ -35,7 +38,7 @@ def _oracle(cfg):
                         init_hi=cfg.init_hi, seed=cfg.seed, precision=32)
 
 
-@pytest.mark.parametrize("s,host_buffers", [(1, False), (2, False), (1, True)])
+@pytest.mark.parametrize("s,host_buffers", [(1, False), (2, False), (1, True), (100, False), (ASYNC, False)])
 def test_stale_synchronous_training_loop(s, host_buffers):
     """host_buffers: the host-buffer calls, whose keys and gradients are staged
     on the device inside the call (a Get's staging must not be an apply's)."""
@@ -104,7 +107,7 @@ def test_stale_synchronous_training_loop(s, host_buffers):
     for t, (keys, _) in enumerate(steps):
         got = outs[t].numpy() if host_buffers else host(outs[t])
         ok = np.zeros_like(got, dtype=bool)
-        for j in range(max(0, t - s), t + 1):
+        for j in range(max(0, t - s), t + 1):  # (s above 64 is kept as 64: within the bound too)
             want = np.stack([snaps[j].get(k, first[k]) for k in keys.tolist()])
             ok |= got.view(np.int32) == want.view(np.int32)
         assert ok.all(), f"s={s}, step {t}: {int((~ok).sum())} elements outside the staleness bound"

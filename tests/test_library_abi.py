@@ -106,3 +106,4 @@ def test_binding_constants_match_header():
             assert getattr(_lib, name) == value, name
             checked += 1
     assert checked >= 20  # status codes, kernel ids, flags and limits
+    assert re.search(r"#define MLKV_STALENESS_ASYNC INT64_MAX\b", src) and _lib.STALENESS_ASYNC == 2**63 - 1
