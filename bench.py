@@ -218,16 +218,18 @@ KERNEL_SOURCES = {1: "mlkv_index.cu", 2: "mlkv_index.cu", 3: "mlkv_sort.cu", 4: 
                   9: "mlkv_index.cu", 10: "mlkv_apply.cu"}
 
 
-def traffic_for(kid: int):
+def traffic_for(kid: int, cfg, path=None):
     """DRAM bytes per launch from the committed ncu summary, if it was taken on
-    the current source of that kernel (source hash match), else None."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
+    this workload (name, rows and batch) and on the current source of that
+    kernel (source hash match), else None."""
+    path = path or os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f).get(str(kid))
     except (OSError, ValueError):
         return None
-    if not rec:
+    if not rec or (rec.get("workload"), rec.get("rows"), rec.get("batch_lookups")) != (cfg.name, cfg.n_keys,
+                                                                                        cfg.batch):
         return None
     src = os.path.join(ROOT, "paper_2504_01506_gb300", "csrc", KERNEL_SOURCES[kid])
     h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
@@ -573,7 +575,7 @@ def run_ours(args, cfg):
         achieved = per_launch_bytes / (avg_ms / 1e3) / 1e9
         roofline = {"bound": "hbm", "kernel": KERNEL_NAMES[dominant], "achieved": achieved, "peak": hbm_peak,
                     "unit": "GB/s", "frac": achieved / hbm_peak, "peak_kind": peak_kind,
-                    "traffic": traffic_for(dominant), "bytes_per_launch": per_launch_bytes,
+                    "traffic": traffic_for(dominant, cfg), "bytes_per_launch": per_launch_bytes,
                     "avg_launch_ms": avg_ms, "launches": dom_n,
                     "share_of_step": dom_ms / roof_region_ms if roof_region_ms else None,
                     "timed_over": "the timed steps run call by call right after the graph-replayed ones"

@@ -1,5 +1,5 @@
 """bench.py's algorithmic byte model (what roofline.achieved divides by), on a
-batch whose runs are counted by hand.
+batch whose runs are counted by hand, and the rule for its measured traffic.
 
 Batch: key 7 once (a run of one lookup), key 5 twice and key 9 three times
 (short runs), key 3 forty times (a long run: more than 32 lookups, one chunk
@@ -58,3 +58,26 @@ def test_every_row_byte_is_counted_once_across_the_reduce_kernels():
     assert grads == s["B"] * ROW
     rmw = (s["U1"] + s["Um"] + s["Ul"]) * 4 * ROW
     assert rmw == s["U"] * 4 * ROW
+
+
+def test_traffic_figures_only_for_their_workload_and_source(tmp_path):
+    """roofline.traffic comes from a committed ncu figure only when it was taken
+    on the same workload (name, rows, batch) and the kernel's current source."""
+    import hashlib
+    import json
+
+    import workloads as W
+
+    src = os.path.join(ROOT, "paper_2504_01506_gb300", "csrc", bench.KERNEL_SOURCES[1])
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    dlrm = W.dlrm()
+    rec = {"workload": "dlrm", "rows": dlrm.n_keys, "batch_lookups": dlrm.batch, "bytes_per_launch": 123.0,
+           "source_sha": sha}
+    path = tmp_path / "traffic.json"
+    path.write_text(json.dumps({"1": rec}))
+    assert bench.traffic_for(1, dlrm, str(path)) == 123.0
+    assert bench.traffic_for(1, W.kg(), str(path)) is None                     # another workload
+    assert bench.traffic_for(1, W.scaled(dlrm, 10, 1), str(path)) is None      # same name, smaller table
+    assert bench.traffic_for(2, dlrm, str(path)) is None                       # no figure for the kernel
+    path.write_text(json.dumps({"1": dict(rec, source_sha="0" * 16)}))
+    assert bench.traffic_for(1, dlrm, str(path)) is None                       # kernel source changed since
