@@ -1,5 +1,7 @@
 // C ABI of the store (declared in include/mlkv_gpu.h): argument checks, the
-// table's memory, the order of kernels of each call, status and timing.
+// table's memory, the order of kernels of each call, the ordering of calls
+// across streams under a staleness bound (bulk-synchronous, stale-synchronous
+// or asynchronous, MLKV Section 3.3.1), status and timing.
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
