@@ -65,10 +65,23 @@ class EmbeddingStore:
             raise TypeError("keys must be a 1-d int64 tensor on the store's device")
         return keys.contiguous()
 
-    def _rows(self, x: torch.Tensor, n: int) -> torch.Tensor:
-        if x.dtype != torch.float32 or x.device != self.device or tuple(x.shape) != (n, self.dim):
-            raise TypeError(f"expected float32 [{n}, {self.dim}] on the store's device")
+    def _rows(self, x: torch.Tensor, n: int, device=None) -> torch.Tensor:
+        device = device or self.device
+        if x.dtype != torch.float32 or x.device != device or tuple(x.shape) != (n, self.dim):
+            raise TypeError(f"expected float32 [{n}, {self.dim}] on {device}")
         return x.contiguous()
+
+    def _check_out(self, out: torch.Tensor, n: int, device=None) -> torch.Tensor:
+        """An output buffer is written in place, so it must be contiguous already."""
+        if not out.is_contiguous():
+            raise TypeError("output buffer must be contiguous (it is written in place)")
+        return self._rows(out, n, device)
+
+    @staticmethod
+    def _host_keys(keys: torch.Tensor) -> torch.Tensor:
+        if keys.dtype != torch.int64 or keys.device.type != "cpu" or keys.dim() != 1:
+            raise TypeError("keys must be a 1-d int64 host tensor")
+        return keys.contiguous()
 
     def close(self):
         if getattr(self, "h", None):
@@ -89,7 +102,7 @@ class EmbeddingStore:
         n = keys.numel()
         if out is None:
             out = torch.empty((n, self.dim), dtype=torch.float32, device=self.device)
-        out = self._rows(out, n)
+        out = self._check_out(out, n)
         self._check(self.lib.mlkv_get(self.h, keys.data_ptr(), n, out.data_ptr(), _stream(self.device)))
         return out
 
@@ -194,15 +207,15 @@ class EmbeddingStore:
     def get_host(self, keys: torch.Tensor, out: torch.Tensor):
         """Get from and into host tensors (pinned for asynchronous copies); `out` is
         valid once the stream has synchronised."""
-        if keys.device.type != "cpu" or out.device.type != "cpu":
-            raise TypeError("get_host takes host tensors")
+        keys = self._host_keys(keys)
+        out = self._check_out(out, keys.numel(), torch.device("cpu"))
         self._check(self.lib.mlkv_get_host(self.h, keys.data_ptr(), keys.numel(), out.data_ptr(),
                                            _stream(self.device)))
 
     def apply_grad_host(self, keys: torch.Tensor, grads: torch.Tensor):
         """apply_grad from host tensors (copied to the device inside the call)."""
-        if keys.device.type != "cpu" or grads.device.type != "cpu":
-            raise TypeError("apply_grad_host takes host tensors")
+        keys = self._host_keys(keys)
+        grads = self._rows(grads, keys.numel(), torch.device("cpu"))
         self._check(self.lib.mlkv_apply_grad_host(self.h, keys.data_ptr(), keys.numel(),
                                                   grads.data_ptr(), _stream(self.device)))
 
