@@ -107,3 +107,30 @@ def test_binding_constants_match_header():
             checked += 1
     assert checked >= 20  # status codes, kernel ids, flags and limits
     assert re.search(r"#define MLKV_STALENESS_ASYNC INT64_MAX\b", src) and _lib.STALENESS_ASYNC == 2**63 - 1
+
+
+def test_open_validates_its_config_without_gpu(lib):
+    """mlkv_open checks every field before its first CUDA call: each bad config
+    returns its status here, where no GPU is present."""
+    from paper_2504_01506_gb300 import _lib
+
+    bound = _lib.load()
+    good = dict(dim=8, capacity=100, max_batch=10, lr=0.01, eps=1e-8, state_init=0.0, init_lo=-0.01,
+                init_hi=0.01, seed=1, insert_on_miss=1, staleness_bound=0, hbm_cache_rows=0, flags=0, reserved=0)
+    cases = [
+        (dict(dim=0), _lib.ERR_INVALID), (dict(dim=1025), _lib.ERR_INVALID), (dict(dim=258), _lib.ERR_INVALID),
+        (dict(capacity=0), _lib.ERR_INVALID), (dict(capacity=2**31 - 2), _lib.ERR_INVALID),
+        (dict(max_batch=0), _lib.ERR_INVALID), (dict(max_batch=2**30), _lib.ERR_INVALID),
+        (dict(reserved=1), _lib.ERR_INVALID), (dict(flags=1), _lib.ERR_INVALID),
+        (dict(init_lo=0.5, init_hi=0.1), _lib.ERR_INVALID), (dict(init_lo=float("nan")), _lib.ERR_INVALID),
+        (dict(staleness_bound=-1), _lib.ERR_INVALID),
+        (dict(staleness_bound=1, hbm_cache_rows=1000), _lib.ERR_UNSUPPORTED),
+        (dict(staleness_bound=_lib.STALENESS_ASYNC, hbm_cache_rows=1000), _lib.ERR_UNSUPPORTED),
+        (dict(hbm_cache_rows=-1), _lib.ERR_INVALID),
+        (dict(hbm_cache_rows=2 * 10 + 63), _lib.ERR_INVALID),  # below two batches and 64 lines
+    ]
+    for over, code in cases:
+        cfg = _lib.Config(**dict(good, **over))
+        h = ctypes.c_void_p()
+        assert bound.mlkv_open(ctypes.byref(cfg), ctypes.byref(h)) == code, over
+        assert not h.value, over
