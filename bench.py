@@ -166,8 +166,8 @@ def batch_stats(keys: np.ndarray, d: int) -> dict:
         "reduce_long": Bl * (row + 4) + items * row,
         # chunk sums read, row and state read and written once per long run
         "long_combine": items * row + Ul * 4 * row,
-        # whole step (the survey's accounting: keys twice, output + grads, index
-        # sector + Get row read + row/state RMW per distinct key)
+        # whole step, what the method must move: keys twice, output + grads per
+        # lookup; index sector + Get row read + row/state RMW per distinct key
         "step": B * (16 + 2 * row) + U * (32 + 5 * row),
     }
 

@@ -45,7 +45,7 @@ def test_bytes_per_kernel():
     assert bench.kernel_bytes(s, 7, 3) == 1 * ROW + 1 * 4 * ROW
     # the sort's scatter pass: (row id, position) read and written per lookup
     assert bench.kernel_bytes(s, 3, 3) == 46 * 16
-    # the whole step, the survey's accounting: B(16 + 8d) + U(32 + 20d)
+    # the whole step, what the method must move: B(16 + 8d) + U(32 + 20d)
     assert s["step"] == 46 * (16 + 8 * D) + 4 * (32 + 20 * D)
 
 
