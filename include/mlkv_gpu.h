@@ -139,7 +139,8 @@ typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
  * apply waits for the call issued before it on the other stream (the Get of
  * its keys) and for the apply before it; it inserts no key (an absent key is
  * skipped and MLKV_ERR_NOT_FOUND recorded).  Every other call waits for every
- * apply issued before it.  Rows and state after the applies are what
+ * apply issued before it (mlkv_dump_keys reads only the index, which applies
+ * do not change).  Rows and state after the applies are what
  * bulk-synchronous calls give.  Such a table's calls cannot be captured into a
  * graph (MLKV_ERR_UNSUPPORTED). */
 
