@@ -99,3 +99,28 @@ def test_full_size_batches():
         c = W.ALL[name]()
         b = c.batch_keys(0)
         assert len(b) == want == c.batch
+
+
+@pytest.mark.parametrize("make", [W.ycsb, W.ycsb_uniform])
+def test_ycsb_batches(make):
+    """A YCSB-shaped batch: 1,048,576 operations over 50M records of 256 fp32,
+    each a Get or a Put by a fair coin (the 50/50 mix), written values
+    N(0, 0.01); keys Zipf(0.99) scattered over the records, or uniform."""
+    c = W.scaled(make(), 50, 8)  # 1M records, batches of 131,072: the same distributions
+    r, w, v = c.ops(0)
+    n = len(r) + len(w)
+    assert n == c.batch
+    assert abs(len(r) / n - 0.5) < 4 * math.sqrt(0.25 / n)
+    assert v.shape == (len(w), 256) and v.dtype == np.float32
+    assert abs(float(v.std()) - 0.01) < 1e-4 and abs(float(v.mean())) < 1e-4
+    keys = np.concatenate([r, w])
+    assert keys.min() >= 0 and keys.max() < c.n_keys
+    _, counts = np.unique(keys, return_counts=True)
+    if c.alpha:
+        # Zipf(0.99) over N records: the hottest key takes 1 / H(N, 0.99) of the lookups
+        want = 1.0 / float(np.sum(np.arange(1, c.n_keys + 1, dtype=np.float64) ** -0.99))
+        assert abs(counts.max() / n - want) < 0.1 * want
+    else:
+        assert counts.max() < 10  # uniform over 1M records: no hot key
+    r2, w2, v2 = c.ops(0)
+    assert np.array_equal(r, r2) and np.array_equal(w, w2) and np.array_equal(v, v2)  # seeded
