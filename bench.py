@@ -662,6 +662,7 @@ def run_ours(args, cfg):
             "achieved_gbs": achieved_step, "hbm_frac_measured": achieved_step / hbm_peak,
             "hbm_frac_nominal": achieved_step / NOMINAL_HBM_GBS,
             "distinct_per_step": float(np.mean([s["U"] for s in stats])),
+            "distinct_rows_per_s": float(np.mean([s["U"] for s in stats])) * world * args.steps / (elapsed_ms / 1e3),
             "roofline": roofline, "kernel_ms_one_step": {KERNEL_NAMES[k]: v for k, v in kernel_ms.items()},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clocks.summary(),
             "step_launch": (f"one CUDA graph replay per step (the Get and the {'Put' if kv else 'apply'} of the "
