@@ -14,13 +14,24 @@ inside the timed region; `roofline` is the dominant kernel's algorithmic bytes
 per launch over its CUDA-event duration against the measured HBM copy peak;
 `cpu_baseline` is the oracle (single thread, host cores) on a bounded sample.
 
+With the default DLRM workload at N=1 the same process then measures the
+knowledge-graph, GNN and tiered workloads one after another (each store closed
+before the next opens) and reports them under `per_config`, each with its own
+roofline, clocks and oracle baseline.
+
+`--gpus N` without a launcher's environment starts N replica ranks itself
+(torch.distributed.run on this host, one process per GPU).
+
 --impl reference times the oracle itself on the host, as the reference arm.
 """
 import argparse
 import ctypes
+import gc
 import hashlib
 import json
 import os
+import platform
+import socket
 import statistics
 import subprocess
 import sys
@@ -56,39 +67,57 @@ def peaks():
 # --- clocks during the timed region ---------------------------------------------
 class ClockSampler:
     """Samples SM clock and clock-event reasons with nvidia-smi (-lms) and, where
-    the driver's NVML library loads, a fast NVML poll (short timed regions)."""
+    the driver's NVML library loads, a fast NVML poll.  NVML samples carry their
+    host time, so the summary can say how many fell inside the timed region."""
 
     REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
                0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
 
     def __init__(self, gpu_index: int):
         self.idx = gpu_index
-        self.samples = []  # (sm_mhz, max_mhz, reasons_mask)
+        self.samples = []  # (host time or None, sm_mhz, max_mhz, reasons_mask, source)
         self._stop = threading.Event()
         self._smi = None
         self._thread = None
         self._nvml = None
         self._handle = None
+        self._get_reasons = None
+        self.nvml_status = "not loaded"
         try:
             nv = ctypes.CDLL("libnvidia-ml.so.1")
-            if nv.nvmlInit_v2() == 0:
+            rc = nv.nvmlInit_v2()
+            if rc != 0:
+                self.nvml_status = f"nvmlInit_v2 returned {rc}"
+            else:
                 h = ctypes.c_void_p()
-                if nv.nvmlDeviceGetHandleByIndex_v2(gpu_index, ctypes.byref(h)) == 0:
-                    self._nvml, self._handle = nv, h
-        except OSError:
-            pass
+                rc = nv.nvmlDeviceGetHandleByIndex_v2(gpu_index, ctypes.byref(h))
+                fn = None
+                for name in ("nvmlDeviceGetCurrentClocksEventReasons", "nvmlDeviceGetCurrentClocksThrottleReasons"):
+                    try:
+                        fn = getattr(nv, name)
+                        break
+                    except AttributeError:
+                        continue
+                if rc != 0:
+                    self.nvml_status = f"nvmlDeviceGetHandleByIndex_v2 returned {rc}"
+                elif fn is None:
+                    self.nvml_status = "no clock-event-reasons entry point"
+                else:
+                    self._nvml, self._handle, self._get_reasons = nv, h, fn
+                    self.nvml_status = "ok"
+        except OSError as e:
+            self.nvml_status = f"libnvidia-ml.so.1: {e}"
 
     def _poll(self):
-        nv, h = self._nvml, self._handle
+        nv, h, reasons = self._nvml, self._handle, self._get_reasons
         clk, mx, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
-        get_reasons = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
-            getattr(nv, "nvmlDeviceGetCurrentClocksThrottleReasons")
         while not self._stop.is_set():
+            t = time.perf_counter()
             if nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0 and \
                     nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0 and \
-                    get_reasons(h, ctypes.byref(rs)) == 0:
-                self.samples.append((clk.value, mx.value, rs.value))
-            time.sleep(0.002)
+                    reasons(h, ctypes.byref(rs)) == 0:
+                self.samples.append((t, clk.value, mx.value, rs.value, "nvml"))
+            time.sleep(0.001)
 
     def start(self):
         try:
@@ -120,7 +149,7 @@ class ClockSampler:
                     f = [x.strip() for x in ln.split(",")]
                     if len(f) >= 5 and f[1].isdigit():
                         mask = int(f[4], 16) if f[4].startswith("0x") else 0
-                        self.samples.append((int(f[1]), int(f[2]), mask))
+                        self.samples.append((None, int(f[1]), int(f[2]), mask, "nvidia-smi"))
             except OSError:
                 pass
             try:
@@ -128,16 +157,49 @@ class ClockSampler:
             except OSError:
                 pass
 
-    def summary(self):
+    def summary(self, timed=None, window=None):
+        """Median SM clock, max clock and the union of reasons over every sample
+        of the window; `timed` = (t0, t1) host times of the timed region, to
+        count the NVML samples inside it."""
+        out = {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": len(self.samples),
+               "nvml": self.nvml_status}
+        if window:
+            out["window"] = window
+        if timed is not None:
+            out["samples_in_timed_region"] = sum(1 for s in self.samples
+                                                 if s[0] is not None and timed[0] <= s[0] <= timed[1])
         if not self.samples:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+            return out
         mask = 0
-        for _, _, r in self.samples:
-            mask |= r
-        return {"sm_mhz": statistics.median(s[0] for s in self.samples),
-                "sm_max_mhz": max(s[1] for s in self.samples),
-                "reasons": [v for k, v in sorted(self.REASONS.items()) if mask & k],
-                "samples": len(self.samples)}
+        for s in self.samples:
+            mask |= s[3]
+        out.update(sm_mhz=statistics.median(s[1] for s in self.samples),
+                   sm_max_mhz=max(s[2] for s in self.samples),
+                   reasons=[v for k, v in sorted(self.REASONS.items()) if mask & k])
+        return out
+
+
+def cpu_description() -> dict:
+    """Model and count of the host's cores (lscpu, else /proc/cpuinfo)."""
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.lower().startswith("model name:"):
+                model = ln.split(":", 1)[1].strip()
+                break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    if not model:
+        try:
+            for ln in open("/proc/cpuinfo"):
+                if ln.lower().startswith("model name"):
+                    model = ln.split(":", 1)[1].strip()
+                    break
+        except OSError:
+            pass
+    return {"cpu_model": model or platform.processor() or platform.machine(), "host_cores": os.cpu_count(),
+            "machine": platform.machine()}
 
 
 # --- workload statistics (algorithmic bytes) ----------------------------------------
@@ -238,9 +300,13 @@ def traffic_for(kid: int, cfg, path=None):
 
 # --- distributed plumbing (replicas) --------------------------------------------------
 def dist_setup(n_gpus: int):
+    """This process's rank in a launched job (RANK / LOCAL_RANK / WORLD_SIZE from
+    the launcher); a job of more than one rank joins a process group."""
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != n_gpus:
+        raise SystemExit(f"--gpus {n_gpus} but the launcher started {world} rank(s)")
     if world > 1:
         import torch.distributed as dist
 
@@ -248,6 +314,21 @@ def dist_setup(n_gpus: int):
         dist.init_process_group(backend=backend)
         return dist, rank, local, world
     return None, 0, 0, 1
+
+
+def _free_port() -> int:
+    with socket.socket() as sk:
+        sk.bind(("127.0.0.1", 0))
+        return sk.getsockname()[1]
+
+
+def launch_replicas(n: int, argv) -> int:
+    """`--gpus N` started without a launcher: re-runs this script as N ranks on
+    this host (torch.distributed.run, rendezvous on 127.0.0.1), one per GPU, and
+    returns the job's exit status.  Rank 0 prints the JSON line."""
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={n}",
+           "--master-addr=127.0.0.1", f"--master-port={_free_port()}", os.path.abspath(__file__), *argv]
+    return subprocess.run(cmd, cwd=ROOT).returncode
 
 
 def barrier(dist, torch, sync_cuda: bool = True):
@@ -317,24 +398,41 @@ def oracle_ycsb_steps(cfg, steps: int, sample: int, warmup: int = 0):
 
 
 def run_reference(args, cfg):
-    dist, rank, _, world = None, int(os.environ.get("RANK", "0")), 0, int(os.environ.get("WORLD_SIZE", "1"))
-    if rank != 0:
-        return 0
-    sample = max(1, cfg.batch // 8)
-    kv = isinstance(cfg, W.YcsbConfig)
-    value, dt = (oracle_ycsb_steps if kv else oracle_steps)(cfg, args.steps, sample, args.warmup)
-    line = {
-        "impl": "reference", "metric": METRIC_YCSB if kv else METRIC, "value": value,
-        "unit": UNIT_YCSB if kv else UNIT, "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-        "data": "synthetic", "config": workload_config(cfg),
-        "cpu_baseline": {"value": value, "unit": UNIT_YCSB if kv else UNIT, "cores": 1, "kind": "oracle",
-                         "sample": f"first {sample} of {cfg.batch} operations of each step"},
-        "e2e": {"value": value, "unit": UNIT_YCSB if kv else UNIT, "h2d_bytes_per_step": 0,
-                "d2h_bytes_per_step": 0},
-    }
-    print(json.dumps(line), flush=True)
+    """The reference arm: the oracle on one host thread, rank 0 only.  Under N
+    ranks every rank joins a gloo group (no GPU work), so the line's n_gpus is
+    the job's world size; the other ranks do nothing else."""
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if world != args.gpus:
+        raise SystemExit(f"--gpus {args.gpus} but the launcher started {world} rank(s)")
+    dist = None
+    if world > 1:
+        import datetime
+
+        import torch.distributed as dist
+
+        dist.init_process_group(backend="gloo", timeout=datetime.timedelta(minutes=30))
+        world = dist.get_world_size()
+    if rank == 0:
+        sample = max(1, cfg.batch // 8)
+        kv = isinstance(cfg, W.YcsbConfig)
+        value, dt = (oracle_ycsb_steps if kv else oracle_steps)(cfg, args.steps, sample, args.warmup)
+        line = {
+            "impl": "reference", "metric": METRIC_YCSB if kv else METRIC, "value": value,
+            "unit": UNIT_YCSB if kv else UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": dict(workload_config(cfg), parallelism=f"replicas{world}"),
+            "cpu_baseline": dict({"value": value, "unit": UNIT_YCSB if kv else UNIT, "cores": 1, "kind": "oracle",
+                                  "sample": f"first {sample} of {cfg.batch} operations of each step"},
+                                 **cpu_description()),
+            "e2e": {"value": value, "unit": UNIT_YCSB if kv else UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0},
+        }
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
     return 0
 
 
@@ -376,30 +474,34 @@ def workload_config(cfg) -> dict:
 
 
 # --- our arm ----------------------------------------------------------------------------
-def run_ours(args, cfg):
+CLOCK_WINDOW_S = 1.0  # clocks are sampled over the timed region and, after it, the same steps to this length
+
+
+def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int) -> dict:
+    """Opens the store of `cfg`, preloads it, times `steps` Get + apply steps (or
+    Get + Put batches) and returns the measured fields; the store is closed on
+    return.  `headline`: also the end-to-end host-buffer leg."""
     import torch
 
-    from paper_2504_01506_gb300 import EmbeddingStore, _lib
+    from paper_2504_01506_gb300 import EmbeddingStore
 
-    dist, rank, local, world = dist_setup(args.gpus)
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
     hbm_peak, peak_kind = peaks()
-
+    t_begin = time.perf_counter()
     tiered = cfg.hbm_cache_rows > 0
     kv = isinstance(cfg, W.YcsbConfig)
+    staleness = args.staleness if headline else 0
     store = EmbeddingStore(dim=cfg.dim, capacity=cfg.n_keys, max_batch=cfg.batch, lr=cfg.lr, eps=cfg.eps,
                            state_init=cfg.state_init, init_lo=cfg.init_lo, init_hi=cfg.init_hi,
                            seed=cfg.seed, hbm_cache_rows=cfg.hbm_cache_rows,
-                           staleness_bound=args.staleness, device=dev)
+                           staleness_bound=staleness, device=dev)
     # stale-synchronous steps: each Get on one stream, each apply on another; the
     # table lets Get(t) run beside the last `staleness` applies before it
-    s_get = torch.cuda.Stream(dev) if args.staleness else None
-    s_apply = torch.cuda.Stream(dev) if args.staleness else None
+    s_get = torch.cuda.Stream(dev) if staleness else None
+    s_apply = torch.cuda.Stream(dev) if staleness else None
     # preload every key of the table (untimed), in preload order
     chunk = cfg.batch
-    for s in range(0, cfg.n_keys, chunk):
-        store.insert(torch.from_numpy(cfg.preload_keys(s, s + chunk)).to(dev))
+    for s0 in range(0, cfg.n_keys, chunk):
+        store.insert(torch.from_numpy(cfg.preload_keys(s0, s0 + chunk)).to(dev))
     assert store.sync() == 0, "preload failed"
 
     if tiered and args.tier_prefill:
@@ -413,31 +515,32 @@ def run_ours(args, cfg):
             store.get(k)
             store.apply_grad(k, zeros[:k.numel()])
         assert store.sync() == 0, "prefill failed"
+        del zeros
 
     # The HBM store cycles a pool of batches.  The tiered store gets a fresh batch
     # every step (a cycled pool would end up resident in its cache): one per
     # kernel-class prepass step, warm-up step, timed step, and the last look-ahead.
     kinds = (1, 2, 9) if kv else (1, 2, 3, 4, 5, 6, 7, 10) + ((8,) if tiered else ())
     base = len(kinds) if tiered else 0
-    pool = base + args.warmup + args.steps + 1 if tiered else max(1, min(args.pool, args.steps + args.warmup))
+    pool = base + args.warmup + steps + 1 if tiered else max(1, min(args.pool, steps + args.warmup))
     ngrad = max(1, min(args.pool, pool))
     out = torch.empty((cfg.batch, cfg.dim), dtype=torch.float32, device=dev)
     passes = (int(cfg.n_keys).bit_length() + 7) // 8
     if kv:  # batches of Gets, then Puts
         ops_d = []
         stats = []
-        for s in range(pool):
-            r, w, v = cfg.ops(s)
+        for s0 in range(pool):
+            r, w, v = cfg.ops(s0)
             ops_d.append((torch.from_numpy(r).to(dev), torch.from_numpy(w).to(dev), torch.from_numpy(v).to(dev)))
             stats.append(ycsb_stats(r, w, cfg.dim))
         keys_h = None
     else:
-        keys_h = [cfg.batch_keys(s) for s in range(pool)]
+        keys_h = [cfg.batch_keys(s0) for s0 in range(pool)]
         keys_d = [torch.from_numpy(k).to(dev) for k in keys_h]
         gen = torch.Generator(device=dev)
         grads_d = []
-        for s in range(ngrad):
-            gen.manual_seed(cfg.seed * 1000 + s)
+        for s0 in range(ngrad):
+            gen.manual_seed(cfg.seed * 1000 + s0)
             grads_d.append(torch.randn((cfg.batch, cfg.dim), generator=gen, device=dev) * cfg.grad_sigma)
         stats = [batch_stats(k, cfg.dim) for k in keys_h]
 
@@ -448,7 +551,7 @@ def run_ours(args, cfg):
             store.get(r, out=out[:r.numel()])
             store.put(w, v)
             return
-        if args.staleness:
+        if staleness:
             with torch.cuda.stream(s_get):
                 store.get(keys_d[j], out=out)
             with torch.cuda.stream(s_apply):
@@ -475,7 +578,7 @@ def run_ours(args, cfg):
     # An HBM-resident step is captured into a CUDA graph per batch (the Get and
     # the apply of that batch) and replayed: the calls' work is device-driven,
     # so a replay does all of it with one launch from the host.
-    use_graphs = not tiered and args.graphs and not args.staleness  # stale-synchronous calls refuse capture
+    use_graphs = not tiered and args.graphs and not staleness  # stale-synchronous calls refuse capture
     graphs, launches_per_graph = [], 0
     if use_graphs:
         cap = torch.cuda.Stream(dev)
@@ -510,24 +613,40 @@ def run_ours(args, cfg):
     clocks.start()
     if args.profile:
         torch.cuda.profiler.start()
+    t_timed0 = time.perf_counter()
     ev0.record(stream)
     for side in (s_get, s_apply):
         if side is not None:
             side.wait_stream(stream)
-    for i in range(args.steps):
+    for i in range(steps):
         timed_step(base + args.warmup + i)
     for side in (s_get, s_apply):
         if side is not None:
             stream.wait_stream(side)
     ev1.record(stream)
     barrier(dist, torch)
+    t_timed1 = time.perf_counter()
     if args.profile:
         torch.cuda.profiler.stop()
-    clocks.stop()
-    launches = launches_per_graph * args.steps if use_graphs else store.launch_count() - launches0
+    launches = launches_per_graph * steps if use_graphs else store.launch_count() - launches0
     tier1 = store.tier_stats()
+    if not use_graphs:  # the dominant kernel's launches of the timed region
+        dom_ms, dom_n = store.kernel_time()
+        store.time_kernel(0)
+    # a timed region shorter than the clock window: the sampler keeps running over
+    # the same steps (untimed) right after it, so the record has enough samples
+    n_extra = 0
+    while time.perf_counter() - t_timed0 < CLOCK_WINDOW_S and n_extra < 100_000:
+        for i in range(8):
+            timed_step(base + args.warmup + (n_extra + i) % steps)
+        n_extra += 8
+        torch.cuda.synchronize(dev)
+    clocks.stop()
+    window = (f"the timed region ({steps} steps) and {n_extra} more of the same steps right after it "
+              f"({time.perf_counter() - t_timed0:.2f} s)" if n_extra else f"the timed region ({steps} steps)")
+    clock_summary = clocks.summary(timed=(t_timed0, t_timed1), window=window)
     assert store.sync() == 0, "device status set during the timed region"
-    elapsed_ms, value = job_throughput(dist, torch, ev0.elapsed_time(ev1), cfg.batch * args.steps)
+    elapsed_ms, value = job_throughput(dist, torch, ev0.elapsed_time(ev1), cfg.batch * steps)
     roof_region_ms = elapsed_ms
     if use_graphs:
         # event timings inside a graph are overwritten at every replay: the
@@ -535,16 +654,16 @@ def run_ours(args, cfg):
         store.time_kernel(dominant)
         r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         r0.record(stream)
-        for i in range(args.steps):
+        for i in range(steps):
             step(base + args.warmup + i)
         r1.record(stream)
         torch.cuda.synchronize(dev)
         roof_region_ms = r0.elapsed_time(r1)
-    dom_ms, dom_n = store.kernel_time()
-    store.time_kernel(0)
+        dom_ms, dom_n = store.kernel_time()
+        store.time_kernel(0)
     assert store.sync() == 0, "device status set during the roofline region"
-    step_bytes = np.mean([s["step"] for s in stats])
-    achieved_step = step_bytes * args.steps / (elapsed_ms / 1e3) / 1e9
+    step_bytes = np.mean([st["step"] for st in stats])
+    achieved_step = step_bytes * steps / (elapsed_ms / 1e3) / 1e9
 
     # roofline of the dominant kernel over the timed region
     avg_ms = dom_ms / max(dom_n, 1)
@@ -555,13 +674,14 @@ def run_ours(args, cfg):
         link_bytes = (fetched + written) * slot_bytes
         link_gbs = link_bytes / (elapsed_ms / 1e3) / 1e9
         peak = dma_peak(torch, dev)
-        tier = {"host_rows": cfg.n_keys, "cache_rows": cfg.hbm_cache_rows, "rows_fetched_per_step": fetched / args.steps,
-                "rows_written_back_per_step": written / args.steps,
-                "sweep_lines_per_step": (tier1[2] - tier0[2]) / args.steps,
-                "link_bytes_per_step": link_bytes / args.steps, "link_gbs_over_step": link_gbs,
+        tier = {"host_rows": cfg.n_keys, "cache_rows": cfg.hbm_cache_rows, "rows_fetched_per_step": fetched / steps,
+                "rows_written_back_per_step": written / steps,
+                "sweep_lines_per_step": (tier1[2] - tier0[2]) / steps,
+                "link_bytes_per_step": link_bytes / steps, "link_gbs_over_step": link_gbs,
                 "dma_peak_gbs": peak, "lookahead": bool(args.lookahead), "prefilled": bool(args.tier_prefill)}
     if dominant == 8:
-        # the swap kernel moves each fetched row in and each victim out over the host link
+        # the swap kernel moves each fetched row in and each victim out over the
+        # host link (its launches timed over the timed region)
         per_launch_bytes = link_bytes / max(dom_n, 1)
         achieved = per_launch_bytes / (avg_ms / 1e3) / 1e9
         roofline = {"bound": "host-link", "kernel": KERNEL_NAMES[8], "achieved": achieved, "peak": peak["h2d"],
@@ -570,7 +690,7 @@ def run_ours(args, cfg):
                     "traffic": None, "bytes_per_launch": per_launch_bytes, "avg_launch_ms": avg_ms,
                     "launches": dom_n, "share_of_step": dom_ms / roof_region_ms if roof_region_ms else None}
     else:
-        steps_idx = [(base + args.warmup + i) % pool for i in range(args.steps)]
+        steps_idx = [(base + args.warmup + i) % pool for i in range(steps)]
         per_launch_bytes = np.mean([kernel_bytes(stats[j], dominant, passes) for j in steps_idx])
         achieved = per_launch_bytes / (avg_ms / 1e3) / 1e9
         roofline = {"bound": "hbm", "kernel": KERNEL_NAMES[dominant], "achieved": achieved, "peak": hbm_peak,
@@ -583,14 +703,14 @@ def run_ours(args, cfg):
 
     # end to end through the host-buffer calls (copies inside the timed region)
     e2e = None
-    if not args.no_e2e and kv:
+    if headline and not args.no_e2e and kv:
         # keys and written values from pinned host memory, the Get's output back,
         # around the store's calls
         r, w, v = ops_d[0]
         hr, hw, hv = r.cpu().pin_memory(), w.cpu().pin_memory(), v.cpu().pin_memory()
         hout = torch.empty((r.numel(), cfg.dim), dtype=torch.float32).pin_memory()
         dr, dw, dv = torch.empty_like(r), torch.empty_like(w), torch.empty_like(v)
-        e2e_steps = max(1, min(args.steps, 20))
+        e2e_steps = max(1, min(steps, 20))
 
         def kv_e2e():
             dr.copy_(hr, non_blocking=True)
@@ -616,12 +736,12 @@ def run_ours(args, cfg):
         e2e = {"value": cfg.batch * e2e_steps * world / (e_ms / 1e3), "unit": UNIT_YCSB, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                "link_gbs": (h2d + d2h) * e2e_steps / (e_ms / 1e3) / 1e9}
-    if not args.no_e2e and not tiered and not kv:
+    if headline and not args.no_e2e and not tiered and not kv:
         e2e_pool = min(pool, 2)
         hk = [torch.from_numpy(keys_h[j]).pin_memory() for j in range(e2e_pool)]
         hg = [grads_d[j % ngrad].cpu().pin_memory() for j in range(e2e_pool)]
         hout = torch.empty((cfg.batch, cfg.dim), dtype=torch.float32).pin_memory()
-        e2e_steps = max(1, min(args.steps, 20))
+        e2e_steps = max(1, min(steps, 20))
         for i in range(2):
             store.get_host(hk[i % e2e_pool], hout)
             store.apply_grad_host(hk[i % e2e_pool], hg[i % e2e_pool])
@@ -640,40 +760,92 @@ def run_ours(args, cfg):
         e2e = {"value": cfg.batch * e2e_steps * world / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                "link_gbs": (h2d + d2h) * e2e_steps / (e_ms / 1e3) / 1e9}
+    store.close()
+    del graphs, out
+    if not kv:
+        del keys_d, grads_d
+    else:
+        del ops_d
+    gc.collect()
+    torch.cuda.empty_cache()
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         sample = max(1, cfg.batch // 8)
-        steps = max(1, args.cpu_steps)
-        v, dt = (oracle_ycsb_steps if kv else oracle_steps)(cfg, steps, sample)
-        cpu = {"value": v, "unit": UNIT_YCSB if kv else UNIT, "cores": 1, "kind": "oracle",
-               "sample": f"{steps} steps x first {sample} of {cfg.batch} "
-                         f"{'operations (Get + Put)' if kv else 'lookups (Get + apply)'}, "
-                         f"{dt:.1f} s on one host thread"}
+        csteps = max(1, args.cpu_steps)
+        v, dt = (oracle_ycsb_steps if kv else oracle_steps)(cfg, csteps, sample)
+        cpu = dict({"value": v, "unit": UNIT_YCSB if kv else UNIT, "cores": 1, "kind": "oracle",
+                    "sample": f"{csteps} steps x first {sample} of {cfg.batch} "
+                              f"{'operations (Get + Put)' if kv else 'lookups (Get + apply)'}, "
+                              f"{dt:.1f} s on one host thread"}, **cpu_description())
 
+    res = {
+        "value": value, "ms_per_step": elapsed_ms / steps, "steps": steps,
+        "config": dict(workload_config(cfg), parallelism=f"replicas{world}", distinct_batches=pool,
+                       **({"staleness_bound": staleness} if staleness else {})),
+        "achieved_gbs": achieved_step, "hbm_frac_measured": achieved_step / hbm_peak,
+        "hbm_frac_nominal": achieved_step / NOMINAL_HBM_GBS,
+        "distinct_per_step": float(np.mean([st["U"] for st in stats])),
+        "distinct_rows_per_s": float(np.mean([st["U"] for st in stats])) * world * steps / (elapsed_ms / 1e3),
+        "roofline": roofline, "kernel_ms_one_step": {KERNEL_NAMES[k]: v for k, v in kernel_ms.items()},
+        "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clock_summary,
+        "step_launch": (f"one CUDA graph replay per step (the Get and the {'Put' if kv else 'apply'} of the "
+                        f"batch, captured)" if use_graphs else
+                        "each call launched from the host" + (", Gets and applies on two streams"
+                                                              if staleness else "")),
+        "wall_s": time.perf_counter() - t_begin,
+    }
+    if tier is not None:
+        res["tier"] = tier
+    return res
+
+
+def per_config_names(args, world) -> list:
+    if args.per_config == "none" or world > 1:
+        return []
+    if args.per_config == "auto":
+        return ["kg", "gnn", "tiered"] if args.config == "dlrm" and args.scale == 1 and not args.staleness else []
+    return [c for c in args.per_config.split(",") if c]
+
+
+def tier_scaled(cfg, args):
+    """The tiered workload with its host tier scaled to the machine's host memory
+    (and the HBM cache with it: the same cached fraction of the rows)."""
+    full_rows, full_cache = cfg.n_keys, cfg.hbm_cache_rows
+    cfg.n_keys = args.tier_rows
+    cfg.hbm_cache_rows = args.tier_cache_rows or int(full_cache * args.tier_rows / full_rows)
+    return cfg
+
+
+def run_ours(args, cfg):
+    import torch
+
+    dist, rank, local, world = dist_setup(args.gpus)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    kv = isinstance(cfg, W.YcsbConfig)
+    res = measure(args, cfg, dist, rank, local, world, dev, headline=True, steps=args.steps)
+    extra = {}
+    for name in per_config_names(args, world):
+        c = W.ALL[name]()
+        if name == "tiered":
+            c = tier_scaled(c, args)
+        # each workload's own step count (the timed region stays short), at most --steps
+        r = measure(args, c, dist, rank, local, world, dev, headline=False, steps=min(args.steps, c.steps))
+        r.pop("e2e", None)
+        r["metric"] = METRIC
+        r["unit"] = UNIT
+        extra[name] = r
     if rank == 0:
         line = {
-            "metric": METRIC_YCSB if kv else METRIC, "value": value, "unit": UNIT_YCSB if kv else UNIT,
-            "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": dict(workload_config(cfg), parallelism=f"replicas{world}", distinct_batches=pool,
-                           **({"staleness_bound": args.staleness} if args.staleness else {})),
-            "achieved_gbs": achieved_step, "hbm_frac_measured": achieved_step / hbm_peak,
-            "hbm_frac_nominal": achieved_step / NOMINAL_HBM_GBS,
-            "distinct_per_step": float(np.mean([s["U"] for s in stats])),
-            "distinct_rows_per_s": float(np.mean([s["U"] for s in stats])) * world * args.steps / (elapsed_ms / 1e3),
-            "roofline": roofline, "kernel_ms_one_step": {KERNEL_NAMES[k]: v for k, v in kernel_ms.items()},
-            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clocks.summary(),
-            "step_launch": (f"one CUDA graph replay per step (the Get and the {'Put' if kv else 'apply'} of the "
-                            f"batch, captured)" if use_graphs else
-                            "each call launched from the host" + (", Gets and applies on two streams"
-                                                                  if args.staleness else "")),
+            "metric": METRIC_YCSB if kv else METRIC, "value": res["value"], "unit": UNIT_YCSB if kv else UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": res["ms_per_step"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         }
-        if tier is not None:
-            line["tier"] = tier
+        line.update({k: v for k, v in res.items() if k not in ("value", "ms_per_step", "steps")})
+        if extra:
+            line["per_config"] = extra
         print(json.dumps(line), flush=True)
-    store.close()
     if dist is not None:
         dist.destroy_process_group()
     return 0
@@ -705,6 +877,9 @@ def main():
                     help="tiered config: no look-ahead; each Get fetches its own missing rows")
     ap.add_argument("--scale", type=int, default=1,
                     help="divide the table's rows by this (same batch); for small profiling cases")
+    ap.add_argument("--per-config", default="auto",
+                    help="workloads measured after the headline one in the same process, comma-separated "
+                         "(auto: kg,gnn,tiered after the default DLRM workload at N=1; none: no others)")
     ap.add_argument("--staleness", type=int, default=0,
                     help="HBM-resident training configs: open the table with this staleness bound (>= 1; "
                          "9223372036854775807 = asynchronous) and run Gets and applies on two streams")
@@ -713,13 +888,15 @@ def main():
         ap.error("--staleness takes a bound >= 1 and an HBM-resident training config")
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.gpus < 1:
+        ap.error("--gpus must be >= 1")
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        # no launcher: start the N replica ranks here
+        return launch_replicas(args.gpus, sys.argv[1:])
     cfg = W.ALL[args.config]()
     if args.config == "tiered":
-        # the host tier must fit the machine's host memory: scale the row count, and
-        # the HBM cache with it (same cached fraction of the rows)
-        full_rows, full_cache = cfg.n_keys, cfg.hbm_cache_rows
-        cfg.n_keys = args.tier_rows
-        cfg.hbm_cache_rows = args.tier_cache_rows or int(full_cache * args.tier_rows / full_rows)
+        # the host tier must fit the machine's host memory
+        cfg = tier_scaled(cfg, args)
     if args.scale > 1:
         cfg = W.scaled(cfg, args.scale, 1)
     if args.impl == "reference":

@@ -67,8 +67,10 @@ extern "C" {
 /* Segments (runs of one key in a gradient batch) of at most this many
  * occurrences are summed by one lane group in occurrence order, so their
  * Adagrad step is the same op sequence as a sequential fp32 statement of it.
- * Longer segments are summed in chunks of 64 lookups and the chunk sums added
- * in a fixed order: deterministic run to run, not the sequential rounding. */
+ * Longer segments are summed in chunks of 64 lookups with compensated (TwoSum)
+ * additions and the chunks' (sum, compensation) pairs combined in a fixed
+ * order, the sum rounded once: deterministic run to run and within about one
+ * rounding of the exact sum, not the sequential fp32 rounding. */
 #define MLKV_SEQ_SEGMENT_MAX 32
 
 /* Flags of mlkv_config.flags. */
@@ -148,10 +150,12 @@ typedef struct mlkv_table mlkv_table; /* opaque; owned by the library */
  * (capacity x 2 x dim fp32, rows padded to 32 bytes), the index (a power of
  * two >= 2 x capacity slots of 16 bytes) and scratch for max_batch.  With
  * hbm_cache_rows > 0 the rows + state are allocated in host memory instead
- * (capacity slots, huge-page backed, registered with CUDA and mapped), with an
- * HBM cache of hbm_cache_rows rows, a row -> location map (cache line or host
- * slot; a row fetched into the cache hands its host slot to the row it
- * evicts), and a side stream for look-ahead.
+ * (capacity slots of pinned host memory from the driver's virtual-memory API,
+ * cuMemCreate on the host NUMA node nearest the GPU in 1 GiB chunks, mapped for
+ * this device only; the CPU never touches it), with an HBM cache of
+ * hbm_cache_rows rows, a row -> location map (cache line or host slot; a row
+ * fetched into the cache hands its host slot to the row it evicts), and a side
+ * stream for look-ahead.
  * Returns MLKV_ERR_INVALID (bad field), MLKV_ERR_UNSUPPORTED
  * (staleness_bound non-zero with hbm_cache_rows > 0),
  * MLKV_ERR_NOMEM or MLKV_ERR_CUDA.  On success *out
@@ -236,10 +240,12 @@ int mlkv_dedup(mlkv_table* t, const int64_t* d_keys, int64_t n, int64_t* d_uniqu
                int32_t* d_counts, int64_t* d_num_unique, void* stream);
 
 /* Dedup of a batch of raw keys that allocates nothing.  The paper has no
- * counterpart; it is here for callers that may not allocate device memory at
- * the moment they need it: code that issues work while a stream is being
- * captured in global mode (where cudaMalloc is refused), or plugins of engines
- * that own every device allocation.  It needs no table.
+ * counterpart; it is here for callers that must not allocate device memory
+ * when they need a dedup: plugins running inside an engine that has reserved
+ * the device's memory up front and owns every allocation (a cudaMalloc of
+ * theirs can fail, or go behind the engine's accounting), and latency-bound
+ * loops where cudaMalloc / cudaFree are banned because they may synchronise
+ * the device and stall every stream.  It needs no table.
  *   d_keys: int64 [n], n <= MLKV_STATIC_MAX_KEYS (larger n: MLKV_ERR_INVALID,
  *   nothing enqueued).  Output: the distinct keys in ascending unsigned order
  *   in d_unique_keys (int64 [n]), their occurrence counts in d_counts
@@ -304,6 +310,23 @@ int mlkv_kernel_time(mlkv_table* t, double* total_ms, int64_t* launches);
 
 /* Distinct keys of the last gradient apply or dedup (synchronises). */
 int64_t mlkv_last_unique(mlkv_table* t);
+
+/* Host-side fault injection, for testing the error paths.  The paper has no
+ * counterpart (failure handling is not discussed there).  After
+ * mlkv_debug_fail(kind, nth), the nth operation of that kind the library
+ * attempts from then on (counting from 1, in any table or in mlkv_open) fails
+ * on the host without calling CUDA: for MLKV_FAULT_ALLOC a device or pinned
+ * host allocation (cudaMalloc, cudaHostAlloc, a host-tier chunk), which then
+ * returns MLKV_ERR_NOMEM; for MLKV_FAULT_COPY a host <-> device copy of a
+ * *_host call, which then returns MLKV_ERR_CUDA with nothing after it
+ * enqueued.  nth = 0 disarms.  One countdown per kind, shared by the whole
+ * process.  No GPU work is affected: nothing faults on the device.  A failed
+ * mlkv_open frees everything it allocated and leaves *out null; a failed
+ * *_host call leaves the table usable.  Returns MLKV_ERR_INVALID for an
+ * unknown kind or nth < 0. */
+#define MLKV_FAULT_ALLOC 1
+#define MLKV_FAULT_COPY 2
+int mlkv_debug_fail(int32_t kind, int64_t nth);
 
 /* Text of the last error this handle saw (static storage of the handle). */
 const char* mlkv_last_error(mlkv_table* t);

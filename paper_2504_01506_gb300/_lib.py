@@ -42,7 +42,10 @@ EXPORTED = [
     "mlkv_apply_grad_host", "mlkv_sync", "mlkv_clear_status", "mlkv_size", "mlkv_launch_count",
     "mlkv_time_kernel", "mlkv_kernel_time", "mlkv_last_unique", "mlkv_last_error",
     "mlkv_status_string", "mlkv_dedup_keys_static", "mlkv_tier_stats", "mlkv_import", "mlkv_dump_keys",
+    "mlkv_debug_fail",
 ]
+FAULT_ALLOC = 1
+FAULT_COPY = 2
 STATIC_MAX_KEYS = 65536
 
 
@@ -101,6 +104,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.mlkv_tier_stats.argtypes = [vp, ctypes.POINTER(i64), ctypes.POINTER(i64), ctypes.POINTER(i64)]
     lib.mlkv_import.argtypes = [vp, vp, i64, vp, vp, vp]
     lib.mlkv_dump_keys.argtypes = [vp, vp, i64, vp]
+    lib.mlkv_debug_fail.argtypes = [i32, i64]
     lib.mlkv_last_unique.argtypes = [vp]
     lib.mlkv_last_unique.restype = i64
     lib.mlkv_last_error.argtypes = [vp]
@@ -111,7 +115,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
                  "mlkv_lookahead", "mlkv_find", "mlkv_export", "mlkv_dedup", "mlkv_get_host",
                  "mlkv_apply_grad_host", "mlkv_sync", "mlkv_clear_status", "mlkv_time_kernel",
                  "mlkv_kernel_time", "mlkv_dedup_keys_static", "mlkv_tier_stats", "mlkv_import",
-                 "mlkv_dump_keys"):
+                 "mlkv_dump_keys", "mlkv_debug_fail"):
         getattr(lib, name).restype = i32
     _lib = lib
     return lib

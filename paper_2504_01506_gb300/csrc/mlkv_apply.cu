@@ -22,10 +22,16 @@
 //                 run's other positions are loaded together, the rest summed in
 //                 occurrence order, then the Adagrad step.
 //  k_long_sum     one lane group per chunk of kChunk lookups of a long run
-//                 (Zipf-hot keys reach 10^4-10^5 lookups): chunk sum to scratch.
-//  k_long_combine one block per long run: the chunk sums are split over the
-//                 block's lane groups in a fixed way, added in that order, and
-//                 the row updated.
+//                 (Zipf-hot keys reach 10^4-10^5 lookups): the chunk's sum,
+//                 compensated, to scratch as a (sum, compensation) pair.
+//  k_long_combine one block per long run: the chunk pairs are split over the
+//                 block's lane groups in a fixed way, added in that order with
+//                 compensation, the sum rounded once, and the row updated.
+// Long runs are summed with compensation because the Adagrad step is
+// ill-conditioned where a summed gradient element lands near eps (with zero
+// state, u = lr * g / (|g| + eps) changes fast in g there): a plain fp32 sum
+// of 10^2-10^4 terms can then move the update by more than 1e-5, while the
+// compensated sum stays within about one rounding of the exact sum.
 // Each is tuned for requests in flight (resident warps against rows in flight
 // per warp): the access pattern is random 512-byte rows, which HBM serves near
 // its copy bandwidth only with many requests in flight.  Results do not depend
@@ -107,9 +113,12 @@ __device__ __forceinline__ unsigned group_mask(int G, int gid) {
 // acc += the gradient rows of sorted positions s .. s+len-1, in that order.
 // The group loads up to G positions at a time (one per lane) and hands them
 // round with group shuffles.  With PRE the first G positions were loaded by
-// the caller (pl_first, one per lane).
-template <int V, int KV, int ROWS = MLKV_REDUCE_ROWS_IN_FLIGHT, bool PRE = false>
-__device__ __forceinline__ void sum_rows(typename Vec<V>::T (&acc)[KV], const float* __restrict__ grads,
+// the caller (pl_first, one per lane).  With COMP every addition is
+// compensated (comp_add): acc + cmp is then the sum to about twice fp32's
+// precision; without it cmp is not touched.
+template <int V, int KV, int ROWS = MLKV_REDUCE_ROWS_IN_FLIGHT, bool PRE = false, bool COMP = false>
+__device__ __forceinline__ void sum_rows(typename Vec<V>::T (&acc)[KV], typename Vec<V>::T (&cmp)[KV],
+                                         const float* __restrict__ grads,
                                          const uint32_t* __restrict__ spos, uint32_t s, uint32_t len, int d,
                                          int NV, int G, int glane, unsigned gmask, uint32_t pl_first = 0u) {
     using VT = typename Vec<V>::T;
@@ -134,7 +143,10 @@ __device__ __forceinline__ void sum_rows(typename Vec<V>::T (&acc)[KV], const fl
             for (int u = 0; u < UNR; ++u)
 #pragma unroll
                 for (int k = 0; k < KV; ++k)
-                    if (x + u < cnt && glane + G * k < NV) Vec<V>::add(acc[k], g[u][k]);
+                    if (x + u < cnt && glane + G * k < NV) {
+                        if (COMP) Vec<V>::cadd(acc[k], cmp[k], g[u][k]);
+                        else Vec<V>::add(acc[k], g[u][k]);
+                    }
         }
     }
 }
@@ -294,8 +306,8 @@ __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, u
         if (j < ra.NV) Vec<V>::add(acc[k], __ldcs(g0 + j));  // 0 + g: first term, in order
     }
     if (len > 1)
-        sum_rows<V, KV, MLKV_REDUCE_ROWS_IN_FLIGHT, true>(acc, a.grads, a.spos, s + 1, rest, ra.d, ra.NV, ra.G,
-                                                          glane, gmask, pl0);
+        sum_rows<V, KV, MLKV_REDUCE_ROWS_IN_FLIGHT, true>(acc, acc, a.grads, a.spos, s + 1, rest, ra.d, ra.NV,
+                                                          ra.G, glane, gmask, pl0);
     adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
 }
 
@@ -568,44 +580,60 @@ __global__ void __launch_bounds__(256, MLKV_LONG_MIN_BLOCKS) k_long_sum(RowArgs 
     const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
     for (uint32_t it = group; it < NI; it += ngroups) {
         const uint32_t s = __ldg(a.item_s + it), e = __ldg(a.item_e + it);
-        VT acc[KV];
+        VT acc[KV], cmp[KV];
 #pragma unroll
-        for (int k = 0; k < KV; ++k) acc[k] = Vec<V>::zero();
-        sum_rows<V, KV, MLKV_LONG_ROWS_IN_FLIGHT>(acc, a.grads, a.spos, s, e > s ? e - s : 0u, ra.d, ra.NV, G,
-                                                  glane, gmask);
-        VT* part = reinterpret_cast<VT*>(a.partial + (size_t)it * ra.dpad);
+        for (int k = 0; k < KV; ++k) {
+            acc[k] = Vec<V>::zero();
+            cmp[k] = Vec<V>::zero();
+        }
+        sum_rows<V, KV, MLKV_LONG_ROWS_IN_FLIGHT, false, true>(acc, cmp, a.grads, a.spos, s, e > s ? e - s : 0u,
+                                                               ra.d, ra.NV, G, glane, gmask);
+        // the chunk's (sum, compensation) pair
+        VT* part = reinterpret_cast<VT*>(a.partial + (size_t)it * 2 * ra.dpad);
 #pragma unroll
         for (int k = 0; k < KV; ++k) {
             const int j = glane + G * k;
-            if (j < ra.NV) __stcg(part + j, acc[k]);
+            if (j < ra.NV) {
+                __stcg(part + j, acc[k]);
+                __stcg(part + ra.dpad / V + j, cmp[k]);
+            }
         }
     }
 }
 
 
-// acc += chunk sums base + k0 .. base + k1 - 1, in that order, with eight
-// vectors per lane in flight.
+// (acc, cmp) += the chunk pairs base + k0 .. base + k1 - 1, in that order, with
+// eight vectors per lane in flight: each chunk's sum added with compensation,
+// then its own compensation added to cmp.
 template <int V, int KV>
-__device__ __forceinline__ void sum_partials(typename Vec<V>::T (&acc)[KV], const RowArgs& ra, const float* partial,
-                                             uint32_t base, uint32_t k0, uint32_t k1, int glane) {
+__device__ __forceinline__ void sum_partials(typename Vec<V>::T (&acc)[KV], typename Vec<V>::T (&cmp)[KV],
+                                             const RowArgs& ra, const float* partial, uint32_t base, uint32_t k0,
+                                             uint32_t k1, int glane) {
     using VT = typename Vec<V>::T;
-    constexpr int UNR = KV >= 8 ? 1 : 8 / KV;
+    constexpr int UNR = KV >= 4 ? 1 : 4 / KV;
+    const int half = ra.dpad / V;
     for (uint32_t x = k0; x < k1; x += UNR) {
-        VT g[UNR][KV];
+        VT g[UNR][KV], c[UNR][KV];
 #pragma unroll
         for (int u = 0; u < UNR; ++u) {
-            const VT* src = reinterpret_cast<const VT*>(partial + (size_t)(base + x + u) * ra.dpad);
+            const VT* src = reinterpret_cast<const VT*>(partial + (size_t)(base + x + u) * 2 * ra.dpad);
 #pragma unroll
             for (int k = 0; k < KV; ++k) {
                 const int j = glane + ra.G * k;
-                if (x + u < k1 && j < ra.NV) g[u][k] = __ldcg(src + j);
+                if (x + u < k1 && j < ra.NV) {
+                    g[u][k] = __ldcg(src + j);
+                    c[u][k] = __ldcg(src + half + j);
+                }
             }
         }
 #pragma unroll
         for (int u = 0; u < UNR; ++u)
 #pragma unroll
             for (int k = 0; k < KV; ++k)
-                if (x + u < k1 && glane + ra.G * k < ra.NV) Vec<V>::add(acc[k], g[u][k]);
+                if (x + u < k1 && glane + ra.G * k < ra.NV) {
+                    Vec<V>::cadd(acc[k], cmp[k], g[u][k]);
+                    Vec<V>::add(cmp[k], c[u][k]);
+                }
     }
 }
 
@@ -617,7 +645,7 @@ template <int V, int KV>
 __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, DevState* ds) {
     pdl_enter();
     using VT = typename Vec<V>::T;
-    extern __shared__ float sh[];  // [groups][dpad]
+    extern __shared__ float sh[];  // [groups][2][dpad]: each group's (sum, compensation) pair
     const uint32_t nl = min(a.cur->n_long, a.max_long), nb = a.cur->n_big;
     if (blockIdx.x == 0 && threadIdx.x == 0)
         ds->last_unique = a.cur->n_single + a.cur->n_short + a.cur->n_long;  // one run per row
@@ -630,28 +658,43 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
         const uint32_t m = (a.long_e[h] - a.long_s[h] + kChunk - 1) / kChunk;
         const uint32_t per = (m + ngroups - 1) / ngroups;
         const uint32_t k0 = min(m, group * per), k1 = min(m, k0 + per);
-        VT acc[KV];
+        VT acc[KV], cmp[KV];
 #pragma unroll
-        for (int k = 0; k < KV; ++k) acc[k] = Vec<V>::zero();
-        sum_partials<V, KV>(acc, ra, a.partial, base, k0, k1, glane);
-        VT* mine = reinterpret_cast<VT*>(sh + (size_t)group * ra.dpad);
+        for (int k = 0; k < KV; ++k) {
+            acc[k] = Vec<V>::zero();
+            cmp[k] = Vec<V>::zero();
+        }
+        sum_partials<V, KV>(acc, cmp, ra, a.partial, base, k0, k1, glane);
+        VT* mine = reinterpret_cast<VT*>(sh + (size_t)group * 2 * ra.dpad);
+        const int half = ra.dpad / V;
 #pragma unroll
         for (int k = 0; k < KV; ++k) {
             const int j = glane + G * k;
-            if (j < ra.NV) mine[j] = acc[k];
+            if (j < ra.NV) {
+                mine[j] = acc[k];
+                mine[half + j] = cmp[k];
+            }
         }
         __syncthreads();
         if (group == 0) {
 #pragma unroll
-            for (int k = 0; k < KV; ++k) acc[k] = Vec<V>::zero();
+            for (int k = 0; k < KV; ++k) {
+                acc[k] = Vec<V>::zero();
+                cmp[k] = Vec<V>::zero();
+            }
             for (int gi = 0; gi < ngroups; ++gi) {
-                const VT* src = reinterpret_cast<const VT*>(sh + (size_t)gi * ra.dpad);
+                const VT* src = reinterpret_cast<const VT*>(sh + (size_t)gi * 2 * ra.dpad);
 #pragma unroll
                 for (int k = 0; k < KV; ++k) {
                     const int j = glane + G * k;
-                    if (j < ra.NV) Vec<V>::add(acc[k], src[j]);
+                    if (j < ra.NV) {
+                        Vec<V>::cadd(acc[k], cmp[k], src[j]);
+                        Vec<V>::add(cmp[k], src[half + j]);
+                    }
                 }
             }
+#pragma unroll
+            for (int k = 0; k < KV; ++k) Vec<V>::add(acc[k], cmp[k]);  // the sum, rounded once
             VT w[KV], Gs[KV];
             const uint32_t row = a.long_row[h];
             load_row_state<V, KV>(ra, row, w, Gs, glane);
@@ -663,12 +706,17 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
     for (uint32_t h = gg; h < nl; h += ngg) {  // uniform within the group
         const uint32_t m = (a.long_e[h] - a.long_s[h] + kChunk - 1) / kChunk;
         if (m > kBigRun) continue;
-        VT acc[KV], w[KV], Gs[KV];
+        VT acc[KV], cmp[KV], w[KV], Gs[KV];
 #pragma unroll
-        for (int k = 0; k < KV; ++k) acc[k] = Vec<V>::zero();
+        for (int k = 0; k < KV; ++k) {
+            acc[k] = Vec<V>::zero();
+            cmp[k] = Vec<V>::zero();
+        }
         const uint32_t row = a.long_row[h];
         load_row_state<V, KV>(ra, row, w, Gs, glane);
-        sum_partials<V, KV>(acc, ra, a.partial, a.long_base[h], 0u, m, glane);
+        sum_partials<V, KV>(acc, cmp, ra, a.partial, a.long_base[h], 0u, m, glane);
+#pragma unroll
+        for (int k = 0; k < KV; ++k) Vec<V>::add(acc[k], cmp[k]);  // the sum, rounded once
         adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
     }
 }
@@ -697,9 +745,9 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, st, ra, a);
     const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);
     MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, st, ra, a);
-    int big = 1024;  // the groups' sums must fit the default 48 KB of shared memory
-    while (big > 64 && (size_t)(big / t->geom.G) * t->geom.dpad * sizeof(float) > 48 * 1024) big /= 2;
-    const size_t smem = (size_t)(big / t->geom.G) * t->geom.dpad * sizeof(float);
+    int big = 1024;  // the groups' (sum, compensation) pairs must fit the default 48 KB of shared memory
+    while (big > 64 && (size_t)(big / t->geom.G) * 2 * t->geom.dpad * sizeof(float) > 48 * 1024) big /= 2;
+    const size_t smem = (size_t)(big / t->geom.G) * 2 * t->geom.dpad * sizeof(float);
     // one block per SM (a 1024-thread block fills the register file): 4,864
     // lane groups of 32 for the ordinary long runs, 152 blocks for the big ones
     MLKV_LAUNCH_PERSISTENT(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), t->num_sms * (1024 / big), big, smem, st, ra, a,

@@ -99,7 +99,7 @@ struct Scratch {
     uint32_t* item_s;       // [max_items] first sorted position of each chunk
     uint32_t* item_e;       // [max_items] one past its last
     uint32_t* big_runs;     // [max_long] long runs with many chunks (combined by wide blocks)
-    float* partial;         // [max_items][dpad] chunk sums
+    float* partial;         // [max_items][2][dpad] chunk sums: compensated (sum, compensation) pairs
     int64_t max_long;
     int64_t max_items;
     int64_t tile_sums_len;
@@ -249,6 +249,19 @@ __device__ __forceinline__ void adagrad_element(float& w, float& G, float g, flo
     w = __fsub_rn(w, u);
 }
 
+// Compensated addition (TwoSum of Knuth and Moller): s <- fl(s + x) and the
+// rounding error of that sum, which is exact, added to the running
+// compensation c.  s + c then carries the sum to about twice fp32's precision.
+// Each operation is rounded on its own (the kernels are built without fused
+// multiply-adds or any other contraction).
+__device__ __forceinline__ void comp_add(float& s, float& c, float x) {
+    const float t = __fadd_rn(s, x);
+    const float bp = __fsub_rn(t, s);
+    const float e = __fadd_rn(__fsub_rn(s, __fsub_rn(t, bp)), __fsub_rn(x, bp));
+    s = t;
+    c = __fadd_rn(c, e);
+}
+
 template <int V> struct Vec;
 template <> struct Vec<4> {
     using T = float4;
@@ -260,6 +273,10 @@ template <> struct Vec<4> {
     static __device__ __forceinline__ void add(T& a, const T& b) {
         a.x = __fadd_rn(a.x, b.x); a.y = __fadd_rn(a.y, b.y);
         a.z = __fadd_rn(a.z, b.z); a.w = __fadd_rn(a.w, b.w);
+    }
+    static __device__ __forceinline__ void cadd(T& s, T& c, const T& x) {
+        comp_add(s.x, c.x, x.x); comp_add(s.y, c.y, x.y);
+        comp_add(s.z, c.z, x.z); comp_add(s.w, c.w, x.w);
     }
     static __device__ __forceinline__ void adagrad(T& w, T& G, const T& g, float lr, float eps) {
         adagrad_element(w.x, G.x, g.x, lr, eps); adagrad_element(w.y, G.y, g.y, lr, eps);
@@ -277,6 +294,7 @@ template <> struct Vec<1> {
     static __device__ __forceinline__ T zero() { return 0.f; }
     static __device__ __forceinline__ T nan() { return __int_as_float(0x7fc00000); }
     static __device__ __forceinline__ void add(T& a, const T& b) { a = __fadd_rn(a, b); }
+    static __device__ __forceinline__ void cadd(T& s, T& c, const T& x) { comp_add(s, c, x); }
     static __device__ __forceinline__ void adagrad(T& w, T& G, const T& g, float lr, float eps) {
         adagrad_element(w, G, g, lr, eps);
     }

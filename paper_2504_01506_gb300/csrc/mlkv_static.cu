@@ -1,8 +1,9 @@
 // Dedup of a batch of raw 64-bit keys that allocates no memory: its working
 // arrays live in one file-scope __device__ array of fixed size.  For callers
-// that may not allocate device memory when they need the dedup (code issuing
-// work while a stream is captured in global mode, where cudaMalloc is refused;
-// plugins of engines that own every device allocation); it needs no table.
+// that must not allocate device memory when they need the dedup: plugins
+// inside an engine that reserved the device's memory up front and owns every
+// allocation, and latency-bound loops that ban cudaMalloc / cudaFree because
+// those may synchronise the device.  It needs no table.
 //
 // Work: a stable LSD radix sort of the keys (8 passes of 8 bits: histogram
 // per 4096-key tile, one-block scan of the [digit][tile] counts, stable

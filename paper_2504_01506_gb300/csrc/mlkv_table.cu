@@ -3,6 +3,7 @@
 // across streams under a staleness bound (bulk-synchronous, stale-synchronous
 // or asynchronous, MLKV Section 3.3.1), status and timing.
 #include <algorithm>
+#include <atomic>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -40,6 +41,45 @@ int cuda_error(mlkv_table* t, cudaError_t e, const char* where) {
     } while (0)
 
 int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+// Host-side fault injection (mlkv_debug_fail): a countdown per kind; the call
+// that takes it from 1 to 0 fails without calling CUDA at all, so no GPU ever
+// sees a fault, and the error paths (MLKV_ERR_NOMEM, MLKV_ERR_CUDA, the
+// clean-up of a half-opened table) run as they would for a real failure.
+std::atomic<int64_t> g_fail_alloc{0};
+std::atomic<int64_t> g_fail_copy{0};
+
+bool injected(std::atomic<int64_t>& countdown) {
+    int64_t v = countdown.load();
+    while (v > 0)
+        if (countdown.compare_exchange_weak(v, v - 1)) return v == 1;
+    return false;
+}
+
+// Every device and pinned allocation and every host <-> device copy of the
+// library goes through these.
+template <class T>
+cudaError_t dev_alloc(T** p, size_t bytes) {
+    if (injected(g_fail_alloc)) {
+        *p = nullptr;
+        return cudaErrorMemoryAllocation;
+    }
+    return cudaMalloc((void**)p, bytes);
+}
+
+template <class T>
+cudaError_t pinned_alloc(T** p, size_t bytes, unsigned flags) {
+    if (injected(g_fail_alloc)) {
+        *p = nullptr;
+        return cudaErrorMemoryAllocation;
+    }
+    return cudaHostAlloc((void**)p, bytes, flags);
+}
+
+cudaError_t copy_async(void* dst, const void* src, size_t bytes, cudaMemcpyKind kind, cudaStream_t st) {
+    if (injected(g_fail_copy)) return cudaErrorInvalidValue;
+    return cudaMemcpyAsync(dst, src, bytes, kind, st);
+}
 
 // The host tier is pinned host memory from the driver's virtual-memory API
 // (cuMemCreate on the host NUMA node nearest the GPU), mapped for the device
@@ -128,7 +168,7 @@ int host_tier_alloc(mlkv_table* t, size_t bytes) {
     tr.host_dev = (float*)va;
     for (int64_t i = 0; i < n; ++i) {
         CUmemGenericAllocationHandle h;
-        if (v.create(&h, tr.host_chunk, &prop, 0) != CUDA_SUCCESS)
+        if (injected(g_fail_alloc) || v.create(&h, tr.host_chunk, &prop, 0) != CUDA_SUCCESS)
             return set_error(t, MLKV_ERR_NOMEM, "host tier: %lld of %lld chunks of %zu bytes", (long long)i,
                              (long long)n, tr.host_chunk);
         if (v.map(va + (size_t)i * tr.host_chunk, tr.host_chunk, 0, h, 0) != CUDA_SUCCESS) {
@@ -424,23 +464,23 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     const int64_t stride = t->geom.stride;
     t->tiered = c.hbm_cache_rows > 0;
     if (!t->tiered) {
-        if (cudaMalloc(&t->slots, (size_t)c.capacity * stride * sizeof(float)) != cudaSuccess)
+        if (dev_alloc(&t->slots, (size_t)c.capacity * stride * sizeof(float)) != cudaSuccess)
             return fail(MLKV_ERR_NOMEM);
     } else {
         Tier& tr = t->tier;
         const int64_t C = c.hbm_cache_rows;
         int rc = host_tier_alloc(t, (size_t)c.capacity * stride * sizeof(float));
         if (rc != MLKV_OK) return fail(rc);
-        if (cudaMalloc(&tr.cache, (size_t)C * stride * sizeof(float)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
-        if (cudaMalloc(&tr.row_loc, (size_t)c.capacity * 4) != cudaSuccess ||
-            cudaMalloc(&tr.line_row, (size_t)C * 4) != cudaSuccess ||
-            cudaMalloc(&tr.line_stamp, (size_t)C * 4) != cudaSuccess ||
-            cudaMalloc(&tr.ctr, 4 * sizeof(unsigned long long)) != cudaSuccess ||
-            cudaMalloc(&tr.fetch, (size_t)c.max_batch * sizeof(uint2)) != cudaSuccess ||
-            cudaMalloc(&tr.n_fetch, 4) != cudaSuccess ||
-            cudaMalloc(&tr.la_rows, (size_t)c.max_batch * 4) != cudaSuccess ||
-            cudaMalloc(&tr.la_fetch, (size_t)c.max_batch * sizeof(uint2)) != cudaSuccess ||
-            cudaMalloc(&tr.la_n_fetch, 4) != cudaSuccess)
+        if (dev_alloc(&tr.cache, (size_t)C * stride * sizeof(float)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
+        if (dev_alloc(&tr.row_loc, (size_t)c.capacity * 4) != cudaSuccess ||
+            dev_alloc(&tr.line_row, (size_t)C * 4) != cudaSuccess ||
+            dev_alloc(&tr.line_stamp, (size_t)C * 4) != cudaSuccess ||
+            dev_alloc(&tr.ctr, 4 * sizeof(unsigned long long)) != cudaSuccess ||
+            dev_alloc(&tr.fetch, (size_t)c.max_batch * sizeof(uint2)) != cudaSuccess ||
+            dev_alloc(&tr.n_fetch, 4) != cudaSuccess ||
+            dev_alloc(&tr.la_rows, (size_t)c.max_batch * 4) != cudaSuccess ||
+            dev_alloc(&tr.la_fetch, (size_t)c.max_batch * sizeof(uint2)) != cudaSuccess ||
+            dev_alloc(&tr.la_n_fetch, 4) != cudaSuccess)
             return fail(MLKV_ERR_NOMEM);
         if (launch_tier_init(t, 0) != cudaSuccess ||  // row r starts in host slot r
             cudaMemset(tr.line_row, 0xFF, (size_t)C * 4) != cudaSuccess ||
@@ -470,16 +510,16 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     }
     int64_t nslots = 64;
     while (nslots < 2 * c.capacity) nslots <<= 1;
-    if (cudaMalloc(&t->index, (size_t)nslots * sizeof(Slot)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
+    if (dev_alloc(&t->index, (size_t)nslots * sizeof(Slot)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
     if (cudaMemset(t->index, 0xFF, (size_t)nslots * sizeof(Slot)) != cudaSuccess) return fail(MLKV_ERR_CUDA);
     t->index_mask = (unsigned long long)(nslots - 1);
     t->bits_rows = bit_width_u64((uint64_t)c.capacity);
     t->bits_lines = t->tiered ? bit_width_u64((uint64_t)c.hbm_cache_rows) : t->bits_rows;
     t->sort_bits = t->bits_rows;
 
-    if (cudaMalloc(&t->dstate, sizeof(DevState)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
+    if (dev_alloc(&t->dstate, sizeof(DevState)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
     if (cudaMemset(t->dstate, 0, sizeof(DevState)) != cudaSuccess) return fail(MLKV_ERR_CUDA);
-    if (cudaHostAlloc(&t->status_host, sizeof(uint32_t), cudaHostAllocMapped) != cudaSuccess)
+    if (pinned_alloc(&t->status_host, sizeof(uint32_t), cudaHostAllocMapped) != cudaSuccess)
         return fail(MLKV_ERR_NOMEM);
     *t->status_host = 0;
     if (cudaHostGetDevicePointer((void**)&t->status_dev_alias, t->status_host, 0) != cudaSuccess)
@@ -515,11 +555,11 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
         {(void**)&s.short_runs, B * 16},
         {(void**)&s.single_runs, B * 8},
         {(void**)&s.run_p0, B * 4},
-        {(void**)&s.partial, s.max_items * t->geom.dpad * 4},
+        {(void**)&s.partial, s.max_items * 2 * t->geom.dpad * 4},
     };
     int64_t total = 0;
     for (auto& p : pieces) total += round_up(p.bytes, 256);
-    if (cudaMalloc(&t->arena, (size_t)total) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
+    if (dev_alloc(&t->arena, (size_t)total) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
     if (cudaMemset(t->arena, 0, (size_t)total) != cudaSuccess) return fail(MLKV_ERR_CUDA);
     t->arena_bytes = total;
     char* base = (char*)t->arena;
@@ -740,8 +780,8 @@ static int ensure_staging(mlkv_table* t, bool apply, int& set) {
     if (t->stage_keys[set]) return MLKV_OK;
     const size_t kb = (size_t)t->cfg.max_batch * sizeof(int64_t);
     const size_t vb = (size_t)t->cfg.max_batch * t->cfg.dim * sizeof(float);
-    if (cudaMalloc(&t->stage_keys[set], kb) != cudaSuccess) return set_error(t, MLKV_ERR_NOMEM, "staging keys");
-    if (cudaMalloc(&t->stage_vals[set], vb) != cudaSuccess) {
+    if (dev_alloc(&t->stage_keys[set], kb) != cudaSuccess) return set_error(t, MLKV_ERR_NOMEM, "staging keys");
+    if (dev_alloc(&t->stage_vals[set], vb) != cudaSuccess) {
         cudaFree(t->stage_keys[set]);
         t->stage_keys[set] = nullptr;
         return set_error(t, MLKV_ERR_NOMEM, "staging values");
@@ -755,9 +795,9 @@ int mlkv_get_host(mlkv_table* t, const int64_t* h_keys, int64_t n, float* h_out,
     int set;
     if ((rc = ensure_staging(t, false, set))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
-    CK(t, cudaMemcpyAsync(t->stage_keys[set], h_keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
+    CK(t, copy_async(t->stage_keys[set], h_keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
     if ((rc = mlkv_get(t, t->stage_keys[set], n, t->stage_vals[set], stream))) return rc;
-    CK(t, cudaMemcpyAsync(h_out, t->stage_vals[set], (size_t)n * t->cfg.dim * 4, cudaMemcpyDeviceToHost, st));
+    CK(t, copy_async(h_out, t->stage_vals[set], (size_t)n * t->cfg.dim * 4, cudaMemcpyDeviceToHost, st));
     return MLKV_OK;
 }
 
@@ -768,8 +808,8 @@ int mlkv_apply_grad_host(mlkv_table* t, const int64_t* h_keys, int64_t n, const 
     int set;
     if ((rc = ensure_staging(t, true, set))) return rc;
     cudaStream_t st = (cudaStream_t)stream;
-    CK(t, cudaMemcpyAsync(t->stage_keys[set], h_keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
-    CK(t, cudaMemcpyAsync(t->stage_vals[set], h_grads, (size_t)n * t->cfg.dim * 4, cudaMemcpyHostToDevice, st));
+    CK(t, copy_async(t->stage_keys[set], h_keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
+    CK(t, copy_async(t->stage_vals[set], h_grads, (size_t)n * t->cfg.dim * 4, cudaMemcpyHostToDevice, st));
     return mlkv_apply_grad(t, t->stage_keys[set], n, t->stage_vals[set], stream);
 }
 
@@ -856,5 +896,14 @@ int mlkv_kernel_time(mlkv_table* t, double* total_ms, int64_t* launches) {
 }
 
 const char* mlkv_last_error(mlkv_table* t) { return t ? t->last_error : "null table"; }
+
+int mlkv_debug_fail(int32_t kind, int64_t nth) {
+    if (nth < 0) return MLKV_ERR_INVALID;
+    switch (kind) {
+        case MLKV_FAULT_ALLOC: g_fail_alloc.store(nth); return MLKV_OK;
+        case MLKV_FAULT_COPY: g_fail_copy.store(nth); return MLKV_OK;
+        default: return MLKV_ERR_INVALID;
+    }
+}
 
 }  // extern "C"

@@ -1,6 +1,7 @@
-"""bench.py's multi-GPU arithmetic on CPU: N replicas (one process each, gloo)
+"""bench.py's multi-GPU path on CPU: N replicas (one process each, gloo)
 report the whole job's rate over the slowest rank's time, every rank agrees on
-it, and the reference arm runs on rank 0 alone."""
+it, `--gpus N` starts its own N ranks, and the reference arm prints from rank 0
+alone."""
 import json
 import os
 import socket
@@ -53,17 +54,29 @@ def test_two_replicas_report_the_job_rate_over_the_slowest_rank():
         assert value == pytest.approx(2_000 / 0.015)  # both ranks' units over the slowest time
 
 
-def _run_reference(rank, world):
-    env = dict(os.environ, RANK=str(rank), WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
-    return subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--config", "tiny", "--steps", "2",
-                           "--warmup", "3"], cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
-
-
-def test_reference_arm_runs_on_rank_zero_only():
-    r1 = _run_reference(1, 2)
-    assert r1.returncode == 0 and r1.stdout.strip() == ""
-    r0 = _run_reference(0, 2)
-    assert r0.returncode == 0
-    line = json.loads(r0.stdout.strip().splitlines()[-1])
+def test_gpus_flag_starts_its_own_ranks():
+    """`bench.py --gpus 2` with no launcher environment starts two ranks itself;
+    on the reference arm (no GPU work) both join one gloo group and rank 0 alone
+    prints the line, with n_gpus = the group's size."""
+    env = {k: v for k, v in os.environ.items()
+           if k not in ("RANK", "WORLD_SIZE", "LOCAL_RANK", "MASTER_ADDR", "MASTER_PORT")}
+    r = subprocess.run([sys.executable, "bench.py", "--gpus", "2", "--impl", "reference", "--config", "tiny",
+                        "--steps", "2", "--warmup", "3"], cwd=ROOT, env=env, capture_output=True, text=True,
+                       timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1, r.stdout  # rank 0 only
+    line = json.loads(lines[0])
     assert line["impl"] == "reference" and line["value"] > 0
+    assert line["n_gpus"] == 2 and line["config"]["parallelism"] == "replicas2"
     assert line["cpu_baseline"]["kind"] == "oracle" and line["e2e"]["h2d_bytes_per_step"] == 0
+    assert line["cpu_baseline"]["cpu_model"]
+
+
+def test_rank_count_must_match_the_flag(monkeypatch):
+    sys.path.insert(0, ROOT)
+    import bench
+
+    monkeypatch.setenv("WORLD_SIZE", "1")
+    with pytest.raises(SystemExit):
+        bench.dist_setup(2)

@@ -37,12 +37,19 @@ def test_tiny_config_full_parity():
     # key -> row resolution: dense ids in preload order, bit-exact
     assert np.array_equal(host(store.find(dev(pre))), np.arange(len(pre)))
     max_count = {}
+    tracker = CountTracker()
+    tracker.max_count = max_count
     for step in range(cfg.steps):
         keys = cfg.batch_keys(step)
         grads = cfg.grads(step)
         out = host(store.get(dev(keys)))
         want, _, _ = ref32.get(keys)
-        ref64.get(keys)
+        want64, _, _ = ref64.get(keys)
+        # every step's Get against the oracle: keys whose runs so far were all
+        # short bit for bit (fp32), the others within tolerance of fp64
+        exact = ~tracker.long_mask(keys)
+        assert_bits(out[exact], want[exact], f"Get of step {step} (short-run keys)")
+        assert_close(out[~exact], want64[~exact], f"Get of step {step} (long-run keys)")
         if step == 0:
             assert_bits(out, want, "Get of step 0")
         # Get is a bit-exact copy of the store's own rows
@@ -56,8 +63,6 @@ def test_tiny_config_full_parity():
             max_count[k] = max(max_count.get(k, 0), n)
     assert store.sync() == 0
     w, G = store.export(dev(pre))
-    tracker = CountTracker()
-    tracker.max_count = max_count
     n_short, n_long = assert_table_parity(host(w), host(G), pre, ref32, ref64, tracker)
     assert n_short > 0.99 * len(pre)
     assert store.size() == len(pre)

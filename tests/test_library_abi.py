@@ -134,3 +134,16 @@ def test_open_validates_its_config_without_gpu(lib):
         h = ctypes.c_void_p()
         assert bound.mlkv_open(ctypes.byref(cfg), ctypes.byref(h)) == code, over
         assert not h.value, over
+
+
+def test_fault_injection_arguments_without_gpu(lib):
+    """mlkv_debug_fail only sets a host-side countdown: it works with no GPU and
+    rejects an unknown kind or a negative count."""
+    from paper_2504_01506_gb300 import _lib
+
+    bound = _lib.load()
+    assert bound.mlkv_debug_fail(99, 1) == _lib.ERR_INVALID
+    assert bound.mlkv_debug_fail(_lib.FAULT_ALLOC, -1) == _lib.ERR_INVALID
+    assert bound.mlkv_debug_fail(_lib.FAULT_ALLOC, 3) == _lib.OK
+    assert bound.mlkv_debug_fail(_lib.FAULT_ALLOC, 0) == _lib.OK
+    assert bound.mlkv_debug_fail(_lib.FAULT_COPY, 0) == _lib.OK

@@ -85,6 +85,19 @@ class StoreConfig:
         return g
 
 
+    def grads_device(self, step: int, device, n: int | None = None):
+        """Per-lookup gradients N(0, sigma) as a float32 [n, dim] CUDA tensor, from
+        torch's device generator seeded by (config, step): for full-size batches,
+        whose host generation would take seconds a step.  Tests copy the rows they
+        need to the host, so both sides see the same array."""
+        import torch
+
+        n = self.batch if n is None else n
+        gen = torch.Generator(device=device)
+        gen.manual_seed(self.seed * 1000 + 977 + step)
+        return torch.randn((n, self.dim), generator=gen, device=device, dtype=torch.float32) * self.grad_sigma
+
+
 class TinyConfig(StoreConfig):
     def _keyset(self):
         if "keyset" not in self._cache:
