@@ -662,6 +662,18 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
         dom_ms, dom_n = store.kernel_time()
         store.time_kernel(0)
     assert store.sync() == 0, "device status set during the roofline region"
+    kernel_avg = None
+    if args.kernel_times:
+        # every kernel class event-timed over the same steps run call by call
+        kernel_avg = {}
+        for kid in kinds:
+            store.time_kernel(kid)
+            for i in range(steps):
+                step(base + args.warmup + i)
+            ms, n = store.kernel_time()
+            kernel_avg[KERNEL_NAMES[kid]] = {"ms_per_step": ms / steps, "launches_per_step": n / steps}
+        store.time_kernel(0)
+        assert store.sync() == 0
     step_bytes = np.mean([st["step"] for st in stats])
     achieved_step = step_bytes * steps / (elapsed_ms / 1e3) / 1e9
 
@@ -788,6 +800,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
         "distinct_per_step": float(np.mean([st["U"] for st in stats])),
         "distinct_rows_per_s": float(np.mean([st["U"] for st in stats])) * world * steps / (elapsed_ms / 1e3),
         "roofline": roofline, "kernel_ms_one_step": {KERNEL_NAMES[k]: v for k, v in kernel_ms.items()},
+        **({"kernel_ms_avg": kernel_avg} if kernel_avg else {}),
         "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clock_summary,
         "step_launch": (f"one CUDA graph replay per step (the Get and the {'Put' if kv else 'apply'} of the "
                         f"batch, captured)" if use_graphs else
@@ -877,6 +890,8 @@ def main():
                     help="tiered config: no look-ahead; each Get fetches its own missing rows")
     ap.add_argument("--scale", type=int, default=1,
                     help="divide the table's rows by this (same batch); for small profiling cases")
+    ap.add_argument("--kernel-times", action="store_true",
+                    help="also event-time every kernel class over the timed steps (run call by call)")
     ap.add_argument("--per-config", default="auto",
                     help="workloads measured after the headline one in the same process, comma-separated "
                          "(auto: kg,gnn,tiered after the default DLRM workload at N=1; none: no others)")

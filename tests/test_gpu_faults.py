@@ -71,8 +71,8 @@ def _store_and_oracle():
     from paper_2504_01506_gb300 import EmbeddingStore
 
     cfg = W.scaled(W.tiny(), 50, 4)
-    store = EmbeddingStore(dim=cfg.dim, capacity=cfg.n_keys, max_batch=cfg.batch, lr=cfg.lr, eps=cfg.eps,
-                           state_init=cfg.state_init, init_lo=cfg.init_lo, init_hi=cfg.init_hi, seed=cfg.seed,
+    store = EmbeddingStore(dim=cfg.dim, capacity=cfg.n_keys, max_batch=max(cfg.batch, cfg.n_keys), lr=cfg.lr,
+                           eps=cfg.eps, state_init=cfg.state_init, init_lo=cfg.init_lo, init_hi=cfg.init_hi, seed=cfg.seed,
                            device="cuda:0")
     ref = oracle.Table(cfg.dim, lr=cfg.lr, eps=cfg.eps, state_init=cfg.state_init, init_lo=cfg.init_lo,
                        init_hi=cfg.init_hi, seed=cfg.seed, precision=32)
