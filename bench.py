@@ -52,6 +52,7 @@ METRIC_YCSB = "key-value operations/s (YCSB-shaped batches of Gets and Puts)"
 UNIT_YCSB = "ops/s"
 NOMINAL_HBM_GBS = 8000.0
 SEQ_SEGMENT_MAX = 32
+SMALL_RUN = 4  # runs of 2 .. SMALL_RUN lookups go to k_small (their positions in their record)
 CHUNK = 64
 
 
@@ -211,16 +212,22 @@ def batch_stats(keys: np.ndarray, d: int) -> dict:
     Bl, Ul = int(counts[long_].sum()), int(long_.sum())
     Bs, Us = B - Bl, U - Ul
     U1 = int((counts == 1).sum())  # runs of one lookup (k_single)
-    Bm, Um = Bs - U1, Us - U1      # the other short runs (k_short)
+    small = (counts >= 2) & (counts <= SMALL_RUN)
+    Usm, Bsm = int(small.sum()), int(counts[small].sum())  # runs of 2 .. SMALL_RUN lookups (k_small)
+    Bm, Um = Bs - U1 - Bsm, Us - U1 - Usm                  # the other short runs (k_short)
     items = int(np.ceil(counts[long_] / CHUNK).sum())
     row = 4 * d
     return {
         "B": B, "U": U, "Bs": Bs, "Us": Us, "Bl": Bl, "Ul": Ul, "items": items, "U1": U1, "Um": Um,
+        "Usm": Usm, "Bsm": Bsm,
         # Get: keys + output per lookup; index sector + row per distinct key
         "get_gather": B * (8 + row) + U * (32 + row),
-        # short runs of 2+ lookups: gradient rows + sorted position per lookup;
-        # row and state read and written once plus the run's 16-byte record
+        # runs of SMALL_RUN + 1 .. 32 lookups: gradient rows + sorted position per
+        # lookup; row and state read and written once plus the run's 16-byte record
         "reduce_short": Bm * (row + 4) + Um * (4 * row + 16),
+        # runs of 2 .. SMALL_RUN lookups: gradient rows; row and state read and
+        # written once, the 20-byte record with the run's positions
+        "reduce_small": Bsm * row + Usm * (4 * row + 20),
         # runs of one lookup: the gradient row, row and state read and written
         # once, the 8-byte record
         "reduce_single": U1 * (row + 4 * row + 8),
@@ -257,6 +264,8 @@ def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
         return stats["reduce_short"]
     if kid == 10:
         return stats["reduce_single"]
+    if kid == 11:
+        return stats["reduce_small"]
     if kid == 5:
         return stats["reduce_long"]
     if kid == 7:
@@ -265,8 +274,8 @@ def kernel_bytes(stats: dict, kid: int, sort_passes: int) -> float:
         return stats["B"] * 16.0  # per pass: (row id, position) read and written
     if kid == 2:
         return stats["B"] * 12.0 + stats["U"] * 32.0
-    if kid == 6:  # each sorted row id read twice, run records written (with the run's first position)
-        return stats["B"] * 8.0 + stats["Um"] * 20.0 + stats["U1"] * 12.0
+    if kid == 6:  # each sorted row id read twice and each position once; the run records written
+        return stats["B"] * 12.0 + stats["U1"] * 8.0 + stats["Usm"] * 20.0 + stats["Um"] * 16.0
     return 0.0
 
 
@@ -274,10 +283,10 @@ KERNEL_NAMES = {1: "k_get (probe + row gather)", 2: "k_probe", 3: "k_sort_scatte
                 4: "k_short (run sum + Adagrad)", 5: "k_long_sum (chunk sums of long runs)",
                 6: "k_heads (runs found in the sorted ids)", 7: "k_long_combine (chunk sums + Adagrad)",
                 8: "k_tier_fetch (host <-> HBM row swap)", 9: "k_put_scatter (Put: last occurrence writes)",
-                10: "k_single (runs of one lookup + Adagrad)"}
+                10: "k_single (runs of one lookup + Adagrad)", 11: "k_small (runs of 2-4 lookups + Adagrad)"}
 KERNEL_SOURCES = {1: "mlkv_index.cu", 2: "mlkv_index.cu", 3: "mlkv_sort.cu", 4: "mlkv_apply.cu",
                   5: "mlkv_apply.cu", 6: "mlkv_apply.cu", 7: "mlkv_apply.cu", 8: "mlkv_tier.cu",
-                  9: "mlkv_index.cu", 10: "mlkv_apply.cu"}
+                  9: "mlkv_index.cu", 10: "mlkv_apply.cu", 11: "mlkv_apply.cu"}
 
 
 def traffic_for(kid: int, cfg, path=None):
@@ -520,7 +529,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
     # The HBM store cycles a pool of batches.  The tiered store gets a fresh batch
     # every step (a cycled pool would end up resident in its cache): one per
     # kernel-class prepass step, warm-up step, timed step, and the last look-ahead.
-    kinds = (1, 2, 9) if kv else (1, 2, 3, 4, 5, 6, 7, 10) + ((8,) if tiered else ())
+    kinds = (1, 2, 9) if kv else (1, 2, 3, 4, 5, 6, 7, 10, 11) + ((8,) if tiered else ())
     base = len(kinds) if tiered else 0
     pool = base + args.warmup + steps + 1 if tiered else max(1, min(args.pool, steps + args.warmup))
     ngrad = max(1, min(args.pool, pool))

@@ -305,6 +305,7 @@ int mlkv_tier_stats(mlkv_table* t, int64_t* rows_fetched, int64_t* rows_written_
 #define MLKV_K_TIER_FETCH 8
 #define MLKV_K_PUT_SCATTER 9
 #define MLKV_K_REDUCE_SINGLE 10
+#define MLKV_K_REDUCE_SMALL 11
 int mlkv_time_kernel(mlkv_table* t, int32_t kernel_id);
 int mlkv_kernel_time(mlkv_table* t, double* total_ms, int64_t* launches);
 

@@ -35,6 +35,7 @@ K_LONG_COMBINE = 7
 K_TIER_FETCH = 8
 K_PUT_SCATTER = 9
 K_REDUCE_SINGLE = 10
+K_REDUCE_SMALL = 11
 
 EXPORTED = [
     "mlkv_open", "mlkv_close", "mlkv_get", "mlkv_put", "mlkv_insert", "mlkv_apply_grad",

@@ -10,17 +10,23 @@
 //
 //  k_heads        a warp per window of 32 sorted positions finds the runs
 //                 that start there (a row id unlike its left neighbour) and
-//                 their lengths; runs of one lookup and the other runs of
-//                 <= MLKV_SEQ_SEGMENT_MAX lookups go to two lists (one atomic
+//                 their lengths; runs of one lookup, of 2 .. kSmallRun lookups
+//                 (with their positions) and the other runs of <=
+//                 MLKV_SEQ_SEGMENT_MAX lookups go to three lists (one atomic
 //                 per block and list; any order: every run is summed on its
 //                 own), longer ones are measured (a warp-wide search for their
 //                 end) and listed for k_long_*.
 //  k_single       one lane group per run of one lookup: row, state and the
 //                 gradient row loaded together, then the Adagrad step.
-//  k_short        one lane group per run of 2 .. MLKV_SEQ_SEGMENT_MAX
-//                 lookups: the row, the state, the first gradient row and the
-//                 run's other positions are loaded together, the rest summed in
-//                 occurrence order, then the Adagrad step.
+//  k_small        one lane group per run of 2 .. kSmallRun lookups, whose
+//                 positions k_heads wrote into the run's record: row, state and
+//                 every gradient row in one round trip, the occurrence-order
+//                 sum, then the Adagrad step.
+//  k_short        one lane group per run of kSmallRun + 1 ..
+//                 MLKV_SEQ_SEGMENT_MAX lookups: the row, the state, the first
+//                 gradient row and the run's other positions are loaded
+//                 together, the rest summed in occurrence order, then the
+//                 Adagrad step.
 //  k_long_sum     one lane group per chunk of kChunk lookups of a long run
 //                 (Zipf-hot keys reach 10^4-10^5 lookups): the chunk's sum,
 //                 compensated, to scratch as a (sum, compensation) pair.
@@ -66,6 +72,11 @@ constexpr uint32_t kBigRun = 32;
 #ifndef MLKV_SINGLE_MIN_BLOCKS
 #define MLKV_SINGLE_MIN_BLOCKS 6
 #endif
+// k_small: blocks per SM the register allocation must allow.
+#ifndef MLKV_SMALL_MIN_BLOCKS
+#define MLKV_SMALL_MIN_BLOCKS 4
+#endif
+constexpr uint32_t NONE = 0xFFFFFFFFu;  // no position (a small run's record past its end)
 #ifndef MLKV_LONG_ROWS_IN_FLIGHT
 #define MLKV_LONG_ROWS_IN_FLIGHT 8
 #endif
@@ -92,6 +103,9 @@ struct RunArgs {
     uint4* runs;           // [max_batch] short runs of 2 or more lookups: (first sorted position, one
                            //   past the last, row, first lookup position)
     uint2* singles;        // [max_batch] runs of one lookup: (row, lookup position)
+    uint4* smalls;         // [max_batch] runs of 2 .. kSmallRun lookups: (row, p0, p1, p2), positions in
+                           //   occurrence order, NONE past the run's end
+    uint32_t* small_p3;    // [max_batch] their fourth position (or NONE)
     uint32_t* long_s;      // [max_long] first sorted position
     uint32_t* long_e;      // [max_long] one past the last
     uint32_t* long_row;    // [max_long]
@@ -322,34 +336,47 @@ __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, u
 // two run lists, the long-run list and the chunk list with one atomic each and
 // the warps copy their runs out.  (Counters that every warp bumps queue up at
 // the end of the kernel.)
-__global__ void __launch_bounds__(256, 5) k_heads(RunArgs a) {
+#ifndef MLKV_HEADS_MIN_BLOCKS
+#define MLKV_HEADS_MIN_BLOCKS 4
+#endif
+__global__ void __launch_bounds__(256, MLKV_HEADS_MIN_BLOCKS) k_heads(RunArgs a) {
     pdl_enter();
-    constexpr int kList = 128, kQueue = 16;
-    __shared__ uint4 lst[8][kList];  // (start, end, row, first lookup) of short runs
-    __shared__ uint2 sgl[8][kList];  // (row, lookup) of runs of one lookup
+    constexpr int kList = 128, kListS = 64, kQueue = 16;
+    __shared__ uint4 lst[8][kListS];  // (start, end, row, first lookup) of short runs
+    __shared__ uint2 sgl[8][kList];   // (row, lookup) of runs of one lookup
+    __shared__ uint4 sml[8][kListS];  // (row, p0, p1, p2) of small runs
+    __shared__ uint32_t sp3[8][kListS];  // ... and their p3
     __shared__ uint32_t qs[8][kQueue], qr[8][kQueue], qe[8][kQueue];  // long runs: start, row, end (0: unknown)
-    __shared__ uint32_t wsh[8], wlg[8], wit[8], ws1[8];  // per warp: short runs, long runs, chunks,
-                                                         // runs of one lookup; then their bases
+    __shared__ uint32_t wsh[8], wlg[8], wit[8], ws1[8], ws2[8];  // per warp: short runs, long runs, chunks,
+                                                                 // runs of one lookup, small runs; then
+                                                                 // their bases
     const uint32_t n = a.n, sent = a.sent;
     const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
     const uint32_t lt = lanemask_lt();
     const uint32_t warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t nwarps = (gridDim.x * blockDim.x) >> 5;
     const uint32_t nwin = (n + 31) >> 5;
-    int cnt = 0, cnt1 = 0, nq = 0;  // warp-uniform
+    int cnt = 0, cnt1 = 0, cnt2 = 0, nq = 0;  // warp-uniform
     // full lists or a full queue go out at once (only batches far above a few
     // runs per window and warp get here)
     auto flush = [&]() {
         __syncwarp();
-        uint32_t base = 0, base1 = 0;
+        uint32_t base = 0, base1 = 0, base2 = 0;
         if (lane == 0 && cnt) base = atomicAdd(&a.cur->n_short, (uint32_t)cnt);
         if (lane == 0 && cnt1) base1 = atomicAdd(&a.cur->n_single, (uint32_t)cnt1);
+        if (lane == 0 && cnt2) base2 = atomicAdd(&a.cur->n_small, (uint32_t)cnt2);
         base = __shfl_sync(0xffffffffu, base, 0);
         base1 = __shfl_sync(0xffffffffu, base1, 0);
+        base2 = __shfl_sync(0xffffffffu, base2, 0);
         for (int k = lane; k < cnt; k += 32) a.runs[base + k] = lst[wib][k];
         for (int k = lane; k < cnt1; k += 32) a.singles[base1 + k] = sgl[wib][k];
+        for (int k = lane; k < cnt2; k += 32) {
+            a.smalls[base2 + k] = sml[wib][k];
+            a.small_p3[base2 + k] = sp3[wib][k];
+        }
         cnt = 0;
         cnt1 = 0;
+        cnt2 = 0;
         __syncwarp();
     };
     auto measure = [&]() {  // fills in the unknown ends of the queued long runs
@@ -402,13 +429,29 @@ __global__ void __launch_bounds__(256, 5) k_heads(RunArgs a) {
             lng = lng || len > MLKV_SEQ_SEGMENT_MAX;
         }
         const bool shrt = head && !lng;  // len >= 1
-        const unsigned sm = __ballot_sync(0xffffffffu, shrt && len > 1);
+        const bool smll = shrt && len > 1 && len <= kSmallRun;
+        const unsigned sm = __ballot_sync(0xffffffffu, shrt && len > kSmallRun);
         const unsigned s1 = __ballot_sync(0xffffffffu, shrt && len == 1);
-        if (cnt + __popc(sm) > kList || cnt1 + __popc(s1) > kList) flush();
-        if (shrt && len > 1) lst[wib][cnt + __popc(sm & lt)] = make_uint4(p, p + len, r, pos);
+        const unsigned s2 = __ballot_sync(0xffffffffu, smll);
+        // a small run's other positions: from the lanes after its head, or, where
+        // the run goes on into the next window, from the sorted positions
+        const uint32_t q1 = __shfl_down_sync(0xffffffffu, pos, 1);
+        const uint32_t q2 = __shfl_down_sync(0xffffffffu, pos, 2);
+        const uint32_t q3 = __shfl_down_sync(0xffffffffu, pos, 3);
+        if (cnt + __popc(sm) > kListS || cnt1 + __popc(s1) > kList || cnt2 + __popc(s2) > kListS) flush();
+        if (shrt && len > kSmallRun) lst[wib][cnt + __popc(sm & lt)] = make_uint4(p, p + len, r, pos);
         if (shrt && len == 1) sgl[wib][cnt1 + __popc(s1 & lt)] = make_uint2(r, pos);
+        if (smll) {
+            const uint32_t p1 = lane + 1 < 32 ? q1 : __ldg(a.spos + p + 1);
+            const uint32_t p2 = len < 3 ? NONE : lane + 2 < 32 ? q2 : __ldg(a.spos + p + 2);
+            const uint32_t p3 = len < 4 ? NONE : lane + 3 < 32 ? q3 : __ldg(a.spos + p + 3);
+            const int k = cnt2 + __popc(s2 & lt);
+            sml[wib][k] = make_uint4(r, pos, p1, p2);
+            sp3[wib][k] = p3;
+        }
         cnt += __popc(sm);
         cnt1 += __popc(s1);
+        cnt2 += __popc(s2);
         for (unsigned lm = __ballot_sync(0xffffffffu, head && lng); lm; lm &= lm - 1) {
             const int i = __ffs(lm) - 1;
             if (nq == kQueue) {
@@ -446,35 +489,44 @@ __global__ void __launch_bounds__(256, 5) k_heads(RunArgs a) {
         wlg[wib] = (uint32_t)nq;
         wit[wib] = items;
         ws1[wib] = (uint32_t)cnt1;
+        ws2[wib] = (uint32_t)cnt2;
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-        uint32_t ts = 0, tl = 0, ti = 0, t1 = 0;
+        uint32_t ts = 0, tl = 0, ti = 0, t1 = 0, t2 = 0;
         for (int k = 0; k < 8; ++k) {
             ts += wsh[k];
             tl += wlg[k];
             ti += wit[k];
             t1 += ws1[k];
+            t2 += ws2[k];
         }
         uint32_t bs = ts ? atomicAdd(&a.cur->n_short, ts) : 0u;
         uint32_t bl = tl ? atomicAdd(&a.cur->n_long, tl) : 0u;
         uint32_t bi = ti ? atomicAdd(&a.cur->n_items, ti) : 0u;
         uint32_t b1 = t1 ? atomicAdd(&a.cur->n_single, t1) : 0u;
+        uint32_t b2 = t2 ? atomicAdd(&a.cur->n_small, t2) : 0u;
         for (int k = 0; k < 8; ++k) {
-            const uint32_t c0 = wsh[k], c1 = wlg[k], c2 = wit[k], c3 = ws1[k];
+            const uint32_t c0 = wsh[k], c1 = wlg[k], c2 = wit[k], c3 = ws1[k], c4 = ws2[k];
             wsh[k] = bs;
             wlg[k] = bl;
             wit[k] = bi;
             ws1[k] = b1;
+            ws2[k] = b2;
             bs += c0;
             bl += c1;
             bi += c2;
             b1 += c3;
+            b2 += c4;
         }
     }
     __syncthreads();
     for (int k = lane; k < cnt; k += 32) a.runs[wsh[wib] + k] = lst[wib][k];
     for (int k = lane; k < cnt1; k += 32) a.singles[ws1[wib] + k] = sgl[wib][k];
+    for (int k = lane; k < cnt2; k += 32) {
+        a.smalls[ws2[wib] + k] = sml[wib][k];
+        a.small_p3[ws2[wib] + k] = sp3[wib][k];
+    }
     if (wlg[wib] + nq > a.max_long || wit[wib] + items > a.max_items) {
         if (lane == 0 && nq) record_error(a.err, MLKV_ERR_FULL);
         return;
@@ -569,6 +621,54 @@ __global__ void __launch_bounds__(256, MLKV_SINGLE_MIN_BLOCKS) k_single(RowArgs 
     }
 }
 
+// One lane group per run of 2 .. kSmallRun lookups (most runs of more than one
+// lookup in a Zipf batch).  k_heads put the run's positions in its record, so
+// the row, the state and every gradient row of the run load together, in one
+// round trip (records loaded one run ahead); then the sum 0 + g0 + g1 + ... in
+// occurrence order and the Adagrad step.  No loop over positions: few
+// registers and many warps, as in k_single.
+template <int V, int KV>
+__global__ void __launch_bounds__(256, KV >= 4 ? 2 : MLKV_SMALL_MIN_BLOCKS) k_small(RowArgs ra, RunArgs a) {
+    pdl_enter();
+    using VT = typename Vec<V>::T;
+    const uint32_t U = a.cur->n_small;
+    const int lane = threadIdx.x & 31, G = ra.G, glane = lane & (G - 1);
+    const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
+    const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
+    uint4 next = group < U ? __ldg(a.smalls + group) : make_uint4(0u, 0u, 0u, 0u);
+    uint32_t next3 = group < U ? __ldg(a.small_p3 + group) : NONE;
+    for (uint32_t u = group; u < U; u += ngroups) {  // uniform within the group
+        const uint4 m = next;  // (row, p0, p1, p2)
+        const uint32_t p3 = next3;
+        const uint32_t v = u + ngroups;
+        next = v < U ? __ldg(a.smalls + v) : make_uint4(0u, 0u, 0u, 0u);
+        next3 = v < U ? __ldg(a.small_p3 + v) : NONE;
+        VT w[KV], Gs[KV], g[kSmallRun][KV];
+        load_row_state<V, KV>(ra, m.x, w, Gs, glane);
+        const uint32_t ps[kSmallRun] = {m.y, m.z, m.w, p3};
+#pragma unroll
+        for (int i = 0; i < kSmallRun; ++i) {
+            if (ps[i] == NONE) continue;  // uniform within the group
+            const VT* src = reinterpret_cast<const VT*>(a.grads + (size_t)ps[i] * ra.d);
+#pragma unroll
+            for (int k = 0; k < KV; ++k) {
+                const int j = glane + G * k;
+                if (j < ra.NV) g[i][k] = __ldcs(src + j);
+            }
+        }
+        VT acc[KV];
+#pragma unroll
+        for (int k = 0; k < KV; ++k) {
+            acc[k] = Vec<V>::zero();
+            if (glane + G * k >= ra.NV) continue;
+#pragma unroll
+            for (int i = 0; i < kSmallRun; ++i)
+                if (ps[i] != NONE) Vec<V>::add(acc[k], g[i][k]);  // 0 + g0 + g1 + ...: occurrence order
+        }
+        adagrad_store<V, KV>(ra, m.x, w, Gs, acc, glane, a.lr, a.eps);
+    }
+}
+
 template <int V, int KV>
 __global__ void __launch_bounds__(256, MLKV_LONG_MIN_BLOCKS) k_long_sum(RowArgs ra, RunArgs a) {
     pdl_enter();
@@ -648,7 +748,7 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
     extern __shared__ float sh[];  // [groups][2][dpad]: each group's (sum, compensation) pair
     const uint32_t nl = min(a.cur->n_long, a.max_long), nb = a.cur->n_big;
     if (blockIdx.x == 0 && threadIdx.x == 0)
-        ds->last_unique = a.cur->n_single + a.cur->n_short + a.cur->n_long;  // one run per row
+        ds->last_unique = a.cur->n_single + a.cur->n_small + a.cur->n_short + a.cur->n_long;  // one run per row
     const int G = ra.G, glane = threadIdx.x & (G - 1);
     const int group = threadIdx.x / G;
     const int ngroups = blockDim.x / G;
@@ -725,7 +825,8 @@ template <int V, int KV>
 cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, const uint32_t* spos,
                        int64_t n, uint32_t sent, cudaStream_t st, CallCounters* cur) {
     RowArgs ra{t->slots, t->geom.stride, t->geom.dpad, t->geom.NV, t->geom.G, t->geom.d};
-    RunArgs a{grads, srow, spos, (uint32_t)n, sent, cur, t->s.short_runs, t->s.single_runs, t->s.long_s, t->s.long_e,
+    RunArgs a{grads, srow, spos, (uint32_t)n, sent, cur, t->s.short_runs, t->s.single_runs, t->s.small_runs,
+              t->s.small_p3, t->s.long_s, t->s.long_e,
               t->s.long_row, t->s.long_base, t->s.item_s, t->s.item_e, t->s.big_runs, t->s.partial,
               (uint32_t)t->s.max_long,
               (uint32_t)t->s.max_items, ErrSink{&t->dstate->status, t->status_dev_alias}, t->cfg.lr, t->cfg.eps};
@@ -741,6 +842,8 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     MLKV_LAUNCH(t, MLKV_K_SEGMENTS, k_heads, (unsigned)gh, 256, 0, st, a);
     const int g1 = persistent_blocks(t, (const void*)k_single<V, KV>, 256);
     MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, st, ra, a);
+    const int g2 = persistent_blocks(t, (const void*)k_small<V, KV>, 256);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, st, ra, a);
     const int gs = persistent_blocks(t, (const void*)k_short<V, KV>, 256);
     MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, st, ra, a);
     const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);

@@ -30,6 +30,7 @@ constexpr int kSortMaxPasses = 4;      // row ids have at most 31 bits
 constexpr int kSortMaxDigitBits = 9;   // radix <= 512
 constexpr int kSortMaxRadix = 1 << kSortMaxDigitBits;
 constexpr int kSortTile = 4096;        // lookups per tile of a sort pass
+constexpr int kSmallRun = 4;           // runs of 2 .. kSmallRun lookups carry their positions in their record
 constexpr int64_t kMaxStaleness = MLKV_MAX_STALENESS;  // largest bound kept below no bound
 
 // Per-call counters.  Two copies: a call uses cc[p] and its first kernel
@@ -45,6 +46,7 @@ struct CallCounters {
     uint32_t n_big;      // long runs whose chunk sums are combined by the wide blocks
     uint32_t n_single;   // runs of one lookup
     uint32_t short_next; // next chunk of short runs to claim (k_short's dynamic hand-out)
+    uint32_t n_small;    // runs of 2 .. kSmallRun lookups (their positions in the record)
 };
 
 struct DevState {
@@ -92,6 +94,8 @@ struct Scratch {
     uint32_t* run_p0;       // [max_batch] first lookup position of each run (dedup)
     uint4* short_runs;      // [max_batch] the apply's runs of 2 .. MLKV_SEQ_SEGMENT_MAX lookups
     uint2* single_runs;     // [max_batch] its runs of one lookup: (row, lookup position)
+    uint4* small_runs;      // [max_batch] runs of 2 .. kSmallRun lookups: (row, p0, p1, p2)
+    uint32_t* small_p3;     // [max_batch] their fourth position (or none)
     uint32_t* long_s;       // [max_long] long runs: first sorted position
     uint32_t* long_e;       // [max_long] one past the last
     uint32_t* long_row;     // [max_long]

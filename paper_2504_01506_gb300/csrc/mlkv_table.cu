@@ -554,6 +554,8 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
         {(void**)&s.big_runs, s.max_long * 4},
         {(void**)&s.short_runs, B * 16},
         {(void**)&s.single_runs, B * 8},
+        {(void**)&s.small_runs, B * 16},
+        {(void**)&s.small_p3, B * 4},
         {(void**)&s.run_p0, B * 4},
         {(void**)&s.partial, s.max_items * 2 * t->geom.dpad * 4},
     };

@@ -50,12 +50,15 @@ def test_single_lookup():
     assert_bits(host(store.export(dev(k))[0]), ref.export(k)[0], "single apply")
 
 
-@pytest.mark.parametrize("shape", ["all_distinct", "one_key", "every_length", "no_singletons"])
+@pytest.mark.parametrize("shape", ["all_distinct", "one_key", "every_length", "no_singletons", "small_runs"])
 def test_run_length_mixes(shape):
     """Batches made only of runs of one lookup, of one long run, of runs of
-    every length 1..40 (singletons, short runs, the 32/33 boundary, long
-    runs) and of no singletons at all: rows and state against the oracle, and
-    the apply's count of distinct rows (last_unique) against the batch's."""
+    every length 1..40 (singletons, small and short runs, the 4/5 and 32/33
+    boundaries, long runs), of no singletons at all, and of runs of 2-4 lookups
+    at every offset of the 32-position windows (those that start in the last
+    lanes of a window take their later positions from the next): rows and
+    state against the oracle, and the apply's count of distinct rows
+    (last_unique) against the batch's."""
     cfg = _small(dim=16)
     store, ref = make_pair(cfg, capacity=8192, max_batch=4096)
     rng = np.random.default_rng(11)
@@ -65,6 +68,9 @@ def test_run_length_mixes(shape):
         keys = np.full(4096, 99, np.int64)
     elif shape == "every_length":
         keys = np.concatenate([np.full(m, 1000 + m, np.int64) for m in range(1, 41)])
+    elif shape == "small_runs":
+        lens = rng.integers(2, 5, 1300)
+        keys = np.repeat(np.arange(len(lens), dtype=np.int64) * 3 + 7, lens)
     else:
         keys = np.repeat(np.arange(2000, dtype=np.int64) * 5 + 1, 2)
     keys = keys[rng.permutation(len(keys))]  # occurrences scattered over the batch
