@@ -180,6 +180,14 @@ class ClockSampler:
         return out
 
 
+def sync_ok(store, what: str):
+    """Waits for the store; a device status set by its kernels raises with the
+    library's text of it."""
+    rc = store.sync()
+    if rc:
+        raise RuntimeError(f"{what}: status {rc}: {store.lib.mlkv_last_error(store.h).decode()}")
+
+
 def cpu_description() -> dict:
     """Model and count of the host's cores (lscpu, else /proc/cpuinfo)."""
     model = None
@@ -511,7 +519,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
     chunk = cfg.batch
     for s0 in range(0, cfg.n_keys, chunk):
         store.insert(torch.from_numpy(cfg.preload_keys(s0, s0 + chunk)).to(dev))
-    assert store.sync() == 0, "preload failed"
+    sync_ok(store, "preload failed")
 
     if tiered and args.tier_prefill:
         # fill the HBM cache with rows of random keys, each updated once (so the
@@ -523,7 +531,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
             k = torch.from_numpy(fill[s0:s0 + cfg.batch]).to(dev)  # tiered keys are 0..n_keys-1
             store.get(k)
             store.apply_grad(k, zeros[:k.numel()])
-        assert store.sync() == 0, "prefill failed"
+        sync_ok(store, "prefill failed")
         del zeros
 
     # The HBM store cycles a pool of batches.  The tiered store gets a fresh batch
@@ -582,7 +590,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
     dominant = max(kernel_ms, key=kernel_ms.get)
     for i in range(args.warmup):
         step(base + i)
-    assert store.sync() == 0
+    sync_ok(store, "device status")
 
     # An HBM-resident step is captured into a CUDA graph per batch (the Get and
     # the apply of that batch) and replayed: the calls' work is device-driven,
@@ -603,7 +611,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
         launches_per_graph = (store.launch_count() - l0) // pool
         for i in range(args.warmup):
             graphs[(base + i) % pool].replay()
-        assert store.sync() == 0
+        sync_ok(store, "device status")
 
     def timed_step(i):
         if use_graphs:
@@ -654,7 +662,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
     window = (f"the timed region ({steps} steps) and {n_extra} more of the same steps right after it "
               f"({time.perf_counter() - t_timed0:.2f} s)" if n_extra else f"the timed region ({steps} steps)")
     clock_summary = clocks.summary(timed=(t_timed0, t_timed1), window=window)
-    assert store.sync() == 0, "device status set during the timed region"
+    sync_ok(store, "device status set during the timed region")
     elapsed_ms, value = job_throughput(dist, torch, ev0.elapsed_time(ev1), cfg.batch * steps)
     roof_region_ms = elapsed_ms
     if use_graphs:
@@ -670,7 +678,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
         roof_region_ms = r0.elapsed_time(r1)
         dom_ms, dom_n = store.kernel_time()
         store.time_kernel(0)
-    assert store.sync() == 0, "device status set during the roofline region"
+    sync_ok(store, "device status set during the roofline region")
     kernel_avg = None
     if args.kernel_times:
         # every kernel class event-timed over the same steps run call by call
@@ -682,7 +690,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
             ms, n = store.kernel_time()
             kernel_avg[KERNEL_NAMES[kid]] = {"ms_per_step": ms / steps, "launches_per_step": n / steps}
         store.time_kernel(0)
-        assert store.sync() == 0
+        sync_ok(store, "device status")
     step_bytes = np.mean([st["step"] for st in stats])
     achieved_step = step_bytes * steps / (elapsed_ms / 1e3) / 1e9
 
@@ -751,7 +759,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
         e1.record(stream)
         barrier(dist, torch)
         e_ms = max_over_ranks(dist, torch, e0.elapsed_time(e1))
-        assert store.sync() == 0
+        sync_ok(store, "device status")
         h2d = (r.numel() + w.numel()) * 8 + v.numel() * 4
         d2h = r.numel() * cfg.dim * 4
         e2e = {"value": cfg.batch * e2e_steps * world / (e_ms / 1e3), "unit": UNIT_YCSB, "h2d_bytes_per_step": h2d,
@@ -775,7 +783,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
         e1.record(stream)
         barrier(dist, torch)
         e_ms = max_over_ranks(dist, torch, e0.elapsed_time(e1))
-        assert store.sync() == 0
+        sync_ok(store, "device status")
         h2d = cfg.batch * 8 * 2 + cfg.batch * cfg.dim * 4
         d2h = cfg.batch * cfg.dim * 4
         e2e = {"value": cfg.batch * e2e_steps * world / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,

@@ -91,6 +91,13 @@ struct RowArgs {
     int NV;
     int G;
     int d;
+    uint32_t nrows;  // rows of the slot array (bounds-checked build)
+};
+
+// Sites of the bounds-checked build (in_bounds).
+enum CheckSite : uint32_t {
+    kChkSingleRow = 1, kChkSinglePos, kChkSmallRow, kChkSmallPos, kChkShortRun, kChkShortRow, kChkShortPos,
+    kChkLongItem, kChkLongPos, kChkCombineRun, kChkCombineRow, kChkHeadsPos, kChkListEntry
 };
 
 struct RunArgs {
@@ -134,18 +141,21 @@ template <int V, int KV, int ROWS = MLKV_REDUCE_ROWS_IN_FLIGHT, bool PRE = false
 __device__ __forceinline__ void sum_rows(typename Vec<V>::T (&acc)[KV], typename Vec<V>::T (&cmp)[KV],
                                          const float* __restrict__ grads,
                                          const uint32_t* __restrict__ spos, uint32_t s, uint32_t len, int d,
-                                         int NV, int G, int glane, unsigned gmask, uint32_t pl_first = 0u) {
+                                         int NV, int G, int glane, unsigned gmask, const ErrSink& err,
+                                         uint32_t site, uint32_t n, uint32_t pl_first = 0u) {
     using VT = typename Vec<V>::T;
     constexpr int UNR = KV >= ROWS ? 1 : ROWS / KV;
     for (uint32_t base = 0; base < len; base += G) {
         const uint32_t cnt = min((uint32_t)G, len - base);
+        if (MLKV_CHECK && !in_bounds(err, site, s + base + cnt - 1, n)) return;
         const uint32_t pl = (PRE && base == 0) ? pl_first
                             : (uint32_t)glane < cnt ? __ldg(spos + s + base + glane) : 0u;
         for (uint32_t x = 0; x < cnt; x += UNR) {
             VT g[UNR][KV];
 #pragma unroll
             for (int u = 0; u < UNR; ++u) {
-                const uint32_t p = __shfl_sync(gmask, pl, (int)(x + u) & (G - 1), G);
+                uint32_t p = __shfl_sync(gmask, pl, (int)(x + u) & (G - 1), G);
+                if (MLKV_CHECK && x + u < cnt && !in_bounds(err, site, p, n)) p = 0;
                 const VT* src = reinterpret_cast<const VT*>(grads + (size_t)p * d);
 #pragma unroll
                 for (int k = 0; k < KV; ++k) {
@@ -306,6 +316,10 @@ template <int V, int KV>
 __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, uint32_t s, uint32_t len,
                                           uint32_t row, uint32_t p0, int glane, unsigned gmask) {
     using VT = typename Vec<V>::T;
+    if (MLKV_CHECK && !(in_bounds(a.err, kChkShortRun, s + len, (unsigned long long)a.n + 1) &&
+                        in_bounds(a.err, kChkShortRun, 1, len) && in_bounds(a.err, kChkShortRow, row, ra.nrows) &&
+                        in_bounds(a.err, kChkShortPos, p0, a.n)))
+        return;
     VT w[KV], Gs[KV], acc[KV];
     // the positions of the run's other lookups load beside its row, state and
     // first gradient row, so a run of a few lookups costs two round trips
@@ -321,7 +335,7 @@ __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, u
     }
     if (len > 1)
         sum_rows<V, KV, MLKV_REDUCE_ROWS_IN_FLIGHT, true>(acc, acc, a.grads, a.spos, s + 1, rest, ra.d, ra.NV,
-                                                          ra.G, glane, gmask, pl0);
+                                                          ra.G, glane, gmask, a.err, kChkShortPos, a.n, pl0);
     adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
 }
 
@@ -441,7 +455,8 @@ __global__ void __launch_bounds__(256, MLKV_HEADS_MIN_BLOCKS) k_heads(RunArgs a)
         if (cnt + __popc(sm) > kListS || cnt1 + __popc(s1) > kList || cnt2 + __popc(s2) > kListS) flush();
         if (shrt && len > kSmallRun) lst[wib][cnt + __popc(sm & lt)] = make_uint4(p, p + len, r, pos);
         if (shrt && len == 1) sgl[wib][cnt1 + __popc(s1 & lt)] = make_uint2(r, pos);
-        if (smll) {
+        if (smll && MLKV_CHECK && !in_bounds(a.err, kChkHeadsPos, p + len - 1, n)) len = 2;
+        if (smll && (!MLKV_CHECK || in_bounds(a.err, kChkHeadsPos, p + len - 1, n))) {
             const uint32_t p1 = lane + 1 < 32 ? q1 : __ldg(a.spos + p + 1);
             const uint32_t p2 = len < 3 ? NONE : lane + 2 < 32 ? q2 : __ldg(a.spos + p + 2);
             const uint32_t p3 = len < 4 ? NONE : lane + 3 < 32 ? q3 : __ldg(a.spos + p + 3);
@@ -545,7 +560,8 @@ __device__ __forceinline__ uint4 run_meta(const RunArgs& a, uint32_t u, uint32_t
 template <int V, int KV>
 __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra, RunArgs a) {
     pdl_enter();
-    const uint32_t U = a.cur->n_short;
+    if (MLKV_CHECK && !in_bounds(a.err, kChkListEntry, a.cur->n_short, (unsigned long long)a.n + 1)) return;
+    const uint32_t U = min(a.cur->n_short, a.n);  // a list never holds more runs than lookups
     const int lane = threadIdx.x & 31, G = ra.G, glane = lane & (G - 1), gid = lane / G;
     const unsigned gmask = group_mask(G, gid);
     const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
@@ -579,7 +595,8 @@ __global__ void __launch_bounds__(256, MLKV_SINGLE_MIN_BLOCKS) k_single(RowArgs 
     pdl_enter();
     using VT = typename Vec<V>::T;
     constexpr int SG = MLKV_SINGLES;
-    const uint32_t U = a.cur->n_single;
+    if (MLKV_CHECK && !in_bounds(a.err, kChkListEntry, a.cur->n_single, (unsigned long long)a.n + 1)) return;
+    const uint32_t U = min(a.cur->n_single, a.n);  // a list never holds more runs than lookups
     const int lane = threadIdx.x & 31, G = ra.G, glane = lane & (G - 1);
     const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
     const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
@@ -599,6 +616,11 @@ __global__ void __launch_bounds__(256, MLKV_SINGLE_MIN_BLOCKS) k_single(RowArgs 
 #pragma unroll
         for (int j = 0; j < SG; ++j) {
             if (m[j].x == 0xFFFFFFFFu) continue;
+            if (MLKV_CHECK && !(in_bounds(a.err, kChkSingleRow, m[j].x, ra.nrows) &&
+                                in_bounds(a.err, kChkSinglePos, m[j].y, a.n))) {
+                m[j].x = 0xFFFFFFFFu;
+                continue;
+            }
             load_row_state<V, KV>(ra, m[j].x, w[j], Gs[j], glane);
             const VT* src = reinterpret_cast<const VT*>(a.grads + (size_t)m[j].y * ra.d);
 #pragma unroll
@@ -631,7 +653,8 @@ template <int V, int KV>
 __global__ void __launch_bounds__(256, KV >= 4 ? 2 : MLKV_SMALL_MIN_BLOCKS) k_small(RowArgs ra, RunArgs a) {
     pdl_enter();
     using VT = typename Vec<V>::T;
-    const uint32_t U = a.cur->n_small;
+    if (MLKV_CHECK && !in_bounds(a.err, kChkListEntry, a.cur->n_small, (unsigned long long)a.n + 1)) return;
+    const uint32_t U = min(a.cur->n_small, a.n);  // a list never holds more runs than lookups
     const int lane = threadIdx.x & 31, G = ra.G, glane = lane & (G - 1);
     const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
     const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
@@ -644,6 +667,11 @@ __global__ void __launch_bounds__(256, KV >= 4 ? 2 : MLKV_SMALL_MIN_BLOCKS) k_sm
         next = v < U ? __ldg(a.smalls + v) : make_uint4(0u, 0u, 0u, 0u);
         next3 = v < U ? __ldg(a.small_p3 + v) : NONE;
         VT w[KV], Gs[KV], g[kSmallRun][KV];
+        if (MLKV_CHECK && !(in_bounds(a.err, kChkSmallRow, m.x, ra.nrows) && in_bounds(a.err, kChkSmallPos, m.y, a.n) &&
+                            in_bounds(a.err, kChkSmallPos, m.z, a.n) &&
+                            (m.w == NONE || in_bounds(a.err, kChkSmallPos, m.w, a.n)) &&
+                            (p3 == NONE || in_bounds(a.err, kChkSmallPos, p3, a.n))))
+            continue;
         load_row_state<V, KV>(ra, m.x, w, Gs, glane);
         const uint32_t ps[kSmallRun] = {m.y, m.z, m.w, p3};
 #pragma unroll
@@ -680,6 +708,7 @@ __global__ void __launch_bounds__(256, MLKV_LONG_MIN_BLOCKS) k_long_sum(RowArgs 
     const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
     for (uint32_t it = group; it < NI; it += ngroups) {
         const uint32_t s = __ldg(a.item_s + it), e = __ldg(a.item_e + it);
+        if (MLKV_CHECK && !in_bounds(a.err, kChkLongItem, e, (unsigned long long)a.n + 1)) continue;
         VT acc[KV], cmp[KV];
 #pragma unroll
         for (int k = 0; k < KV; ++k) {
@@ -687,7 +716,8 @@ __global__ void __launch_bounds__(256, MLKV_LONG_MIN_BLOCKS) k_long_sum(RowArgs 
             cmp[k] = Vec<V>::zero();
         }
         sum_rows<V, KV, MLKV_LONG_ROWS_IN_FLIGHT, false, true>(acc, cmp, a.grads, a.spos, s, e > s ? e - s : 0u,
-                                                               ra.d, ra.NV, G, glane, gmask);
+                                                               ra.d, ra.NV, G, glane, gmask, a.err, kChkLongPos,
+                                                               a.n);
         // the chunk's (sum, compensation) pair
         VT* part = reinterpret_cast<VT*>(a.partial + (size_t)it * 2 * ra.dpad);
 #pragma unroll
@@ -753,9 +783,14 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
     const int group = threadIdx.x / G;
     const int ngroups = blockDim.x / G;
     for (uint32_t i = blockIdx.x; i < nb; i += gridDim.x) {  // block-uniform
+        if (MLKV_CHECK && !in_bounds(a.err, kChkCombineRun, i, a.max_long)) break;
         const uint32_t h = a.big_runs[i];
+        if (MLKV_CHECK && !in_bounds(a.err, kChkCombineRun, h, nl)) continue;
         const uint32_t base = a.long_base[h];
         const uint32_t m = (a.long_e[h] - a.long_s[h] + kChunk - 1) / kChunk;
+        if (MLKV_CHECK && !(in_bounds(a.err, kChkCombineRun, base + m, (unsigned long long)a.max_items + 1) &&
+                            in_bounds(a.err, kChkCombineRow, a.long_row[h], ra.nrows)))
+            continue;
         const uint32_t per = (m + ngroups - 1) / ngroups;
         const uint32_t k0 = min(m, group * per), k1 = min(m, k0 + per);
         VT acc[KV], cmp[KV];
@@ -806,6 +841,9 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
     for (uint32_t h = gg; h < nl; h += ngg) {  // uniform within the group
         const uint32_t m = (a.long_e[h] - a.long_s[h] + kChunk - 1) / kChunk;
         if (m > kBigRun) continue;
+        if (MLKV_CHECK && !(in_bounds(a.err, kChkCombineRun, a.long_base[h] + m, (unsigned long long)a.max_items + 1) &&
+                            in_bounds(a.err, kChkCombineRow, a.long_row[h], ra.nrows)))
+            continue;
         VT acc[KV], cmp[KV], w[KV], Gs[KV];
 #pragma unroll
         for (int k = 0; k < KV; ++k) {
@@ -824,12 +862,14 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
 template <int V, int KV>
 cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, const uint32_t* spos,
                        int64_t n, uint32_t sent, cudaStream_t st, CallCounters* cur) {
-    RowArgs ra{t->slots, t->geom.stride, t->geom.dpad, t->geom.NV, t->geom.G, t->geom.d};
+    RowArgs ra{t->slots, t->geom.stride, t->geom.dpad, t->geom.NV, t->geom.G, t->geom.d,
+               (uint32_t)(t->tiered ? t->cfg.hbm_cache_rows : t->cfg.capacity)};
     RunArgs a{grads, srow, spos, (uint32_t)n, sent, cur, t->s.short_runs, t->s.single_runs, t->s.small_runs,
               t->s.small_p3, t->s.long_s, t->s.long_e,
               t->s.long_row, t->s.long_base, t->s.item_s, t->s.item_e, t->s.big_runs, t->s.partial,
               (uint32_t)t->s.max_long,
-              (uint32_t)t->s.max_items, ErrSink{&t->dstate->status, t->status_dev_alias}, t->cfg.lr, t->cfg.eps};
+              (uint32_t)t->s.max_items, ErrSink{&t->dstate->status, t->status_dev_alias, t->dstate->chk},
+              t->cfg.lr, t->cfg.eps};
     // a warp per 32 positions, the windows dealt out grid-stride over at most
     // one wave of blocks
 #ifndef MLKV_HEADS_ONE_WAVE

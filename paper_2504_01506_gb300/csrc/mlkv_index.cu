@@ -72,9 +72,11 @@ __device__ __forceinline__ uint32_t probe_key(const IndexArgs& ia, unsigned long
     return ROW_ABSENT;
 }
 
-// Appends (pos, slot) to the miss list with one atomic per converged group of lanes.
+// Appends (pos, slot) to the miss list with one atomic per converged group of
+// lanes.  The list holds at most one entry per lookup (n): an entry past that
+// could only come from a counter left set, and is not written.
 __device__ __forceinline__ void append_miss(CallCounters* cur, uint32_t* miss_pos,
-                                            uint32_t* miss_slot, uint32_t pos, uint32_t slot) {
+                                            uint32_t* miss_slot, uint32_t pos, uint32_t slot, uint32_t n) {
     const unsigned m = __activemask();
     const int lane = threadIdx.x & 31;
     const int leader = __ffs(m) - 1;
@@ -82,8 +84,10 @@ __device__ __forceinline__ void append_miss(CallCounters* cur, uint32_t* miss_po
     if (lane == leader) base = atomicAdd(&cur->n_miss, (uint32_t)__popc(m));
     base = __shfl_sync(m, base, leader);
     const uint32_t i = base + __popc(m & lanemask_lt());
-    miss_pos[i] = pos;
-    miss_slot[i] = slot;
+    if (i < n) {
+        miss_pos[i] = pos;
+        miss_slot[i] = slot;
+    }
 }
 
 __device__ __forceinline__ void zero_counters(CallCounters* nxt) {
@@ -157,7 +161,7 @@ __global__ void __launch_bounds__(COUNT ? 1024 : 256) k_probe(IndexArgs ia, cons
             row = probe_key<INSERT>(ia, k[j], p, slot);
             if (!INSERT && report_absent && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
             if (slot_of_pos) slot_of_pos[p] = slot;
-            if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
+            if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot, n);
             if (memo_use == (int)MemoUse::Save) {
                 memo.key[p] = (int64_t)k[j];
                 memo.row[p] = row;
@@ -227,7 +231,7 @@ __global__ void __launch_bounds__(256, MLKV_GET_MIN_BLOCKS) k_get(IndexArgs ia, 
         uint32_t slot = 0;
         const int64_t key = keys[p];
         row = probe_key<INSERT>(ia, (unsigned long long)key, p, slot);
-        if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot);
+        if (INSERT && row == ROW_PENDING) append_miss(cur, miss_pos, miss_slot, p, slot, n);
         if (!INSERT && row == ROW_ABSENT) record_error(ia.err, MLKV_ERR_NOT_FOUND);
         memo.key[p] = key;
         memo.row[p] = row;
@@ -268,9 +272,9 @@ __global__ void __launch_bounds__(256, MLKV_GET_MIN_BLOCKS) k_get(IndexArgs ia, 
 // Miss path 1/3: flag the first occurrence of every new key.
 __global__ void k_miss_flag(const Slot* __restrict__ index, const uint32_t* __restrict__ miss_pos,
                             const uint32_t* __restrict__ miss_slot, uint32_t* __restrict__ flag,
-                            const CallCounters* cur) {
+                            const CallCounters* cur, uint32_t n) {
     pdl_enter();
-    const uint32_t m = cur->n_miss;
+    const uint32_t m = min(cur->n_miss, n);  // never more misses than lookups
     for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < m; i += gridDim.x * blockDim.x) {
         const uint32_t p = miss_pos[i];
         if (index[miss_slot[i]].aux == p) flag[p] = 1u;
@@ -288,10 +292,10 @@ __global__ void __launch_bounds__(256) k_miss_assign(IndexArgs ia, RowArgs ra,
                                                      const CallCounters* cur, const DevState* ds,
                                                      unsigned long long capacity, int init_row,
                                                      unsigned long long seed, float lo, float span,
-                                                     float state_init) {
+                                                     float state_init, uint32_t n) {
     pdl_enter();
     using VT = typename Vec<V>::T;
-    const uint32_t m = cur->n_miss;
+    const uint32_t m = min(cur->n_miss, n);
     const int G = ra.G, glane = threadIdx.x & (G - 1);
     const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
     const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
@@ -334,9 +338,9 @@ __global__ void __launch_bounds__(256) k_miss_finish(IndexArgs ia, RowArgs ra,
                                                      uint32_t* __restrict__ flag,
                                                      float* __restrict__ out,
                                                      const CallCounters* cur, DevState* ds,
-                                                     unsigned long long capacity) {
+                                                     unsigned long long capacity, uint32_t n) {
     pdl_enter();
-    const uint32_t m = cur->n_miss;
+    const uint32_t m = min(cur->n_miss, n);
     if (blockIdx.x == 0 && threadIdx.x == 0 && m) {
         const unsigned long long nr = ds->next_row + cur->n_new;
         ds->next_row = nr < capacity ? nr : capacity;
@@ -532,11 +536,11 @@ struct MissRun {
         MLKV_LAUNCH(t, 0, (k_miss_assign<V, KV>), g, 256, 0, st, index_args(t), init_ra, keys,
                     t->s.miss_pos, t->s.miss_slot, t->s.rank, cur, t->dstate,
                     (unsigned long long)t->cfg.capacity, mode == MissMode::Put ? 0 : 1,
-                    (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init);
+                    (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init, (uint32_t)n);
         MLKV_LAUNCH(t, 0, (k_miss_finish<V, KV>), g, 256, 0, st, index_args(t), init_ra,
                     t->s.miss_pos, t->s.miss_slot, mode == MissMode::Get ? nullptr : t->s.row_of_pos,
                     t->s.first_flag, mode == MissMode::Get ? out : nullptr, cur, t->dstate,
-                    (unsigned long long)t->cfg.capacity);
+                    (unsigned long long)t->cfg.capacity, (uint32_t)n);
         return cudaGetLastError();
     }
 };
@@ -626,7 +630,7 @@ cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n,
                                   float* out, cudaStream_t st, CallCounters* cur) {
     MLKV_LAUNCH(t, 0, k_miss_flag, capped_grid(t, n, 256, MLKV_MISS_BLOCKS_PER_SM), 256, 0, st, t->index,
                 t->s.miss_pos,
-                t->s.miss_slot, t->s.first_flag, cur);
+                t->s.miss_slot, t->s.first_flag, cur, (uint32_t)n);
     cudaError_t e = launch_exclusive_scan(t, t->s.first_flag, t->s.rank, n, &cur->n_new,
                                           &cur->n_miss, st);
     if (e != cudaSuccess) return e;

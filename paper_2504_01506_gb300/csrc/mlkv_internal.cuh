@@ -55,6 +55,7 @@ struct DevState {
     uint32_t last_unique;         // distinct rows of the last gradient apply
     CallCounters cc[2];           // the counters of every call but the gradient apply, in turn
     CallCounters cca[2];          // the gradient apply's, in turn
+    uint32_t chk[3];              // bounds-checked build: first failed check (site, index, bound)
 };
 
 // Row-kernel geometry: a row of d floats is NV vectors of V floats; a group of
@@ -177,6 +178,7 @@ struct mlkv_table {
     int other_recorded;
     int64_t n_applies;
     int64_t launches;
+    int captured;                // some call of this table was captured into a graph (see begin_call)
     mlkv::KernelTimer timer;
     double timed_ms;
     int64_t timed_launches;
@@ -189,10 +191,30 @@ namespace mlkv {
 struct ErrSink {
     uint32_t* dev;             // DevState::status
     volatile uint32_t* host;   // mapped pinned mirror
+    uint32_t* chk;             // DevState::chk (bounds-checked build), or null
 };
 
 __device__ __forceinline__ void record_error(const ErrSink& e, uint32_t code) {
     if (atomicCAS(e.dev, 0u, code) == 0u && e.host) *e.host = code;
+}
+
+// Bounds-checked build (-DMLKV_CHECK=1): the reduce kernels test the indices
+// they are about to use (rows, lookup positions, list entries); a failed test
+// records the first failing site with its index and bound and
+// MLKV_ERR_INVALID, and the access is skipped.  mlkv_sync reports the site.
+// In the normal build every test is compiled out.
+#ifndef MLKV_CHECK
+#define MLKV_CHECK 0
+#endif
+__device__ __forceinline__ bool in_bounds(const ErrSink& e, uint32_t site, unsigned long long idx,
+                                          unsigned long long bound) {
+    if (!MLKV_CHECK || idx < bound) return true;
+    if (e.chk && atomicCAS(e.chk, 0u, site) == 0u) {
+        e.chk[1] = (uint32_t)idx;
+        e.chk[2] = (uint32_t)bound;
+    }
+    record_error(e, MLKV_ERR_INVALID);
+    return false;
 }
 
 // row_loc encoding of the tiered store

@@ -256,6 +256,9 @@ bool capturing(cudaStream_t st) {
 // other copy for the next one in its first kernel, so no memset is enqueued.
 // A captured graph replays a fixed sequence of calls, which may be odd in
 // number: there every call zeroes its own copy first, with a one-block kernel.
+// Replays do not pass through the host, so after the first capture the host
+// no longer knows which copy the last replay left set: from then on a call
+// launched directly zeroes its own copy first too.
 //
 // Stale-synchronous mode (staleness_bound s >= 1, Gets and applies on two
 // streams): a Get waits for every apply issued more than s applies before it,
@@ -264,6 +267,11 @@ bool capturing(cudaStream_t st) {
 // apply waits for the call before it on the other stream (the Get whose keys
 // it updates) and for the apply before it.  Applies count their own counters,
 // so a Get and an apply in flight together never share them.
+void own_counters(mlkv_table* t, CallCounters* cur, cudaStream_t st) {
+    if (capturing(st)) t->captured = 1;
+    if (t->captured) launch_zero_counters(t, cur, st);
+}
+
 CallScope begin_call(mlkv_table* t, cudaStream_t st, bool get = false) {
     const int p = t->parity;
     t->parity ^= 1;
@@ -277,7 +285,7 @@ CallScope begin_call(mlkv_table* t, cudaStream_t st, bool get = false) {
         cs.t = t;
         cs.st = st;
     }
-    if (capturing(st)) launch_zero_counters(t, cs.cur, st);
+    own_counters(t, cs.cur, st);
     return cs;
 }
 
@@ -295,7 +303,7 @@ CallScope begin_apply(mlkv_table* t, cudaStream_t st) {
         cs.st = st;
         cs.apply = true;
     }
-    if (capturing(st)) launch_zero_counters(t, cs.cur, st);
+    own_counters(t, cs.cur, st);
     return cs;
 }
 
@@ -309,9 +317,15 @@ int check_call(mlkv_table* t, const void* keys, int64_t n, const void* buf, bool
                          (long long)t->cfg.max_batch);
     if (n > 0 && (!keys || (need_buf && !buf))) return set_error(t, MLKV_ERR_INVALID, "null pointer");
     const uint32_t sticky = *(volatile uint32_t*)t->status_host;
-    if (sticky)
+    if (sticky) {
+        uint32_t chk[3] = {0, 0, 0};
+        if (MLKV_CHECK) cudaMemcpy(chk, t->dstate->chk, sizeof(chk), cudaMemcpyDeviceToHost);
+        if (chk[0])  // a bounds-checked build found an index out of range
+            return set_error(t, (int)sticky, "sticky device status %u (%s) from an earlier call; check site %u, "
+                             "index %u >= bound %u", sticky, mlkv_status_string((int)sticky), chk[0], chk[1], chk[2]);
         return set_error(t, (int)sticky, "sticky device status %u (%s) from an earlier call", sticky,
                          mlkv_status_string((int)sticky));
+    }
     return n == 0 ? -1 : MLKV_OK;
 }
 
@@ -822,7 +836,15 @@ int mlkv_sync(mlkv_table* t) {
     if (t->tiered) CK(t, cudaStreamSynchronize(t->tier.la_stream));
     uint32_t st = 0;
     CK(t, cudaMemcpy(&st, &t->dstate->status, sizeof(st), cudaMemcpyDeviceToHost));
-    if (st) set_error(t, (int)st, "device status %u (%s)", st, mlkv_status_string((int)st));
+    if (st) {
+        uint32_t chk[3] = {0, 0, 0};
+        CK(t, cudaMemcpy(chk, t->dstate->chk, sizeof(chk), cudaMemcpyDeviceToHost));
+        if (chk[0])  // a bounds-checked build found an index out of range
+            set_error(t, (int)st, "device status %u (%s): check site %u, index %u >= bound %u", st,
+                      mlkv_status_string((int)st), chk[0], chk[1], chk[2]);
+        else
+            set_error(t, (int)st, "device status %u (%s)", st, mlkv_status_string((int)st));
+    }
     return (int)st;
 }
 
@@ -830,6 +852,7 @@ int mlkv_clear_status(mlkv_table* t) {
     if (!t) return MLKV_ERR_INVALID;
     CK(t, cudaDeviceSynchronize());
     CK(t, cudaMemset(&t->dstate->status, 0, sizeof(uint32_t)));
+    CK(t, cudaMemset(t->dstate->chk, 0, sizeof(t->dstate->chk)));
     CK(t, cudaDeviceSynchronize());
     *(volatile uint32_t*)t->status_host = 0;
     t->last_error[0] = 0;

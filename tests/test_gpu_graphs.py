@@ -75,3 +75,74 @@ def test_tiered_calls_refuse_capture():
     store.clear_status()
     store.get(keys)  # still usable after the refused capture
     assert store.sync() == 0
+
+
+@pytest.mark.parametrize("last", [0, 1])
+def test_direct_calls_after_replays(last):
+    """Replays do not pass through the host, so the host cannot tell which
+    counters the last replayed call left set.  Two graphs are captured (one
+    per counter copy), replayed in either order, and then the same kind of
+    calls is made directly: the table must match one driven by direct calls
+    only, and the oracle.  The batch is mostly runs of one lookup and
+    max_batch is its size, so a run list counted twice would run past its end."""
+    torch = torch_cuda()
+    import oracle
+
+    rng = np.random.default_rng(31 + last)
+    n = 3000
+    cfg = W.scaled(W.tiny(), 20, 1)
+    cfg.batch = n
+    graphed, ref = make_pair(cfg, capacity=cfg.n_keys, max_batch=n)
+    plain, _ = make_pair(cfg, capacity=cfg.n_keys, max_batch=n)
+    pre = cfg.preload_keys()
+    for st in (graphed, plain):
+        st.insert(dev(pre[:n]))
+        st.insert(dev(pre[n:]))
+    ref.insert(pre)
+    batches = []
+    for b in range(4):
+        k = rng.choice(pre, n, replace=False)
+        k[:300] = k[300:600]  # a few runs of two; the rest runs of one
+        batches.append((k, (rng.standard_normal((n, cfg.dim)) * 0.01).astype(np.float32)))
+    kd = [dev(k) for k, _ in batches]
+    gd = [dev(g) for _, g in batches]
+    outs = [torch.empty((n, cfg.dim), device="cuda") for _ in batches]
+    torch.cuda.synchronize()
+    s = torch.cuda.Stream()
+    graphs = []
+    with torch.cuda.stream(s):
+        for j in range(2):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s):
+                graphed.get(kd[j], out=outs[j])
+                graphed.apply_grad(kd[j], gd[j])
+            graphs.append(g)
+    torch.cuda.synchronize()
+    order = [1 - last, last]
+    for j in order:  # replays, the last one `last`
+        graphs[j].replay()
+    for j in (2, 3):  # then direct calls
+        graphed.get(kd[j], out=outs[j])
+        graphed.apply_grad(kd[j], gd[j])
+    assert graphed.sync() == 0
+    for j in order + [2, 3]:  # the same calls, made directly, and in the oracle
+        want = plain.get(kd[j])
+        plain.apply_grad(kd[j], gd[j])
+        k, g = batches[j]
+        rw, _, _ = ref.get(k)
+        ref.apply_grad(k, g)
+        if j >= 2:
+            assert_bits(host(outs[j]), host(want), f"Get of direct call {j}")
+            assert_bits(host(outs[j]), rw, f"Get of direct call {j} vs oracle")
+    assert plain.sync() == 0
+
+    def export(store):  # max_batch keys at a time
+        parts = [store.export(dev(pre[i:i + n])) for i in range(0, len(pre), n)]
+        return (np.concatenate([host(p[0]) for p in parts]), np.concatenate([host(p[1]) for p in parts]))
+
+    (w, G), (pw, pG) = export(graphed), export(plain)
+    rw, rG = ref.export(pre)
+    assert_bits(w, pw, "rows vs direct calls only")
+    assert_bits(G, pG, "state vs direct calls only")
+    assert_bits(w, rw, "rows vs oracle")
+    assert_bits(G, rG, "state vs oracle")
