@@ -38,7 +38,10 @@
  *   - No call allocates device memory except mlkv_open (the table, its index,
  *     its scratch sized for max_batch) and the first *_host call (staging
  *     sized for max_batch).  Every loop inside a kernel is bounded (the probe
- *     limit, the tier's sweep limit); no kernel spins on a flag.
+ *     limit, the tier's sweep limit).  The only waits are the grid barriers of
+ *     the kernel that gives new keys their rows, between the blocks of that
+ *     one grid (one block per SM; the next kernel may launch only after them),
+ *     bounded: one that runs out records MLKV_ERR_TIMEOUT.
  */
 #ifndef MLKV_GPU_H
 #define MLKV_GPU_H
@@ -58,8 +61,8 @@ extern "C" {
 #define MLKV_ERR_FULL 5        /* more distinct keys than `capacity` */
 #define MLKV_ERR_PROBE_LIMIT 6 /* an index probe exceeded the probe bound */
 #define MLKV_ERR_NOT_FOUND 7   /* absent key and insert_on_miss == 0 */
-#define MLKV_ERR_TIMEOUT 8     /* reserved for a bounded wait inside a kernel that ran out; no kernel
-                                  of this library waits on a flag or another kernel, so none records it */
+#define MLKV_ERR_TIMEOUT 8     /* a bounded wait inside a kernel ran out: the grid barriers of the
+                                  miss path (new keys) of a call, between blocks of one grid */
 
 /* Largest dimension the row kernels take (8 vectors per lane of a warp). */
 #define MLKV_MAX_DIM 1024  /* dim > 256 needs dim % 4 == 0 */
@@ -67,10 +70,11 @@ extern "C" {
 /* Segments (runs of one key in a gradient batch) of at most this many
  * occurrences are summed by one lane group in occurrence order, so their
  * Adagrad step is the same op sequence as a sequential fp32 statement of it.
- * Longer segments are summed in chunks of 64 lookups with compensated (TwoSum)
- * additions and the chunks' (sum, compensation) pairs combined in a fixed
- * order, the sum rounded once: deterministic run to run and within about one
- * rounding of the exact sum, not the sequential fp32 rounding. */
+ * Longer segments are summed in chunks (64 lookups in calls of at least 2^19
+ * lookups, 16 in smaller ones) with compensated (TwoSum) additions and the
+ * chunks' (sum, compensation) pairs combined in a fixed order, the sum rounded
+ * once: deterministic run to run and within about one rounding of the exact
+ * sum, not the sequential fp32 rounding. */
 #define MLKV_SEQ_SEGMENT_MAX 32
 
 /* Flags of mlkv_config.flags. */

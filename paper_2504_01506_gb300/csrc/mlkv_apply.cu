@@ -27,7 +27,8 @@
 //                 gradient row and the run's other positions are loaded
 //                 together, the rest summed in occurrence order, then the
 //                 Adagrad step.
-//  k_long_sum     one lane group per chunk of kChunk lookups of a long run
+//  k_long_sum     one lane group per chunk of 64 lookups (16 in calls of
+//                 fewer than 2^19 lookups) of a long run
 //                 (Zipf-hot keys reach 10^4-10^5 lookups): the chunk's sum,
 //                 compensated, to scratch as a (sum, compensation) pair.
 //  k_long_combine one block per long run: the chunk pairs are split over the
@@ -42,13 +43,24 @@
 // per warp): the access pattern is random 512-byte rows, which HBM serves near
 // its copy bandwidth only with many requests in flight.  Results do not depend
 // on scheduling.
+#include <algorithm>
+
 #include "mlkv_internal.cuh"
 
 namespace mlkv {
 
 namespace {
 
-constexpr int kChunk = 64;
+// Long runs are summed in chunks: of kChunkLarge lookups in calls of at least
+// MLKV_SMALL_BATCH lookups, of kChunkSmall in smaller ones (few long runs:
+// more chunks to sum in parallel).  Set at build time.
+#ifndef MLKV_SMALL_BATCH
+#define MLKV_SMALL_BATCH (1u << 19)
+#endif
+#ifndef MLKV_CHUNK_SMALL
+#define MLKV_CHUNK_SMALL 16
+#endif
+constexpr uint32_t kChunkLarge = 64, kChunkSmall = MLKV_CHUNK_SMALL, kSmallBatch = MLKV_SMALL_BATCH;
 // Long runs of more than kBigRun chunk sums (the hottest rows) are combined by
 // a whole 1024-thread block of k_long_combine; the rest by one lane group each.
 constexpr uint32_t kBigRun = 32;
@@ -81,7 +93,7 @@ constexpr uint32_t NONE = 0xFFFFFFFFu;  // no position (a small run's record pas
 #define MLKV_LONG_ROWS_IN_FLIGHT 8
 #endif
 #ifndef MLKV_LONG_MIN_BLOCKS
-#define MLKV_LONG_MIN_BLOCKS 3
+#define MLKV_LONG_MIN_BLOCKS 2
 #endif
 
 struct RowArgs {
@@ -123,6 +135,7 @@ struct RunArgs {
     float* partial;        // [max_items][dpad]
     uint32_t max_long;
     uint32_t max_items;
+    uint32_t chunk;        // lookups per chunk of a long run (kChunkLarge or kChunkSmall)
     ErrSink err;
     float lr, eps;
 };
@@ -268,11 +281,11 @@ __device__ __forceinline__ uint32_t scan_end(const uint32_t* __restrict__ srow, 
     return run_end(srow, n, q0 + 1023u, row, lane);
 }
 
-// Chunks of kChunk lookups of the long runs qs[k] .. qe[k] (k < nq): this
+// Chunks of `chunk` lookups of the long runs qs[k] .. qe[k] (k < nq): this
 // lane's run's count, and the exclusive prefix over the lanes (the whole warp).
 __device__ __forceinline__ uint32_t long_chunks(const uint32_t* qs, const uint32_t* qe, int nq, int lane,
-                                                uint32_t& excl) {
-    const uint32_t nit = lane < nq ? (qe[lane] - qs[lane] + kChunk - 1) / kChunk : 0u;
+                                                uint32_t chunk, uint32_t& excl) {
+    const uint32_t nit = lane < nq ? (qe[lane] - qs[lane] + chunk - 1) / chunk : 0u;
     uint32_t x = nit;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -290,21 +303,22 @@ __device__ __forceinline__ void write_long_runs(const RunArgs& a, const uint32_t
                                                 const uint32_t* qr, int nq, uint32_t h0, uint32_t ib0,
                                                 int lane) {
     uint32_t excl;
-    long_chunks(qs, qe, nq, lane, excl);
+    const uint32_t chunk = a.chunk;
+    long_chunks(qs, qe, nq, lane, chunk, excl);
     if (lane < nq) {
         a.long_s[h0 + lane] = qs[lane];
         a.long_e[h0 + lane] = qe[lane];
         a.long_row[h0 + lane] = qr[lane];
         a.long_base[h0 + lane] = ib0 + excl;
-        if ((qe[lane] - qs[lane] + kChunk - 1) / kChunk > kBigRun) a.big_runs[atomicAdd(&a.cur->n_big, 1u)] = h0 + lane;
+        if ((qe[lane] - qs[lane] + chunk - 1) / chunk > kBigRun) a.big_runs[atomicAdd(&a.cur->n_big, 1u)] = h0 + lane;
     }
     for (int k = 0; k < nq; ++k) {
         const uint32_t s = qs[k], e = qe[k];
-        const uint32_t m = (e - s + kChunk - 1) / kChunk;
+        const uint32_t m = (e - s + chunk - 1) / chunk;
         const uint32_t ib = ib0 + __shfl_sync(0xffffffffu, excl, k);
         for (uint32_t c = lane; c < m; c += 32) {
-            a.item_s[ib + c] = s + c * kChunk;
-            a.item_e[ib + c] = min(s + (c + 1) * kChunk, e);
+            a.item_s[ib + c] = s + c * chunk;
+            a.item_e[ib + c] = min(s + (c + 1) * chunk, e);
         }
     }
 }
@@ -472,7 +486,7 @@ __global__ void __launch_bounds__(256, MLKV_HEADS_MIN_BLOCKS) k_heads(RunArgs a)
             if (nq == kQueue) {
                 measure();
                 uint32_t excl, h0 = 0, ib0 = 0;
-                const uint32_t items = long_chunks(qs[wib], qe[wib], nq, lane, excl);
+                const uint32_t items = long_chunks(qs[wib], qe[wib], nq, lane, a.chunk, excl);
                 if (lane == 0) {
                     h0 = atomicAdd(&a.cur->n_long, (uint32_t)nq);
                     ib0 = atomicAdd(&a.cur->n_items, items);
@@ -498,7 +512,7 @@ __global__ void __launch_bounds__(256, MLKV_HEADS_MIN_BLOCKS) k_heads(RunArgs a)
     }
     measure();
     uint32_t excl;
-    const uint32_t items = long_chunks(qs[wib], qe[wib], nq, lane, excl);
+    const uint32_t items = long_chunks(qs[wib], qe[wib], nq, lane, a.chunk, excl);
     if (lane == 0) {
         wsh[wib] = (uint32_t)cnt;
         wlg[wib] = (uint32_t)nq;
@@ -566,13 +580,15 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
     const unsigned gmask = group_mask(G, gid);
     const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
     const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
-    // Runs take 2 .. 32 lookups, so fixed shares would leave the kernel to the
-    // group with the most lookups: each group claims chunks of kGrab runs, its
-    // first chunk by its index, the rest from a counter (one atomic a chunk)
-    constexpr uint32_t kGrab = MLKV_SHORT_GRAB;
-    uint32_t base = group * kGrab;
+    // Runs take 5 .. 32 lookups, so fixed shares would leave the kernel to the
+    // group with the most lookups: each group claims chunks of `grab` runs, its
+    // first chunk by its index, the rest from a counter (one atomic a chunk).
+    // With fewer runs than MLKV_SHORT_GRAB per group, one run at a time: every
+    // run then starts at once instead of queueing behind others.
+    const uint32_t grab = U >= ngroups * (uint32_t)MLKV_SHORT_GRAB ? (uint32_t)MLKV_SHORT_GRAB : 1u;
+    uint32_t base = group * grab;
     while (base < U) {  // uniform within the group
-        const uint32_t end = min(U, base + kGrab);
+        const uint32_t end = min(U, base + grab);
         uint4 next = run_meta(a, base, end);
         for (uint32_t u = base; u < end; ++u) {
             const uint4 m = next;  // (start, end, row, first lookup)
@@ -580,8 +596,8 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
             short_run<V, KV>(ra, a, m.x, m.y - m.x, m.z, m.w, glane, gmask);
         }
         uint32_t c = 0;
-        if (glane == 0) c = atomicAdd(&a.cur->short_next, kGrab);
-        base = ngroups * kGrab + __shfl_sync(gmask, c, 0, G);
+        if (glane == 0) c = atomicAdd(&a.cur->short_next, grab);
+        base = ngroups * grab + __shfl_sync(gmask, c, 0, G);
     }
 }
 
@@ -787,7 +803,7 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
         const uint32_t h = a.big_runs[i];
         if (MLKV_CHECK && !in_bounds(a.err, kChkCombineRun, h, nl)) continue;
         const uint32_t base = a.long_base[h];
-        const uint32_t m = (a.long_e[h] - a.long_s[h] + kChunk - 1) / kChunk;
+        const uint32_t m = (a.long_e[h] - a.long_s[h] + a.chunk - 1) / a.chunk;
         if (MLKV_CHECK && !(in_bounds(a.err, kChkCombineRun, base + m, (unsigned long long)a.max_items + 1) &&
                             in_bounds(a.err, kChkCombineRow, a.long_row[h], ra.nrows)))
             continue;
@@ -839,7 +855,7 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
     }
     const uint32_t gg = blockIdx.x * ngroups + group, ngg = gridDim.x * ngroups;
     for (uint32_t h = gg; h < nl; h += ngg) {  // uniform within the group
-        const uint32_t m = (a.long_e[h] - a.long_s[h] + kChunk - 1) / kChunk;
+        const uint32_t m = (a.long_e[h] - a.long_s[h] + a.chunk - 1) / a.chunk;
         if (m > kBigRun) continue;
         if (MLKV_CHECK && !(in_bounds(a.err, kChkCombineRun, a.long_base[h] + m, (unsigned long long)a.max_items + 1) &&
                             in_bounds(a.err, kChkCombineRow, a.long_row[h], ra.nrows)))
@@ -868,8 +884,8 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
               t->s.small_p3, t->s.long_s, t->s.long_e,
               t->s.long_row, t->s.long_base, t->s.item_s, t->s.item_e, t->s.big_runs, t->s.partial,
               (uint32_t)t->s.max_long,
-              (uint32_t)t->s.max_items, ErrSink{&t->dstate->status, t->status_dev_alias, t->dstate->chk},
-              t->cfg.lr, t->cfg.eps};
+              (uint32_t)t->s.max_items, n >= kSmallBatch ? kChunkLarge : kChunkSmall,
+              ErrSink{&t->dstate->status, t->status_dev_alias, t->dstate->chk}, t->cfg.lr, t->cfg.eps};
     // a warp per 32 positions, the windows dealt out grid-stride over at most
     // one wave of blocks
 #ifndef MLKV_HEADS_ONE_WAVE
@@ -902,7 +918,11 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
 
 int64_t long_runs_bound(int64_t max_batch) { return max_batch / (MLKV_SEQ_SEGMENT_MAX + 1) + 1; }
 
-int64_t long_items_bound(int64_t max_batch) { return max_batch / kChunk + long_runs_bound(max_batch) + 1; }
+int64_t long_items_bound(int64_t max_batch) {
+    // chunks of kChunkLarge lookups in calls of at least kSmallBatch lookups, of kChunkSmall below
+    const int64_t small = std::min<int64_t>(max_batch, (int64_t)kSmallBatch - 1) / kChunkSmall;
+    return std::max<int64_t>(max_batch / kChunkLarge, small) + long_runs_bound(max_batch) + 1;
+}
 
 cudaError_t launch_reduce_apply(mlkv_table* t, const float* grads, const uint32_t* srow,
                                 const uint32_t* spos, int64_t n, uint32_t sent, cudaStream_t st,

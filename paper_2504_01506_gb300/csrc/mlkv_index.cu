@@ -269,41 +269,152 @@ __global__ void __launch_bounds__(256, MLKV_GET_MIN_BLOCKS) k_get(IndexArgs ia, 
     }
 }
 
-// Miss path 1/3: flag the first occurrence of every new key.
-__global__ void k_miss_flag(const Slot* __restrict__ index, const uint32_t* __restrict__ miss_pos,
-                            const uint32_t* __restrict__ miss_slot, uint32_t* __restrict__ flag,
-                            const CallCounters* cur, uint32_t n) {
-    pdl_enter();
-    const uint32_t m = min(cur->n_miss, n);  // never more misses than lookups
-    for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < m; i += gridDim.x * blockDim.x) {
-        const uint32_t p = miss_pos[i];
-        if (index[miss_slot[i]].aux == p) flag[p] = 1u;
-    }
+// ---------------------------------------------------------------------------
+// The miss path: new keys of a call get rows.  One kernel, one block per SM.
+// In steady-state training nothing misses and every block returns at once; a
+// call with misses runs four phases separated by grid barriers:
+//   1. flag the first occurrence of each new key (the lookup whose position
+//      survived in the slot's aux);
+//   2. rank the flags: an exclusive scan over the call's positions, block b
+//      owning positions [b * per, (b + 1) * per);
+//   3. each first occurrence takes row = rows handed out so far + rank and
+//      writes its init row (not for Put) and state_init;
+//   4. every missed lookup reads its key's row (a Get gathers it into its
+//      output), flags and the slot's aux go back to idle, the row counter
+//      advances.
+// Data written by other blocks within the kernel is read from L2 (ld.cg).
+constexpr int kMissThreads = 512;
+constexpr int kMissWarps = kMissThreads / 32;
+constexpr uint32_t kBarrierSpins = 1u << 21;  // with its L2 load and 100 ns sleep, 1-2 s a barrier
+
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
 }
 
-// Miss path 2/3 (after the scan of the flags): hand out rows and write the
-// new rows (init row unless Put, state_init).
+// Every block of the grid arrives at `ctr` (zero at the call's start) and waits
+// until all have.  Only blocks of this one grid wait here, and the kernel lets
+// the next kernel launch only after its last barrier, so every block of the
+// grid (one per SM) can become resident.  The wait is bounded: a spin that runs
+// out records MLKV_ERR_TIMEOUT and the block returns (false).
+__device__ bool grid_barrier(uint32_t* ctr, const ErrSink& err) {
+    __shared__ int ok;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        ok = 1;
+        __threadfence();
+        atomicAdd(ctr, 1u);
+        uint32_t spins = 0;
+        while (ld_acquire_u32(ctr) < gridDim.x) {
+            if (++spins > kBarrierSpins) {
+                record_error(err, MLKV_ERR_TIMEOUT);
+                ok = 0;
+                break;
+            }
+            __nanosleep(100);
+        }
+        __threadfence();
+    }
+    __syncthreads();
+    return ok != 0;
+}
+
+// Sum over the block of one value per thread.
+__device__ __forceinline__ uint32_t miss_block_sum(uint32_t v) {
+    __shared__ uint32_t part[kMissWarps];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();
+    if (lane == 0) part[w] = v;
+    __syncthreads();
+    uint32_t t = 0;
+#pragma unroll
+    for (int k = 0; k < kMissWarps; ++k) t += part[k];
+    return t;
+}
+
+// Exclusive scan over the block of one value per thread; *total = the sum.
+__device__ __forceinline__ uint32_t miss_block_scan(uint32_t v, uint32_t& total) {
+    __shared__ uint32_t part[kMissWarps];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    uint32_t x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    __syncthreads();
+    if (lane == 31) part[w] = x;
+    __syncthreads();
+    uint32_t before = 0;
+    total = 0;
+#pragma unroll
+    for (int k = 0; k < kMissWarps; ++k) {
+        if (k < w) before += part[k];
+        total += part[k];
+    }
+    return before + x - v;
+}
+
 template <int V, int KV>
-__global__ void __launch_bounds__(256) k_miss_assign(IndexArgs ia, RowArgs ra,
-                                                     const int64_t* __restrict__ keys,
-                                                     const uint32_t* __restrict__ miss_pos,
-                                                     const uint32_t* __restrict__ miss_slot,
-                                                     const uint32_t* __restrict__ rank,
-                                                     const CallCounters* cur, const DevState* ds,
-                                                     unsigned long long capacity, int init_row,
-                                                     unsigned long long seed, float lo, float span,
-                                                     float state_init, uint32_t n) {
-    pdl_enter();
+__global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra, const int64_t* __restrict__ keys,
+                                                       uint32_t n, const uint32_t* __restrict__ miss_pos,
+                                                       const uint32_t* __restrict__ miss_slot,
+                                                       uint32_t* __restrict__ flag, uint32_t* __restrict__ rank,
+                                                       uint32_t* __restrict__ block_sums,
+                                                       uint32_t* __restrict__ row_of_pos, float* __restrict__ out,
+                                                       CallCounters* cur, DevState* ds,
+                                                       unsigned long long capacity, int init_row,
+                                                       unsigned long long seed, float lo, float span,
+                                                       float state_init) {
+    // waits for the kernel before it, like every kernel; lets the next one
+    // launch only once the grid barriers are behind it (see grid_barrier)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const uint32_t m = min(cur->n_miss, n);  // never more misses than lookups
+    if (m == 0) {
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+        return;
+    }
     using VT = typename Vec<V>::T;
-    const uint32_t m = min(cur->n_miss, n);
+    const uint32_t nthreads = gridDim.x * blockDim.x;
+    const uint32_t tid = blockIdx.x * blockDim.x + threadIdx.x;
+    // 1. first occurrences
+    for (uint32_t i = tid; i < m; i += nthreads) {
+        const uint32_t p = miss_pos[i];
+        if (ia.index[miss_slot[i]].aux == p) flag[p] = 1u;
+    }
+    if (!grid_barrier(&cur->bar[0], ia.err)) return;
+    // 2. ranks: the first occurrences at earlier positions
+    const uint32_t per = (n + gridDim.x - 1) / gridDim.x;
+    const uint32_t p_lo = min(n, blockIdx.x * per), p_hi = min(n, p_lo + per);
+    uint32_t cnt = 0;
+    for (uint32_t p = p_lo + threadIdx.x; p < p_hi; p += blockDim.x) cnt += __ldcg(flag + p);
+    const uint32_t mine = miss_block_sum(cnt);
+    if (threadIdx.x == 0) block_sums[blockIdx.x] = mine;
+    if (!grid_barrier(&cur->bar[1], ia.err)) return;
+    uint32_t b_before = 0;
+    for (uint32_t b = threadIdx.x; b < blockIdx.x; b += blockDim.x) b_before += __ldcg(block_sums + b);
+    uint32_t run = miss_block_sum(b_before);
+    for (uint32_t p0 = p_lo; p0 < p_hi; p0 += blockDim.x) {  // uniform
+        const uint32_t p = p0 + threadIdx.x;
+        const uint32_t f = p < p_hi ? __ldcg(flag + p) : 0u;
+        uint32_t tot;
+        const uint32_t ex = miss_block_scan(f, tot);
+        if (f) rank[p] = run + ex;
+        run += tot;
+    }
+    if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) cur->n_new = run;  // every first occurrence
+    if (!grid_barrier(&cur->bar[2], ia.err)) return;
+    // 3. rows of the first occurrences
     const int G = ra.G, glane = threadIdx.x & (G - 1);
-    const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
-    const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
+    const uint32_t group = tid / G, ngroups = nthreads / G;
     const unsigned long long next = ds->next_row;
     for (uint32_t i = group; i < m; i += ngroups) {
         const uint32_t p = miss_pos[i], s = miss_slot[i];
         if (ia.index[s].aux != p) continue;
-        const unsigned long long r = next + rank[p];
+        const unsigned long long r = next + __ldcg(rank + p);
         if (r >= capacity) {
             if (glane == 0) record_error(ia.err, MLKV_ERR_FULL);
             continue;
@@ -326,31 +437,15 @@ __global__ void __launch_bounds__(256) k_miss_assign(IndexArgs ia, RowArgs ra,
         }
         if (glane == 0) ia.index[s].row = (uint32_t)r;
     }
-}
-
-// Miss path 3/3: every missed lookup reads its key's row id (gathering the
-// row for Get), clears its flag and the slot's aux; the row counter advances.
-template <int V, int KV>
-__global__ void __launch_bounds__(256) k_miss_finish(IndexArgs ia, RowArgs ra,
-                                                     const uint32_t* __restrict__ miss_pos,
-                                                     const uint32_t* __restrict__ miss_slot,
-                                                     uint32_t* __restrict__ row_of_pos,
-                                                     uint32_t* __restrict__ flag,
-                                                     float* __restrict__ out,
-                                                     const CallCounters* cur, DevState* ds,
-                                                     unsigned long long capacity, uint32_t n) {
-    pdl_enter();
-    const uint32_t m = min(cur->n_miss, n);
-    if (blockIdx.x == 0 && threadIdx.x == 0 && m) {
-        const unsigned long long nr = ds->next_row + cur->n_new;
+    if (!grid_barrier(&cur->bar[3], ia.err)) return;
+    // 4. every missed lookup takes its key's row
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        const unsigned long long nr = next + __ldcg(&cur->n_new);
         ds->next_row = nr < capacity ? nr : capacity;
     }
-    const int G = ra.G, glane = threadIdx.x & (G - 1);
-    const uint32_t group = (blockIdx.x * blockDim.x + threadIdx.x) / G;
-    const uint32_t ngroups = (gridDim.x * blockDim.x) / G;
     for (uint32_t i = group; i < m; i += ngroups) {
         const uint32_t p = miss_pos[i], s = miss_slot[i];
-        const uint32_t r0 = ia.index[s].row;
+        const uint32_t r0 = ld_u32_relaxed(&ia.index[s].row);
         const uint32_t r = r0 == ROW_PENDING ? ROW_ABSENT : r0;
         if (glane == 0) {
             if (row_of_pos) row_of_pos[p] = r;
@@ -361,6 +456,7 @@ __global__ void __launch_bounds__(256) k_miss_finish(IndexArgs ia, RowArgs ra,
             copy_row<V, KV>(ra.slots + (size_t)(r == ROW_ABSENT ? 0 : r) * ra.stride,
                             out + (size_t)p * ra.d, ra.NV, G, glane, r == ROW_ABSENT);
     }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 // Put 1/2: the last occurrence of each key wins: aux = min over its
@@ -518,29 +614,18 @@ struct GetRun {
     }
 };
 
-// Blocks per SM of the miss path's kernels (grid-stride loops over the device's
-// miss count; set at build time).  In steady-state training nothing misses and
-// they return at once, at a cost that grows with the blocks launched.
-#ifndef MLKV_MISS_BLOCKS_PER_SM
-#define MLKV_MISS_BLOCKS_PER_SM 4
-#endif
-
 template <int V, int KV>
 struct MissRun {
     static cudaError_t run(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode, float* out,
                            cudaStream_t st, CallCounters* cur) {
-        const unsigned g = capped_grid(t, n * (int64_t)t->geom.G, 256, MLKV_MISS_BLOCKS_PER_SM);
         const float span = t->cfg.init_hi - t->cfg.init_lo;
         RowArgs init_ra = row_args(t);  // new rows live in the host tier when tiered
         if (t->tiered) init_ra.slots = t->tier.host_dev;
-        MLKV_LAUNCH(t, 0, (k_miss_assign<V, KV>), g, 256, 0, st, index_args(t), init_ra, keys,
-                    t->s.miss_pos, t->s.miss_slot, t->s.rank, cur, t->dstate,
-                    (unsigned long long)t->cfg.capacity, mode == MissMode::Put ? 0 : 1,
-                    (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init, (uint32_t)n);
-        MLKV_LAUNCH(t, 0, (k_miss_finish<V, KV>), g, 256, 0, st, index_args(t), init_ra,
-                    t->s.miss_pos, t->s.miss_slot, mode == MissMode::Get ? nullptr : t->s.row_of_pos,
-                    t->s.first_flag, mode == MissMode::Get ? out : nullptr, cur, t->dstate,
-                    (unsigned long long)t->cfg.capacity, (uint32_t)n);
+        MLKV_LAUNCH(t, 0, (k_miss<V, KV>), t->num_sms, kMissThreads, 0, st, index_args(t), init_ra, keys,
+                    (uint32_t)n, t->s.miss_pos, t->s.miss_slot, t->s.first_flag, t->s.rank, t->s.tile_sums,
+                    mode == MissMode::Get ? nullptr : t->s.row_of_pos, mode == MissMode::Get ? out : nullptr, cur,
+                    t->dstate, (unsigned long long)t->cfg.capacity, mode == MissMode::Put ? 0 : 1,
+                    (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init);
         return cudaGetLastError();
     }
 };
@@ -628,12 +713,6 @@ cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out
 
 cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode,
                                   float* out, cudaStream_t st, CallCounters* cur) {
-    MLKV_LAUNCH(t, 0, k_miss_flag, capped_grid(t, n, 256, MLKV_MISS_BLOCKS_PER_SM), 256, 0, st, t->index,
-                t->s.miss_pos,
-                t->s.miss_slot, t->s.first_flag, cur, (uint32_t)n);
-    cudaError_t e = launch_exclusive_scan(t, t->s.first_flag, t->s.rank, n, &cur->n_new,
-                                          &cur->n_miss, st);
-    if (e != cudaSuccess) return e;
     return dispatch_row<MissRun>(t->geom, t, keys, n, mode, out, st, cur);
 }
 

@@ -47,6 +47,7 @@ struct CallCounters {
     uint32_t n_single;   // runs of one lookup
     uint32_t short_next; // next chunk of short runs to claim (k_short's dynamic hand-out)
     uint32_t n_small;    // runs of 2 .. kSmallRun lookups (their positions in the record)
+    uint32_t bar[4];     // arrivals at the miss kernel's grid barriers
 };
 
 struct DevState {
@@ -89,7 +90,7 @@ struct Scratch {
     uint32_t* sort_offsets; // [tiles][512] output position of each tile's first element of each digit
     uint32_t* sort_dtot;    // [kSortMaxPasses][512] digit totals of each pass, zero between sorts
     uint32_t* sort_dirty;   // [tiles] 1: the first pass's counts of the tile are left to the histogram kernel
-    uint32_t* tile_sums;    // [scan tiles]
+    uint32_t* tile_sums;    // [max(scan tiles, SMs)]: per-tile sums of the dedup's scan, per-block of the miss kernel
     uint32_t* seg_start;    // [max_batch + 1] run starts in sorted order (dedup)
     uint32_t* run_row;      // [max_batch] row of each run (dedup)
     uint32_t* run_p0;       // [max_batch] first lookup position of each run (dedup)
@@ -453,8 +454,6 @@ cudaError_t launch_export(mlkv_table* t, const int64_t* keys, int64_t n, float* 
                           float* state, cudaStream_t st, CallCounters* nxt);
 
 // mlkv_sort.cu
-cudaError_t launch_exclusive_scan(mlkv_table* t, const uint32_t* in, uint32_t* out, int64_t n,
-                                  uint32_t* total, const uint32_t* enable, cudaStream_t st);
 // The first pass's counts for the probe to make (t->sort_bits rows, n lookups).
 FirstCounts first_counts(mlkv_table* t, int64_t n);
 // first_dirty: null, or FirstCounts::dirty of a probe that counted the first pass.

@@ -29,8 +29,6 @@ constexpr int kTile = kThreads * kItems;  // 4096
 static_assert(kTile == kSortTile, "the probe counts tiles of the sort's size");
 constexpr int kWarps = kThreads / 32;
 
-__device__ __forceinline__ int spad(int i) { return i + (i >> 5); }
-
 // Exclusive scan of one value per thread over a block of THREADS threads.
 template <int THREADS>
 __device__ __forceinline__ uint32_t block_exclusive_scan_n(uint32_t v, uint32_t& total) {
@@ -72,59 +70,6 @@ __device__ __forceinline__ uint32_t tiles_before(const uint32_t* __restrict__ ti
     uint32_t total;
     block_exclusive_scan(s, total);
     return total;
-}
-
-// --- generic exclusive scan -------------------------------------------------
-__global__ void __launch_bounds__(kThreads) k_scan_reduce(const uint32_t* __restrict__ in, uint32_t n,
-                                                          uint32_t* __restrict__ tile_sums,
-                                                          const uint32_t* enable) {
-    pdl_enter();
-    if (enable && *enable == 0u) return;
-    const uint32_t base = blockIdx.x * kTile;
-    uint32_t s = 0;
-#pragma unroll
-    for (int k = 0; k < kItems; ++k) {
-        const uint32_t i = base + k * kThreads + threadIdx.x;
-        if (i < n) s += in[i];
-    }
-    uint32_t total;
-    block_exclusive_scan(s, total);
-    if (threadIdx.x == 0) tile_sums[blockIdx.x] = total;
-}
-
-__global__ void __launch_bounds__(kThreads) k_scan_down(const uint32_t* in, uint32_t* out, uint32_t n,
-                                                        const uint32_t* __restrict__ tile_sums,
-                                                        uint32_t* total_out, const uint32_t* enable) {
-    pdl_enter();
-    if (enable && *enable == 0u) return;
-    __shared__ uint32_t tile[kTile + kTile / 32];
-    const uint32_t base = blockIdx.x * kTile;
-    const uint32_t prefix = tiles_before(tile_sums, blockIdx.x);
-#pragma unroll
-    for (int k = 0; k < kItems; ++k) {
-        const int i = k * kThreads + threadIdx.x;
-        tile[spad(i)] = (base + i < n) ? in[base + i] : 0u;
-    }
-    __syncthreads();
-    uint32_t local = 0;
-#pragma unroll
-    for (int k = 0; k < kItems; ++k) local += tile[spad(threadIdx.x * kItems + k)];
-    uint32_t block_total;
-    uint32_t run = block_exclusive_scan(local, block_total) + prefix;
-#pragma unroll
-    for (int k = 0; k < kItems; ++k) {
-        const int i = spad(threadIdx.x * kItems + k);
-        const uint32_t v = tile[i];
-        tile[i] = run;
-        run += v;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int k = 0; k < kItems; ++k) {
-        const int i = k * kThreads + threadIdx.x;
-        if (base + i < n) out[base + i] = tile[spad(i)];
-    }
-    if (total_out && blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) *total_out = prefix + block_total;
 }
 
 // --- radix sort ---------------------------------------------------------------
@@ -454,14 +399,6 @@ __global__ void k_dedup_out(const int64_t* __restrict__ keys, const uint32_t* __
 inline unsigned tiles(int64_t n) { return (unsigned)((n + kTile - 1) / kTile); }
 
 }  // namespace
-
-cudaError_t launch_exclusive_scan(mlkv_table* t, const uint32_t* in, uint32_t* out, int64_t n,
-                                  uint32_t* total, const uint32_t* enable, cudaStream_t st) {
-    const unsigned nt = tiles(n);
-    MLKV_LAUNCH(t, 0, k_scan_reduce, nt, kThreads, 0, st, in, (uint32_t)n, t->s.tile_sums, enable);
-    MLKV_LAUNCH(t, 0, k_scan_down, nt, kThreads, 0, st, in, out, (uint32_t)n, t->s.tile_sums, total, enable);
-    return cudaGetLastError();
-}
 
 namespace {
 // Passes and digit width for ids of `bits` bits: the fewest passes of at most

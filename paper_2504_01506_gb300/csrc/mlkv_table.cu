@@ -544,7 +544,7 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     Scratch& s = t->s;
     s.max_long = long_runs_bound(B);
     s.max_items = long_items_bound(B);
-    s.tile_sums_len = tiles_of(B) + 1;
+    s.tile_sums_len = std::max<int64_t>(tiles_of(B) + 1, t->num_sms);
     struct Piece {
         void** ptr;
         int64_t bytes;
