@@ -61,9 +61,12 @@ namespace {
 #define MLKV_CHUNK_SMALL 16
 #endif
 constexpr uint32_t kChunkLarge = 64, kChunkSmall = MLKV_CHUNK_SMALL, kSmallBatch = MLKV_SMALL_BATCH;
-// Long runs of more than kBigRun chunk sums (the hottest rows) are combined by
-// a whole 1024-thread block of k_long_combine; the rest by one lane group each.
-constexpr uint32_t kBigRun = 32;
+// Long runs of more than `big` chunk sums (the hottest rows) are combined by a
+// whole 1024-thread block of k_long_combine; the rest by one lane group each.
+// In calls of at least kSmallBatch lookups, big = kBigRunLarge (many long
+// runs: lane groups keep the SMs busy); below, kBigRunSmall (few long runs:
+// blocks sum their chunks in parallel).
+constexpr uint32_t kBigRunLarge = 32, kBigRunSmall = 4;
 
 // Tuning (set at build time): gradient rows in flight per lane group, and the
 // minimum resident blocks per SM the register allocation must allow.
@@ -131,11 +134,12 @@ struct RunArgs {
     uint32_t* long_base;   // [max_long] first chunk item
     uint32_t* item_s;      // [max_items] first sorted position of each chunk
     uint32_t* item_e;      // [max_items] one past its last
-    uint32_t* big_runs;    // [max_long] long runs of more than kBigRun chunks
+    uint32_t* big_runs;    // [max_long] long runs of more than `big` chunks
     float* partial;        // [max_items][dpad]
     uint32_t max_long;
     uint32_t max_items;
     uint32_t chunk;        // lookups per chunk of a long run (kChunkLarge or kChunkSmall)
+    uint32_t big;          // long runs of more chunks than this are combined by a whole block
     ErrSink err;
     float lr, eps;
 };
@@ -310,7 +314,7 @@ __device__ __forceinline__ void write_long_runs(const RunArgs& a, const uint32_t
         a.long_e[h0 + lane] = qe[lane];
         a.long_row[h0 + lane] = qr[lane];
         a.long_base[h0 + lane] = ib0 + excl;
-        if ((qe[lane] - qs[lane] + chunk - 1) / chunk > kBigRun) a.big_runs[atomicAdd(&a.cur->n_big, 1u)] = h0 + lane;
+        if ((qe[lane] - qs[lane] + chunk - 1) / chunk > a.big) a.big_runs[atomicAdd(&a.cur->n_big, 1u)] = h0 + lane;
     }
     for (int k = 0; k < nq; ++k) {
         const uint32_t s = qs[k], e = qe[k];
@@ -783,7 +787,7 @@ __device__ __forceinline__ void sum_partials(typename Vec<V>::T (&acc)[KV], type
     }
 }
 
-// One launch for every long run.  A run of more than kBigRun chunk sums (the
+// One launch for every long run.  A run of more than a.big chunk sums (the
 // hottest rows) takes a whole block: its lane groups split the sums in a fixed
 // way, then group 0 adds the groups' results in order.  Every other long run
 // takes one lane group, which adds its sums in order.  Then the Adagrad step.
@@ -856,7 +860,7 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
     const uint32_t gg = blockIdx.x * ngroups + group, ngg = gridDim.x * ngroups;
     for (uint32_t h = gg; h < nl; h += ngg) {  // uniform within the group
         const uint32_t m = (a.long_e[h] - a.long_s[h] + a.chunk - 1) / a.chunk;
-        if (m > kBigRun) continue;
+        if (m > a.big) continue;
         if (MLKV_CHECK && !(in_bounds(a.err, kChkCombineRun, a.long_base[h] + m, (unsigned long long)a.max_items + 1) &&
                             in_bounds(a.err, kChkCombineRow, a.long_row[h], ra.nrows)))
             continue;
@@ -885,6 +889,7 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
               t->s.long_row, t->s.long_base, t->s.item_s, t->s.item_e, t->s.big_runs, t->s.partial,
               (uint32_t)t->s.max_long,
               (uint32_t)t->s.max_items, n >= kSmallBatch ? kChunkLarge : kChunkSmall,
+              n >= kSmallBatch ? kBigRunLarge : kBigRunSmall,
               ErrSink{&t->dstate->status, t->status_dev_alias, t->dstate->chk}, t->cfg.lr, t->cfg.eps};
     // a warp per 32 positions, the windows dealt out grid-stride over at most
     // one wave of blocks

@@ -207,10 +207,10 @@ __device__ __forceinline__ void copy_row(const float* __restrict__ src, float* _
 // Tuning (set at build time): minimum resident blocks per SM for the Get
 // kernel's register allocation, and rows each lane group has in flight.
 #ifndef MLKV_GET_MIN_BLOCKS
-#define MLKV_GET_MIN_BLOCKS 6
+#define MLKV_GET_MIN_BLOCKS 8
 #endif
 #ifndef MLKV_GET_ROWS_IN_FLIGHT
-#define MLKV_GET_ROWS_IN_FLIGHT 4
+#define MLKV_GET_ROWS_IN_FLIGHT 1
 #endif
 
 template <int V, int KV, bool INSERT>
