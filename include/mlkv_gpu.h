@@ -281,7 +281,9 @@ int mlkv_apply_grad_host(mlkv_table* t, const int64_t* h_keys, int64_t n, const 
  * status (MLKV_OK when none) or MLKV_ERR_CUDA. */
 int mlkv_sync(mlkv_table* t);
 
-/* Clears the sticky device status (synchronises first). */
+/* Clears the sticky device status (synchronises first), and puts back to idle
+ * what a call that a device error cut short may have left half done (keys
+ * being inserted get no row; a later call inserts them afresh). */
 int mlkv_clear_status(mlkv_table* t);
 
 /* Number of distinct keys stored (synchronises). -1 on a null table. */
@@ -324,13 +326,18 @@ int64_t mlkv_last_unique(mlkv_table* t);
  * host allocation (cudaMalloc, cudaHostAlloc, a host-tier chunk), which then
  * returns MLKV_ERR_NOMEM; for MLKV_FAULT_COPY a host <-> device copy of a
  * *_host call, which then returns MLKV_ERR_CUDA with nothing after it
- * enqueued.  nth = 0 disarms.  One countdown per kind, shared by the whole
+ * enqueued; for MLKV_FAULT_WAIT a launch of the kernel that gives new keys
+ * their rows (launched by every call that may insert), whose grid barriers then wait for one
+ * block more than the grid has: if the call has new keys, every wait runs out
+ * (in a second or two), MLKV_ERR_TIMEOUT is recorded and the keys get no rows
+ * (mlkv_clear_status then makes the table whole again).  nth = 0 disarms.  One countdown per kind, shared by the whole
  * process.  No GPU work is affected: nothing faults on the device.  A failed
  * mlkv_open frees everything it allocated and leaves *out null; a failed
  * *_host call leaves the table usable.  Returns MLKV_ERR_INVALID for an
  * unknown kind or nth < 0. */
 #define MLKV_FAULT_ALLOC 1
 #define MLKV_FAULT_COPY 2
+#define MLKV_FAULT_WAIT 3
 int mlkv_debug_fail(int32_t kind, int64_t nth);
 
 /* Text of the last error this handle saw (static storage of the handle). */

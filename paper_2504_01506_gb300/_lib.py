@@ -47,6 +47,7 @@ EXPORTED = [
 ]
 FAULT_ALLOC = 1
 FAULT_COPY = 2
+FAULT_WAIT = 3
 STATIC_MAX_KEYS = 65536
 
 

@@ -298,7 +298,9 @@ __device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
 // the next kernel launch only after its last barrier, so every block of the
 // grid (one per SM) can become resident.  The wait is bounded: a spin that runs
 // out records MLKV_ERR_TIMEOUT and the block returns (false).
-__device__ bool grid_barrier(uint32_t* ctr, const ErrSink& err) {
+// (`extra` is 0; mlkv_debug_fail's wait injection makes it 1, a count that
+// no grid reaches, so that the wait runs out.)
+__device__ bool grid_barrier(uint32_t* ctr, uint32_t extra, const ErrSink& err) {
     __shared__ int ok;
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -306,7 +308,7 @@ __device__ bool grid_barrier(uint32_t* ctr, const ErrSink& err) {
         __threadfence();
         atomicAdd(ctr, 1u);
         uint32_t spins = 0;
-        while (ld_acquire_u32(ctr) < gridDim.x) {
+        while (ld_acquire_u32(ctr) < gridDim.x + extra) {
             if (++spins > kBarrierSpins) {
                 record_error(err, MLKV_ERR_TIMEOUT);
                 ok = 0;
@@ -368,7 +370,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
                                                        CallCounters* cur, DevState* ds,
                                                        unsigned long long capacity, int init_row,
                                                        unsigned long long seed, float lo, float span,
-                                                       float state_init) {
+                                                       float state_init, uint32_t bar_extra) {
     // waits for the kernel before it, like every kernel; lets the next one
     // launch only once the grid barriers are behind it (see grid_barrier)
     asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -385,7 +387,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
         const uint32_t p = miss_pos[i];
         if (ia.index[miss_slot[i]].aux == p) flag[p] = 1u;
     }
-    if (!grid_barrier(&cur->bar[0], ia.err)) return;
+    if (!grid_barrier(&cur->bar[0], bar_extra, ia.err)) return;
     // 2. ranks: the first occurrences at earlier positions
     const uint32_t per = (n + gridDim.x - 1) / gridDim.x;
     const uint32_t p_lo = min(n, blockIdx.x * per), p_hi = min(n, p_lo + per);
@@ -393,7 +395,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
     for (uint32_t p = p_lo + threadIdx.x; p < p_hi; p += blockDim.x) cnt += __ldcg(flag + p);
     const uint32_t mine = miss_block_sum(cnt);
     if (threadIdx.x == 0) block_sums[blockIdx.x] = mine;
-    if (!grid_barrier(&cur->bar[1], ia.err)) return;
+    if (!grid_barrier(&cur->bar[1], bar_extra, ia.err)) return;
     uint32_t b_before = 0;
     for (uint32_t b = threadIdx.x; b < blockIdx.x; b += blockDim.x) b_before += __ldcg(block_sums + b);
     uint32_t run = miss_block_sum(b_before);
@@ -406,7 +408,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
         run += tot;
     }
     if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) cur->n_new = run;  // every first occurrence
-    if (!grid_barrier(&cur->bar[2], ia.err)) return;
+    if (!grid_barrier(&cur->bar[2], bar_extra, ia.err)) return;
     // 3. rows of the first occurrences
     const int G = ra.G, glane = threadIdx.x & (G - 1);
     const uint32_t group = tid / G, ngroups = nthreads / G;
@@ -437,7 +439,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
         }
         if (glane == 0) ia.index[s].row = (uint32_t)r;
     }
-    if (!grid_barrier(&cur->bar[3], ia.err)) return;
+    if (!grid_barrier(&cur->bar[3], bar_extra, ia.err)) return;
     // 4. every missed lookup takes its key's row
     if (blockIdx.x == 0 && threadIdx.x == 0) {
         const unsigned long long nr = next + __ldcg(&cur->n_new);
@@ -625,7 +627,8 @@ struct MissRun {
                     (uint32_t)n, t->s.miss_pos, t->s.miss_slot, t->s.first_flag, t->s.rank, t->s.tile_sums,
                     mode == MissMode::Get ? nullptr : t->s.row_of_pos, mode == MissMode::Get ? out : nullptr, cur,
                     t->dstate, (unsigned long long)t->cfg.capacity, mode == MissMode::Put ? 0 : 1,
-                    (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init);
+                    (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init,
+                    take_injected_wait() ? 1u : 0u);
         return cudaGetLastError();
     }
 };
@@ -722,6 +725,19 @@ cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, const float* st
 
 cudaError_t launch_zero_counters(mlkv_table* t, CallCounters* c, cudaStream_t st) {
     MLKV_LAUNCH(t, 0, k_zero_counters, 1, 32, 0, st, c);
+    return cudaGetLastError();
+}
+
+// Slots of keys that never got a row (an insert cut short by a device error)
+// go back to idle, so that a later call inserts them afresh.
+__global__ void __launch_bounds__(256) k_reset_pending(Slot* __restrict__ index, unsigned long long nslots) {
+    for (unsigned long long s = blockIdx.x * (unsigned long long)blockDim.x + threadIdx.x; s < nslots;
+         s += (unsigned long long)gridDim.x * blockDim.x)
+        if (index[s].key != EMPTY_KEY && index[s].row == ROW_PENDING) index[s].aux = AUX_IDLE;
+}
+
+cudaError_t launch_reset_pending(mlkv_table* t, cudaStream_t st) {
+    k_reset_pending<<<(unsigned)t->num_sms * 8, 256, 0, st>>>(t->index, t->index_mask + 1);
     return cudaGetLastError();
 }
 

@@ -448,6 +448,8 @@ cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n,
 cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, const float* state, int64_t n, cudaStream_t st);
 cudaError_t launch_dump_keys(mlkv_table* t, int64_t* out, int64_t n_rows, cudaStream_t st);
 cudaError_t launch_zero_counters(mlkv_table* t, CallCounters* c, cudaStream_t st);
+// Every index slot of a key without a row goes back to idle (aux) after a call cut short.
+cudaError_t launch_reset_pending(mlkv_table* t, cudaStream_t st);
 cudaError_t launch_find(mlkv_table* t, const int64_t* keys, int64_t n, int64_t* rows,
                         cudaStream_t st, CallCounters* nxt);
 cudaError_t launch_export(mlkv_table* t, const int64_t* keys, int64_t n, float* rows,
@@ -479,7 +481,9 @@ cudaError_t launch_reduce_apply(mlkv_table* t, const float* grads, const uint32_
                                 const uint32_t* spos, int64_t n, uint32_t sent, cudaStream_t st,
                                 CallCounters* cur);
 
-// mlkv_table.cu: launch bookkeeping and optional per-kernel timing.
+// mlkv_table.cu: launch bookkeeping and optional per-kernel timing; the host
+// side of mlkv_debug_fail's wait injection (true once, for the armed launch).
+bool take_injected_wait();
 void timer_before(mlkv_table* t, int kernel_id, cudaStream_t st);
 void timer_after(mlkv_table* t, int kernel_id, cudaStream_t st);
 int persistent_blocks(mlkv_table* t, const void* kernel, int threads);

@@ -48,6 +48,7 @@ int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 // clean-up of a half-opened table) run as they would for a real failure.
 std::atomic<int64_t> g_fail_alloc{0};
 std::atomic<int64_t> g_fail_copy{0};
+std::atomic<int64_t> g_fail_wait{0};
 
 bool injected(std::atomic<int64_t>& countdown) {
     int64_t v = countdown.load();
@@ -347,6 +348,8 @@ int choose_geom(mlkv_table* t, const void* a, const void* b) {
 }  // namespace
 
 namespace mlkv {
+
+bool take_injected_wait() { return injected(g_fail_wait); }
 
 void timer_before(mlkv_table* t, int kid, cudaStream_t st) {
     KernelTimer& tm = t->timer;
@@ -853,6 +856,10 @@ int mlkv_clear_status(mlkv_table* t) {
     CK(t, cudaDeviceSynchronize());
     CK(t, cudaMemset(&t->dstate->status, 0, sizeof(uint32_t)));
     CK(t, cudaMemset(t->dstate->chk, 0, sizeof(t->dstate->chk)));
+    // a call that a device error cut short may have left keys half inserted:
+    // their slots and the first-occurrence flags go back to idle
+    CK(t, cudaMemset(t->s.first_flag, 0, (size_t)t->cfg.max_batch * 4));
+    CK(t, launch_reset_pending(t, 0));
     CK(t, cudaDeviceSynchronize());
     *(volatile uint32_t*)t->status_host = 0;
     t->last_error[0] = 0;
@@ -927,6 +934,7 @@ int mlkv_debug_fail(int32_t kind, int64_t nth) {
     switch (kind) {
         case MLKV_FAULT_ALLOC: g_fail_alloc.store(nth); return MLKV_OK;
         case MLKV_FAULT_COPY: g_fail_copy.store(nth); return MLKV_OK;
+        case MLKV_FAULT_WAIT: g_fail_wait.store(nth); return MLKV_OK;
         default: return MLKV_ERR_INVALID;
     }
 }

@@ -5,9 +5,14 @@ and copy helpers return an error without calling CUDA, so nothing faults on the
 GPU.  Checked: every allocation mlkv_open makes, failed in turn, gives
 MLKV_ERR_NOMEM, a null handle and no device memory left behind (HBM-resident
 and tiered tables); a failed staging allocation or copy of a host-buffer call
-returns its error, applies nothing and leaves the table usable.
+returns its error, applies nothing and leaves the table usable; a bounded
+wait inside a kernel (the grid barriers of the kernel that gives new keys their
+rows) made to run out returns MLKV_ERR_TIMEOUT within seconds, the context
+stays usable, and after mlkv_clear_status the same keys insert as if the failed
+call had never been made.
 """
 import ctypes
+import time
 
 import numpy as np
 import pytest
@@ -67,11 +72,12 @@ def test_every_allocation_of_open_failed_in_turn(tiered):
     assert _free_bytes(torch) == base
 
 
-def _store_and_oracle():
+def _store_and_oracle(extra_capacity=0):
     from paper_2504_01506_gb300 import EmbeddingStore
 
     cfg = W.scaled(W.tiny(), 50, 4)
-    store = EmbeddingStore(dim=cfg.dim, capacity=cfg.n_keys, max_batch=max(cfg.batch, cfg.n_keys), lr=cfg.lr,
+    store = EmbeddingStore(dim=cfg.dim, capacity=cfg.n_keys + extra_capacity, max_batch=max(cfg.batch, cfg.n_keys),
+                           lr=cfg.lr,
                            eps=cfg.eps, state_init=cfg.state_init, init_lo=cfg.init_lo, init_hi=cfg.init_hi, seed=cfg.seed,
                            device="cuda:0")
     ref = oracle.Table(cfg.dim, lr=cfg.lr, eps=cfg.eps, state_init=cfg.state_init, init_lo=cfg.init_lo,
@@ -136,4 +142,33 @@ def test_failed_staging_allocation_and_copies_leave_the_table_usable():
     short = counts <= 32
     assert_bits(host(w)[short], rw[short], "rows after a good apply")
     assert_bits(host(G)[short], rG[short], "state after a good apply")
+    store.close()
+
+
+def test_wait_that_runs_out_reports_timeout():
+    torch = torch_cuda()
+    L, lib = _lib()
+    cfg, store, ref, pre = _store_and_oracle(extra_capacity=1000)
+    new = (np.arange(600, dtype=np.int64) * 7919 + (1 << 45))[np.random.default_rng(3).permutation(600)]
+    new = np.concatenate([new, new[:100]])  # duplicates: first occurrences decide the row ids
+    lib.mlkv_debug_fail(L.FAULT_WAIT, 1)  # the next launch of the miss kernel
+    t0 = time.time()
+    store.insert(dev(new))
+    rc = store.sync()
+    took = time.time() - t0
+    lib.mlkv_debug_fail(L.FAULT_WAIT, 0)
+    assert rc == L.ERR_TIMEOUT, rc
+    assert took < 60, took
+    assert store.size() == len(pre)  # no row handed out
+    store.clear_status()
+    assert store.sync() == 0
+    # the context and the table work: the same keys insert as if the failed call never ran
+    store.insert(dev(new))
+    assert store.sync() == 0
+    ref.insert(new)
+    assert store.size() == len(pre) + 600 == ref.size()
+    assert np.array_equal(host(store.find(dev(new))), ref.find(new))
+    got = host(store.get(dev(new)))
+    want, _, _ = ref.get(new)
+    assert_bits(got, want, "Get of the keys after the timed-out insert")
     store.close()

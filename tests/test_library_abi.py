@@ -147,3 +147,4 @@ def test_fault_injection_arguments_without_gpu(lib):
     assert bound.mlkv_debug_fail(_lib.FAULT_ALLOC, 3) == _lib.OK
     assert bound.mlkv_debug_fail(_lib.FAULT_ALLOC, 0) == _lib.OK
     assert bound.mlkv_debug_fail(_lib.FAULT_COPY, 0) == _lib.OK
+    assert bound.mlkv_debug_fail(_lib.FAULT_WAIT, 0) == _lib.OK
