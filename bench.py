@@ -542,7 +542,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
     pool = base + args.warmup + steps + 1 if tiered else max(1, min(args.pool, steps + args.warmup))
     ngrad = max(1, min(args.pool, pool))
     out = torch.empty((cfg.batch, cfg.dim), dtype=torch.float32, device=dev)
-    passes = (int(cfg.n_keys).bit_length() + 7) // 8
+    passes = -(-int(cfg.n_keys).bit_length() // 9)  # the sort's passes: digits of at most 9 bits
     if kv:  # batches of Gets, then Puts
         ops_d = []
         stats = []
