@@ -857,8 +857,11 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
         }
         __syncthreads();
     }
-    const uint32_t gg = blockIdx.x * ngroups + group, ngg = gridDim.x * ngroups;
-    for (uint32_t h = gg; h < nl; h += ngg) {  // uniform within the group
+    // the other long runs: on the blocks that took no big run (all blocks when
+    // the big runs outnumber them)
+    const uint32_t b0 = nb < gridDim.x ? nb : 0u;
+    const uint32_t gg = (blockIdx.x - b0) * ngroups + group, ngg = (gridDim.x - b0) * ngroups;
+    for (uint32_t h = blockIdx.x < b0 ? nl : gg; h < nl; h += ngg) {  // uniform within the group
         const uint32_t m = (a.long_e[h] - a.long_s[h] + a.chunk - 1) / a.chunk;
         if (m > a.big) continue;
         if (MLKV_CHECK && !(in_bounds(a.err, kChkCombineRun, a.long_base[h] + m, (unsigned long long)a.max_items + 1) &&
@@ -877,6 +880,7 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
         for (int k = 0; k < KV; ++k) Vec<V>::add(acc[k], cmp[k]);  // the sum, rounded once
         adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
     }
+    release_counters(a.cur);  // the apply's last kernel
 }
 
 template <int V, int KV>

@@ -465,12 +465,13 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
                                                        CallCounters* cur, DevState* ds,
                                                        unsigned long long capacity, int init_row,
                                                        unsigned long long seed, float lo, float span,
-                                                       float state_init, uint32_t bar_extra) {
+                                                       float state_init, uint32_t bar_extra, int release) {
     // waits for the kernel before it, like every kernel; lets the next one
     // launch only once the grid barriers are behind it (see grid_barrier)
     asm volatile("griddepcontrol.wait;" ::: "memory");
     const uint32_t m = min(cur->n_miss, n);  // never more misses than lookups
     if (m == 0) {
+        if (release) release_counters(cur);
         asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
         return;
     }
@@ -553,6 +554,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
             copy_row<V, KV>(ra.slots + (size_t)(r == ROW_ABSENT ? 0 : r) * ra.stride,
                             out + (size_t)p * ra.d, ra.NV, G, glane, r == ROW_ABSENT);
     }
+    if (release) release_counters(cur);
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
@@ -751,7 +753,7 @@ struct GetRun {
 template <int V, int KV>
 struct MissRun {
     static cudaError_t run(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode, float* out,
-                           cudaStream_t st, CallCounters* cur) {
+                           cudaStream_t st, CallCounters* cur, bool release) {
         const float span = t->cfg.init_hi - t->cfg.init_lo;
         RowArgs init_ra = row_args(t);  // new rows live in the host tier when tiered
         if (t->tiered) init_ra.slots = t->tier.host_dev;
@@ -760,7 +762,7 @@ struct MissRun {
                     mode == MissMode::Get ? nullptr : t->s.row_of_pos, mode == MissMode::Get ? out : nullptr, cur,
                     t->dstate, (unsigned long long)t->cfg.capacity, mode == MissMode::Put ? 0 : 1,
                     (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init,
-                    take_injected_wait() ? 1u : 0u);
+                    take_injected_wait() ? 1u : 0u, release ? 1 : 0);
         return cudaGetLastError();
     }
 };
@@ -776,14 +778,6 @@ struct PutRun {
         return cudaGetLastError();
     }
 };
-
-// Zeroes a call's counters before its first kernel (calls captured into a
-// graph, see begin_call); a kernel rather than a memset keeps the chain of
-// programmatic launches.
-__global__ void k_zero_counters(CallCounters* c) {
-    pdl_enter();
-    if (threadIdx.x < sizeof(CallCounters) / 4) reinterpret_cast<uint32_t*>(c)[threadIdx.x] = 0u;
-}
 
 // The key of every row below n_rows, at its row: a checkpoint's keys in row
 // order (rows are dense, handed out in first-occurrence order).
@@ -847,17 +841,12 @@ cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out
 }
 
 cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode,
-                                  float* out, cudaStream_t st, CallCounters* cur) {
-    return dispatch_row<MissRun>(t->geom, t, keys, n, mode, out, st, cur);
+                                  float* out, cudaStream_t st, CallCounters* cur, bool release) {
+    return dispatch_row<MissRun>(t->geom, t, keys, n, mode, out, st, cur, release);
 }
 
 cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, const float* state, int64_t n, cudaStream_t st) {
     return dispatch_row<PutRun>(t->geom, t, vals, state, n, st);
-}
-
-cudaError_t launch_zero_counters(mlkv_table* t, CallCounters* c, cudaStream_t st) {
-    MLKV_LAUNCH(t, 0, k_zero_counters, 1, 32, 0, st, c);
-    return cudaGetLastError();
 }
 
 // Slots of keys that never got a row (an insert cut short by a device error)

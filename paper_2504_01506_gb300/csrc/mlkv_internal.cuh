@@ -48,6 +48,7 @@ struct CallCounters {
     uint32_t short_next; // next chunk of short runs to claim (k_short's dynamic hand-out)
     uint32_t n_small;    // runs of 2 .. kSmallRun lookups (their positions in the record)
     uint32_t bar[4];     // arrivals at the miss kernel's grid barriers
+    uint32_t done;       // blocks of the call's last kernel that have finished (release_counters)
 };
 
 struct DevState {
@@ -179,7 +180,6 @@ struct mlkv_table {
     int other_recorded;
     int64_t n_applies;
     int64_t launches;
-    int captured;                // some call of this table was captured into a graph (see begin_call)
     mlkv::KernelTimer timer;
     double timed_ms;
     int64_t timed_launches;
@@ -197,6 +197,21 @@ struct ErrSink {
 
 __device__ __forceinline__ void record_error(const ErrSink& e, uint32_t code) {
     if (atomicCAS(e.dev, 0u, code) == 0u && e.host) *e.host = code;
+}
+
+// Called by every block of a call's last kernel once it has read the call's
+// counters for the last time: the last block to get here zeroes them, so the
+// counters are zero when their next call starts, however that call was
+// launched (a replayed graph passes through no host code).
+__device__ __forceinline__ void release_counters(CallCounters* c) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        if (atomicAdd(&c->done, 1u) == gridDim.x - 1) {
+            uint32_t* w = reinterpret_cast<uint32_t*>(c);
+            for (unsigned i = 0; i < sizeof(CallCounters) / 4; ++i) w[i] = 0u;
+        }
+    }
 }
 
 // Bounds-checked build (-DMLKV_CHECK=1): the reduce kernels test the indices
@@ -443,11 +458,12 @@ cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool ins
                          CallCounters* nxt, uint32_t* rows_out = nullptr, const FirstCounts* fc = nullptr);
 cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out, cudaStream_t st,
                        CallCounters* cur, CallCounters* nxt);
+// release: the miss kernel is the last of the call to read its counters, and
+// zeroes them when done (release_counters).
 cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode,
-                                  float* out, cudaStream_t st, CallCounters* cur);
+                                  float* out, cudaStream_t st, CallCounters* cur, bool release);
 cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, const float* state, int64_t n, cudaStream_t st);
 cudaError_t launch_dump_keys(mlkv_table* t, int64_t* out, int64_t n_rows, cudaStream_t st);
-cudaError_t launch_zero_counters(mlkv_table* t, CallCounters* c, cudaStream_t st);
 // Every index slot of a key without a row goes back to idle (aux) after a call cut short.
 cudaError_t launch_reset_pending(mlkv_table* t, cudaStream_t st);
 cudaError_t launch_find(mlkv_table* t, const int64_t* keys, int64_t n, int64_t* rows,

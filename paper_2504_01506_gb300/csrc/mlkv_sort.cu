@@ -383,7 +383,7 @@ __global__ void __launch_bounds__(kThreads) k_seg_down(const uint32_t* __restric
 }
 
 __global__ void k_dedup_out(const int64_t* __restrict__ keys, const uint32_t* __restrict__ spos,
-                            const uint32_t* __restrict__ seg_start, const CallCounters* cur,
+                            const uint32_t* __restrict__ seg_start, CallCounters* cur,
                             int64_t* __restrict__ uniq, int32_t* __restrict__ counts, int64_t* num) {
     pdl_enter();
     const uint32_t U = cur->n_unique, nv = cur->n_valid;
@@ -394,6 +394,7 @@ __global__ void k_dedup_out(const int64_t* __restrict__ keys, const uint32_t* __
         uniq[u] = keys[spos[s]];
         counts[u] = (int32_t)(e - s);
     }
+    release_counters(cur);  // the dedup's last kernel
 }
 
 inline unsigned tiles(int64_t n) { return (unsigned)((n + kTile - 1) / kTile); }

@@ -254,12 +254,13 @@ bool capturing(cudaStream_t st) {
 }
 
 // A call's counters: one of two copies, taken in turn; each call zeroes the
-// other copy for the next one in its first kernel, so no memset is enqueued.
-// A captured graph replays a fixed sequence of calls, which may be odd in
-// number: there every call zeroes its own copy first, with a one-block kernel.
-// Replays do not pass through the host, so after the first capture the host
-// no longer knows which copy the last replay left set: from then on a call
-// launched directly zeroes its own copy first too.
+// other copy for the next one in its first kernel, and its last kernel to read
+// them zeroes its own copy when done (release_counters), so no memset is
+// enqueued and a call's copy is zero when it starts even where the host no
+// longer knows which copy is next: a captured graph replays a fixed sequence
+// of calls, which may be odd in number, without passing through the host.
+// (find and export use no counters; every other call's last kernel releases
+// them.)
 //
 // Stale-synchronous mode (staleness_bound s >= 1, Gets and applies on two
 // streams): a Get waits for every apply issued more than s applies before it,
@@ -268,11 +269,6 @@ bool capturing(cudaStream_t st) {
 // apply waits for the call before it on the other stream (the Get whose keys
 // it updates) and for the apply before it.  Applies count their own counters,
 // so a Get and an apply in flight together never share them.
-void own_counters(mlkv_table* t, CallCounters* cur, cudaStream_t st) {
-    if (capturing(st)) t->captured = 1;
-    if (t->captured) launch_zero_counters(t, cur, st);
-}
-
 CallScope begin_call(mlkv_table* t, cudaStream_t st, bool get = false) {
     const int p = t->parity;
     t->parity ^= 1;
@@ -286,7 +282,6 @@ CallScope begin_call(mlkv_table* t, cudaStream_t st, bool get = false) {
         cs.t = t;
         cs.st = st;
     }
-    own_counters(t, cs.cur, st);
     return cs;
 }
 
@@ -304,7 +299,6 @@ CallScope begin_apply(mlkv_table* t, cudaStream_t st) {
         cs.st = st;
         cs.apply = true;
     }
-    own_counters(t, cs.cur, st);
     return cs;
 }
 
@@ -632,14 +626,14 @@ int mlkv_get(mlkv_table* t, const int64_t* d_keys, int64_t n, float* d_out, void
         const uint32_t e = ++t->tier.epoch;
         const bool ins = t->cfg.insert_on_miss != 0;
         CK(t, launch_probe(t, d_keys, n, ins, MemoUse::Save, false, !ins, st, cs.cur, cs.nxt));
-        if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
+        if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur, true));
         if ((rc = tier_map(t, e, 0, n, st))) return rc;
         CK(t, launch_gather_lines(t, t->s.row_of_pos, n, d_out, st));
         return MLKV_OK;
     }
     CallScope cs = begin_call(t, st, true);
     CK(t, launch_get(t, d_keys, n, d_out, st, cs.cur, cs.nxt));
-    if (t->cfg.insert_on_miss) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Get, d_out, st, cs.cur));
+    if (t->cfg.insert_on_miss) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Get, d_out, st, cs.cur, true));
     return MLKV_OK;
 }
 
@@ -651,7 +645,7 @@ int mlkv_insert(mlkv_table* t, const int64_t* d_keys, int64_t n, void* stream) {
     if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
     CK(t, launch_probe(t, d_keys, n, true, MemoUse::None, false, false, st, cs.cur, cs.nxt));
-    CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
+    CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur, true));
     return MLKV_OK;
 }
 
@@ -665,7 +659,7 @@ static int put_rows(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
     if ((rc = wait_lookahead(t, st))) return rc;
     CallScope cs = begin_call(t, st);
     CK(t, launch_probe(t, d_keys, n, true, MemoUse::None, true, false, st, cs.cur, cs.nxt));
-    CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Put, nullptr, st, cs.cur));
+    CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Put, nullptr, st, cs.cur, true));
     if (t->tiered && (rc = tier_map(t, ++t->tier.epoch, 0, n, st))) return rc;
     CK(t, launch_put_scatter(t, d_vals, d_state, n, st));
     return MLKV_OK;
@@ -710,7 +704,7 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
     const FirstCounts fc = first_counts(t, n);
     CK(t, launch_probe(t, d_keys, n, ins, memo, false, !ins, st, cs.cur, cs.nxt, nullptr,
                        t->tiered ? nullptr : &fc));
-    if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur));
+    if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur, false));
     if (t->tiered) {
         const uint32_t e = beside ? t->tier.epoch : ++t->tier.epoch;
         if ((rc = tier_map(t, e, beside ? 1 : 0, n, st))) return rc;
@@ -860,6 +854,9 @@ int mlkv_clear_status(mlkv_table* t) {
     // their slots and the first-occurrence flags go back to idle
     CK(t, cudaMemset(t->s.first_flag, 0, (size_t)t->cfg.max_batch * 4));
     CK(t, launch_reset_pending(t, 0));
+    // ... and its counters, which its last kernel did not release
+    CK(t, cudaMemset(t->dstate->cc, 0, sizeof(t->dstate->cc)));
+    CK(t, cudaMemset(t->dstate->cca, 0, sizeof(t->dstate->cca)));
     CK(t, cudaDeviceSynchronize());
     *(volatile uint32_t*)t->status_host = 0;
     t->last_error[0] = 0;
