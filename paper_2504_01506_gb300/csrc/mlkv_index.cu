@@ -137,7 +137,6 @@ __global__ void __launch_bounds__(COUNT ? 1024 : 256) k_probe(IndexArgs ia, cons
         for (int d = threadIdx.x; d < fc.radix; d += blockDim.x) hist[d] = 0u;
         __syncthreads();
     }
-    bool missed = false;  // a lookup of this thread waits for the miss path for its row
     const uint32_t base = blockIdx.x * (blockDim.x * kProbeKeys) + threadIdx.x;
     unsigned long long k[kProbeKeys];
     uint32_t known[kProbeKeys];
@@ -168,22 +167,17 @@ __global__ void __launch_bounds__(COUNT ? 1024 : 256) k_probe(IndexArgs ia, cons
             }
         }
         row_of_pos[p] = row;
-        if (COUNT) {
-            if (row == ROW_PENDING) missed = true;
-            else atomicAdd(&hist[(row >= ROW_ABSENT ? fc.sent : row) & (uint32_t)(fc.radix - 1)], 1u);
-        }
+        // a lookup of a new key is counted by the miss kernel, once it has its row
+        if (COUNT && row != ROW_PENDING)
+            atomicAdd(&hist[(row >= ROW_ABSENT ? fc.sent : row) & (uint32_t)(fc.radix - 1)], 1u);
     }
     if (COUNT) {
-        // a tile with a miss is counted after the miss path has given its rows
-        const int dirty = __syncthreads_or(missed);
-        if (!dirty) {
-            for (int d = threadIdx.x; d < fc.radix; d += blockDim.x) {
-                const uint32_t c = hist[d];
-                fc.counts[(size_t)d * fc.ntiles + blockIdx.x] = c;
-                if (c) atomicAdd(fc.dtot + d, c);
-            }
+        __syncthreads();
+        for (int d = threadIdx.x; d < fc.radix; d += blockDim.x) {
+            const uint32_t c = hist[d];
+            fc.counts[(size_t)d * fc.ntiles + blockIdx.x] = c;
+            if (c) atomicAdd(fc.dtot + d, c);
         }
-        if (threadIdx.x == 0) fc.dirty[blockIdx.x] = dirty ? 1u : 0u;
     }
 }
 
@@ -465,7 +459,8 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
                                                        CallCounters* cur, DevState* ds,
                                                        unsigned long long capacity, int init_row,
                                                        unsigned long long seed, float lo, float span,
-                                                       float state_init, uint32_t bar_extra, int release) {
+                                                       float state_init, uint32_t bar_extra, int release,
+                                                       FirstCounts fc) {
     // waits for the kernel before it, like every kernel; lets the next one
     // launch only once the grid barriers are behind it (see grid_barrier)
     asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -478,12 +473,26 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
     using VT = typename Vec<V>::T;
     const uint32_t nthreads = gridDim.x * blockDim.x;
     const uint32_t tid = blockIdx.x * blockDim.x + threadIdx.x;
+    const int G = ra.G, glane = threadIdx.x & (G - 1);
+    const uint32_t group = tid / G, ngroups = nthreads / G;
+    // A block whose wait ran out returns at once; the first sort pass's counts
+    // (an apply's) still get its share of the missed lookups, which keep no row
+    // (the phase-4 share, so that every lookup is counted once).
+    auto give_up = [&]() {
+        if (fc.counts && glane == 0)
+            for (uint32_t i = group; i < m; i += ngroups) {
+                const uint32_t p = miss_pos[i];
+                const uint32_t dig = fc.sent & (uint32_t)(fc.radix - 1);
+                atomicAdd(&fc.counts[(size_t)dig * fc.ntiles + p / kSortTile], 1u);
+                atomicAdd(fc.dtot + dig, 1u);
+            }
+    };
     // 1. first occurrences
     for (uint32_t i = tid; i < m; i += nthreads) {
         const uint32_t p = miss_pos[i];
         if (ia.index[miss_slot[i]].aux == p) flag[p] = 1u;
     }
-    if (!grid_barrier(&cur->bar[0], bar_extra, ia.err)) return;
+    if (!grid_barrier(&cur->bar[0], bar_extra, ia.err)) return give_up();
     // 2. ranks: the first occurrences at earlier positions
     const uint32_t per = (n + gridDim.x - 1) / gridDim.x;
     const uint32_t p_lo = min(n, blockIdx.x * per), p_hi = min(n, p_lo + per);
@@ -491,7 +500,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
     for (uint32_t p = p_lo + threadIdx.x; p < p_hi; p += blockDim.x) cnt += __ldcg(flag + p);
     const uint32_t mine = miss_block_sum(cnt);
     if (threadIdx.x == 0) block_sums[blockIdx.x] = mine;
-    if (!grid_barrier(&cur->bar[1], bar_extra, ia.err)) return;
+    if (!grid_barrier(&cur->bar[1], bar_extra, ia.err)) return give_up();
     uint32_t b_before = 0;
     for (uint32_t b = threadIdx.x; b < blockIdx.x; b += blockDim.x) b_before += __ldcg(block_sums + b);
     uint32_t run = miss_block_sum(b_before);
@@ -504,10 +513,8 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
         run += tot;
     }
     if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) cur->n_new = run;  // every first occurrence
-    if (!grid_barrier(&cur->bar[2], bar_extra, ia.err)) return;
+    if (!grid_barrier(&cur->bar[2], bar_extra, ia.err)) return give_up();
     // 3. rows of the first occurrences
-    const int G = ra.G, glane = threadIdx.x & (G - 1);
-    const uint32_t group = tid / G, ngroups = nthreads / G;
     const unsigned long long next = ds->next_row;
     for (uint32_t i = group; i < m; i += ngroups) {
         const uint32_t p = miss_pos[i], s = miss_slot[i];
@@ -535,7 +542,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
         }
         if (glane == 0) ia.index[s].row = (uint32_t)r;
     }
-    if (!grid_barrier(&cur->bar[3], bar_extra, ia.err)) return;
+    if (!grid_barrier(&cur->bar[3], bar_extra, ia.err)) return give_up();
     // 4. every missed lookup takes its key's row
     if (blockIdx.x == 0 && threadIdx.x == 0) {
         const unsigned long long nr = next + __ldcg(&cur->n_new);
@@ -549,6 +556,11 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
             if (row_of_pos) row_of_pos[p] = r;
             flag[p] = 0u;
             ia.index[s].aux = AUX_IDLE;
+            if (fc.counts) {  // the first sort pass's count of this lookup's digit in its tile
+                const uint32_t dig = (r >= ROW_ABSENT ? fc.sent : r) & (uint32_t)(fc.radix - 1);
+                atomicAdd(&fc.counts[(size_t)dig * fc.ntiles + p / kSortTile], 1u);
+                atomicAdd(fc.dtot + dig, 1u);
+            }
         }
         if (out)
             copy_row<V, KV>(ra.slots + (size_t)(r == ROW_ABSENT ? 0 : r) * ra.stride,
@@ -753,7 +765,7 @@ struct GetRun {
 template <int V, int KV>
 struct MissRun {
     static cudaError_t run(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode, float* out,
-                           cudaStream_t st, CallCounters* cur, bool release) {
+                           cudaStream_t st, CallCounters* cur, bool release, const FirstCounts* fc) {
         const float span = t->cfg.init_hi - t->cfg.init_lo;
         RowArgs init_ra = row_args(t);  // new rows live in the host tier when tiered
         if (t->tiered) init_ra.slots = t->tier.host_dev;
@@ -762,7 +774,7 @@ struct MissRun {
                     mode == MissMode::Get ? nullptr : t->s.row_of_pos, mode == MissMode::Get ? out : nullptr, cur,
                     t->dstate, (unsigned long long)t->cfg.capacity, mode == MissMode::Put ? 0 : 1,
                     (unsigned long long)t->cfg.seed, t->cfg.init_lo, span, t->cfg.state_init,
-                    take_injected_wait() ? 1u : 0u, release ? 1 : 0);
+                    take_injected_wait() ? 1u : 0u, release ? 1 : 0, fc ? *fc : FirstCounts{});
         return cudaGetLastError();
     }
 };
@@ -841,8 +853,9 @@ cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out
 }
 
 cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode,
-                                  float* out, cudaStream_t st, CallCounters* cur, bool release) {
-    return dispatch_row<MissRun>(t->geom, t, keys, n, mode, out, st, cur, release);
+                                  float* out, cudaStream_t st, CallCounters* cur, bool release,
+                                  const FirstCounts* fc) {
+    return dispatch_row<MissRun>(t->geom, t, keys, n, mode, out, st, cur, release, fc);
 }
 
 cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, const float* state, int64_t n, cudaStream_t st) {

@@ -90,7 +90,6 @@ struct Scratch {
     uint32_t* sort_counts;  // [512][tiles] digit counts of a sort pass
     uint32_t* sort_offsets; // [tiles][512] output position of each tile's first element of each digit
     uint32_t* sort_dtot;    // [kSortMaxPasses][512] digit totals of each pass, zero between sorts
-    uint32_t* sort_dirty;   // [tiles] 1: the first pass's counts of the tile are left to the histogram kernel
     uint32_t* tile_sums;    // [max(scan tiles, SMs)]: per-tile sums of the dedup's scan, per-block of the miss kernel
     uint32_t* seg_start;    // [max_batch + 1] run starts in sorted order (dedup)
     uint32_t* run_row;      // [max_batch] row of each run (dedup)
@@ -434,15 +433,13 @@ struct Memo {
 };
 enum class MemoUse { None, Read, Save };
 
-// The first sort pass's digit counts, made by the apply's probe: a tile of
-// kSortTile lookups whose rows are all known after the probe (no miss) has its
-// column of counts[digit][tile] written and its counts added to the pass's
-// totals there, and dirty[tile] = 0; a tile with a miss gets dirty[tile] = 1
-// and is counted by the histogram kernel once the miss path has given rows.
+// The first sort pass's digit counts, made by the gradient apply: its probe
+// writes every tile's column of counts[digit][tile] for the lookups whose row
+// it found (and adds them to the pass's totals dtot); the miss kernel adds the
+// lookups it gave rows.  The sort's first pass then needs no histogram kernel.
 struct FirstCounts {
     uint32_t* counts;
     uint32_t* dtot;
-    uint32_t* dirty;
     uint32_t ntiles;
     int radix;       // digits of the first pass
     uint32_t sent;   // sort key of a lookup without a row
@@ -459,9 +456,11 @@ cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool ins
 cudaError_t launch_get(mlkv_table* t, const int64_t* keys, int64_t n, float* out, cudaStream_t st,
                        CallCounters* cur, CallCounters* nxt);
 // release: the miss kernel is the last of the call to read its counters, and
-// zeroes them when done (release_counters).
+// zeroes them when done (release_counters).  fc: the first sort pass's counts
+// the apply's probe made, to which the lookups given rows here are added.
 cudaError_t launch_resolve_misses(mlkv_table* t, const int64_t* keys, int64_t n, MissMode mode,
-                                  float* out, cudaStream_t st, CallCounters* cur, bool release);
+                                  float* out, cudaStream_t st, CallCounters* cur, bool release,
+                                  const FirstCounts* fc = nullptr);
 cudaError_t launch_put_scatter(mlkv_table* t, const float* vals, const float* state, int64_t n, cudaStream_t st);
 cudaError_t launch_dump_keys(mlkv_table* t, int64_t* out, int64_t n_rows, cudaStream_t st);
 // Every index slot of a key without a row goes back to idle (aux) after a call cut short.
@@ -474,9 +473,10 @@ cudaError_t launch_export(mlkv_table* t, const int64_t* keys, int64_t n, float* 
 // mlkv_sort.cu
 // The first pass's counts for the probe to make (t->sort_bits rows, n lookups).
 FirstCounts first_counts(mlkv_table* t, int64_t n);
-// first_dirty: null, or FirstCounts::dirty of a probe that counted the first pass.
+// first_counted: the first pass's counts were made by the apply's probe and
+// miss kernel (FirstCounts).
 cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow,
-                             const uint32_t** spos, const uint32_t* first_dirty = nullptr);
+                             const uint32_t** spos, bool first_counted = false);
 cudaError_t launch_segments(mlkv_table* t, const uint32_t* srow, const uint32_t* spos, int64_t n,
                             cudaStream_t st, CallCounters* cur);
 cudaError_t launch_dedup_out(mlkv_table* t, const int64_t* keys, const uint32_t* spos, int64_t n,

@@ -8,8 +8,8 @@
 //
 // Each pass is a reduce-then-scan pass over 4096-element tiles: one kernel
 // counts the digits of every tile (and the pass's digit totals; in a gradient
-// apply the probe has already counted the first pass's tiles that had no
-// miss, see FirstCounts); one kernel
+// apply the probe and the miss kernel count the first pass, see FirstCounts);
+// one kernel
 // gives every (tile, digit) the output position of its first element (the
 // elements of lower digits plus those of the digit in earlier tiles); a third
 // ranks each tile's elements stably (over rounds of 32, in order) and
@@ -107,14 +107,13 @@ __device__ __forceinline__ uint32_t digit_peers(uint32_t dig, bool valid, int bi
 // added to the pass's digit totals dtot[d].  A thread counts 16 consecutive
 // elements and adds a run of equal digits with one atomic: after the first
 // pass a hot key's lookups are consecutive, and 32 lanes adding to one counter
-// would queue.  In the first pass, a tile the probe has counted already
-// (dirty[tile] == 0) is skipped.
+// would queue.  (In a gradient apply the first pass is counted by the probe
+// and the miss kernel instead, see FirstCounts.)
 __global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restrict__ kin, uint32_t n,
                                                         uint32_t* __restrict__ counts, uint32_t* __restrict__ dtot,
                                                         uint32_t ntiles, int shift, int radix, uint32_t sent,
-                                                        int first, const uint32_t* __restrict__ dirty) {
+                                                        int first) {
     pdl_enter();
-    if (dirty && dirty[blockIdx.x] == 0u) return;  // block-uniform
     __shared__ uint32_t hist[kMaxRadix];
     for (int d = threadIdx.x; d < radix; d += kThreads) hist[d] = 0;
     __syncthreads();
@@ -413,12 +412,12 @@ void sort_geometry(int bits, int& passes, int& D) {
 FirstCounts first_counts(mlkv_table* t, int64_t n) {
     int passes, D;
     sort_geometry(t->sort_bits, passes, D);
-    return FirstCounts{t->s.sort_counts, t->s.sort_dtot, t->s.sort_dirty, tiles(n), 1 << D,
+    return FirstCounts{t->s.sort_counts, t->s.sort_dtot, tiles(n), 1 << D,
                        (uint32_t)((1ull << t->sort_bits) - 1)};
 }
 
 cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow,
-                             const uint32_t** spos, const uint32_t* first_dirty) {
+                             const uint32_t** spos, bool first_counted) {
     const int bits = t->sort_bits;
     int passes, D;
     sort_geometry(bits, passes, D);
@@ -435,8 +434,9 @@ cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const ui
     for (int p = 0; p < passes; ++p) {
         const int first = p == 0;
         uint32_t* dtot = t->s.sort_dtot + p * kMaxRadix;
-        MLKV_LAUNCH(t, 0, k_sort_hist, nt, kThreads, 0, st, kin, (uint32_t)n, counts, dtot, nt, p * D, radix,
-                    sent, first, first ? first_dirty : nullptr);
+        if (!(first && first_counted))
+            MLKV_LAUNCH(t, 0, k_sort_hist, nt, kThreads, 0, st, kin, (uint32_t)n, counts, dtot, nt, p * D, radix,
+                        sent, first);
         MLKV_LAUNCH(t, 0, k_sort_offsets, (unsigned)((radix + kWarps - 1) / kWarps), kThreads, 0, st, counts, dtot,
                     offsets, nt, radix);
         MLKV_LAUNCH(t, MLKV_K_SORT_SCATTER, k_sort_scatter, nt, kSThreads, 0, st, kin, vin, t->s.sk[out],

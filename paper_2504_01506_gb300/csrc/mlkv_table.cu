@@ -557,7 +557,6 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
         {(void**)&s.sort_counts, 512 * tiles_of(B) * 4},
         {(void**)&s.sort_offsets, 512 * tiles_of(B) * 4},
         {(void**)&s.sort_dtot, kSortMaxPasses * 512 * 4},
-        {(void**)&s.sort_dirty, tiles_of(B) * 4},
         {(void**)&s.seg_start, (B + 1) * 4},  {(void**)&s.long_s, s.max_long * 4},
         {(void**)&s.long_e, s.max_long * 4},   {(void**)&s.long_row, s.max_long * 4},
         {(void**)&s.long_base, s.max_long * 4}, {(void**)&s.item_s, s.max_items * 4},
@@ -704,7 +703,9 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
     const FirstCounts fc = first_counts(t, n);
     CK(t, launch_probe(t, d_keys, n, ins, memo, false, !ins, st, cs.cur, cs.nxt, nullptr,
                        t->tiered ? nullptr : &fc));
-    if (ins) CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur, false));
+    if (ins)
+        CK(t, launch_resolve_misses(t, d_keys, n, MissMode::Init, nullptr, st, cs.cur, false,
+                                    t->tiered ? nullptr : &fc));
     if (t->tiered) {
         const uint32_t e = beside ? t->tier.epoch : ++t->tier.epoch;
         if ((rc = tier_map(t, e, beside ? 1 : 0, n, st))) return rc;
@@ -712,7 +713,7 @@ int mlkv_apply_grad(mlkv_table* t, const int64_t* d_keys, int64_t n, const float
     }
     const uint32_t *srow, *spos;
     const uint32_t sent = (uint32_t)((1ull << t->sort_bits) - 1);  // the sort's key of a lookup without a row
-    cudaError_t err = launch_sort_rows(t, n, st, &srow, &spos, t->tiered ? nullptr : fc.dirty);
+    cudaError_t err = launch_sort_rows(t, n, st, &srow, &spos, !t->tiered);
     if (err == cudaSuccess) err = launch_reduce_apply(t, d_grads, srow, spos, n, sent, st, cs.cur);
     t->sort_bits = t->bits_rows;
     if (err != cudaSuccess) return cuda_error(t, err, "apply_grad launches");

@@ -172,3 +172,51 @@ def test_wait_that_runs_out_reports_timeout():
     want, _, _ = ref.get(new)
     assert_bits(got, want, "Get of the keys after the timed-out insert")
     store.close()
+
+
+def test_apply_whose_miss_wait_runs_out_updates_only_known_keys():
+    """An apply with new keys whose miss kernel gives up: the new keys get no
+    rows, the sort still sees every lookup (its first pass is counted by the
+    probe and the miss kernel), the known keys are updated as if the new keys'
+    lookups were not in the batch, and the status is MLKV_ERR_TIMEOUT."""
+    torch = torch_cuda()
+    L, lib = _lib()
+    cfg, store, ref, pre = _store_and_oracle(extra_capacity=2000)
+    keys = cfg.batch_keys(0).copy()
+    grads = cfg.grads(0)
+    rng = np.random.default_rng(11)
+    new = (np.arange(len(keys) // 8, dtype=np.int64) * 104729 + (1 << 46))
+    at = rng.choice(len(keys), size=len(keys) // 4, replace=False)
+    keys[at] = new[rng.integers(0, len(new), size=len(at))]  # new keys, some repeated
+    known = ~np.isin(keys, new)
+    lib.mlkv_debug_fail(L.FAULT_WAIT, 1)  # the apply's miss kernel
+    t0 = time.time()
+    store.apply_grad(dev(keys), dev(grads))
+    rc = store.sync()
+    took = time.time() - t0
+    lib.mlkv_debug_fail(L.FAULT_WAIT, 0)
+    assert rc == L.ERR_TIMEOUT, rc
+    assert took < 60, took
+    store.clear_status()
+    assert store.sync() == 0
+    assert store.size() == len(pre)  # no new key got a row
+    ref.apply_grad(keys[known], grads[known])
+    u, c = np.unique(keys[known], return_counts=True)
+    w, G = store.export(dev(u))
+    rw, rG = ref.export(u)
+    short = c <= 32
+    assert short.sum() > 100
+    assert_bits(host(w)[short], rw[short], "known keys' rows after the timed-out apply")
+    assert_bits(host(G)[short], rG[short], "known keys' state after the timed-out apply")
+    # the same apply again inserts the new keys and updates everything
+    store.apply_grad(dev(keys), dev(grads))
+    assert store.sync() == 0
+    ref.apply_grad(keys, grads)
+    assert store.size() == ref.size() == len(pre) + len(np.unique(keys[~known]))
+    u, c = np.unique(keys, return_counts=True)
+    w, G = store.export(dev(u))
+    rw, rG = ref.export(u)
+    short = c <= 32
+    assert_bits(host(w)[short], rw[short], "rows after the second apply")
+    assert_bits(host(G)[short], rG[short], "state after the second apply")
+    store.close()
