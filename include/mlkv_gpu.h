@@ -330,7 +330,9 @@ int64_t mlkv_last_unique(mlkv_table* t);
  * their rows (launched by every call that may insert), whose grid barriers then wait for one
  * block more than the grid has: if the call has new keys, every wait runs out
  * (in a second or two), MLKV_ERR_TIMEOUT is recorded and the keys get no rows
- * (mlkv_clear_status then makes the table whole again).  nth = 0 disarms.  One countdown per kind, shared by the whole
+ * (a gradient apply still updates the keys that had rows, as if the new keys'
+ * lookups were not in the batch; mlkv_clear_status then makes the table whole
+ * again).  nth = 0 disarms.  One countdown per kind, shared by the whole
  * process.  No GPU work is affected: nothing faults on the device.  A failed
  * mlkv_open frees everything it allocated and leaves *out null; a failed
  * *_host call leaves the table usable.  Returns MLKV_ERR_INVALID for an
