@@ -297,22 +297,92 @@ KERNEL_SOURCES = {1: "mlkv_index.cu", 2: "mlkv_index.cu", 3: "mlkv_sort.cu", 4: 
                   9: "mlkv_index.cu", 10: "mlkv_apply.cu", 11: "mlkv_apply.cu"}
 
 
-def traffic_for(kid: int, cfg, path=None):
-    """DRAM bytes per launch from the committed ncu summary, if it was taken on
-    this workload (name, rows and batch) and on the current source of that
-    kernel (source hash match), else None."""
-    path = path or os.path.join(ROOT, "profiles", "traffic.json")
+# ncu kernel names (demangled, without the namespace) -> kernel class
+KERNEL_PATTERNS = [("k_get_bulk<", 1), ("k_get<", 1), ("k_probe<", 2), ("k_sort_scatter", 3), ("k_short<", 4),
+                   ("k_long_sum<", 5), ("k_heads", 6), ("k_long_combine<", 7), ("k_tier_fetch", 8),
+                   ("k_put_scatter", 9), ("k_single<", 10), ("k_small<", 11)]
+TRAFFIC_PATH = os.path.join(ROOT, "profiles", "traffic.json")
+
+
+def kernel_id_of(name: str):
+    for pat, kid in KERNEL_PATTERNS:
+        if pat in name:
+            return kid
+    return None
+
+
+def source_sha(kid: int) -> str:
+    src = os.path.join(ROOT, "paper_2504_01506_gb300", "csrc", KERNEL_SOURCES[kid])
+    return hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+
+
+def traffic_for(kid: int, cfg, alg_bytes: float, path=None):
+    """DRAM bytes (read + written) of one launch of kernel class `kid` in this
+    workload, from the committed ncu record: the record must have been taken on
+    the same workload and batch size (over the full table, or one `scale` times
+    smaller, which keeps every input and output larger than L2) and on the
+    kernel's current source (hash match).  The captured bytes are scaled to
+    this launch by the algorithmic bytes (this launch's over the captured
+    launches').  None when there is no such record."""
     try:
-        with open(path) as f:
-            rec = json.load(f).get(str(kid))
+        with open(path or TRAFFIC_PATH) as f:
+            rec = json.load(f).get(cfg.name, {}).get(str(kid))
     except (OSError, ValueError):
         return None
-    if not rec or (rec.get("workload"), rec.get("rows"), rec.get("batch_lookups")) != (cfg.name, cfg.n_keys,
-                                                                                        cfg.batch):
+    if not rec or rec.get("batch_lookups") != cfg.batch or rec.get("source_sha") != source_sha(kid):
         return None
-    src = os.path.join(ROOT, "paper_2504_01506_gb300", "csrc", KERNEL_SOURCES[kid])
-    h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-    return rec.get("bytes_per_launch") if rec.get("source_sha") == h else None
+    a = rec.get("algorithmic_bytes_per_launch")
+    return rec["bytes_per_launch"] * alg_bytes / a if a else None
+
+
+def record_traffic(args, cfg, csv_path: str, path=None) -> dict:
+    """Reads an ncu CSV (--metrics dram__bytes_read.sum,dram__bytes_write.sum
+    --csv, launches of the timed steps of this same command line) and writes
+    the per-launch DRAM bytes of each kernel class it holds, beside the
+    algorithmic bytes of the same launches, into the traffic record of this
+    workload.  No GPU work."""
+    import csv
+
+    unit = {"byte": 1.0, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9}
+    per_launch = {}  # ncu launch ID -> [kernel name, bytes]
+    with open(csv_path, newline="") as f:
+        rows = [r for r in csv.reader(f) if len(r) > 10]
+    hdr = rows[0]
+    col = {h: i for i, h in enumerate(hdr)}
+    for r in rows[1:]:
+        if r[col["Metric Name"]] not in ("dram__bytes_read.sum", "dram__bytes_write.sum"):
+            continue
+        v = float(r[col["Metric Value"]].replace(",", "")) * unit[r[col["Metric Unit"]]]
+        e = per_launch.setdefault(r[col["ID"]], [r[col["Kernel Name"]], 0.0])
+        e[1] += v
+    by_kid = {}
+    for name, b in per_launch.values():
+        kid = kernel_id_of(name)
+        if kid is not None:
+            by_kid.setdefault(kid, ([], name))[0].append(b)
+    pool = max(1, min(args.pool, args.steps + args.warmup))
+    steps_idx = [(args.warmup + i) % pool for i in range(args.steps)]
+    stats = {j: batch_stats(cfg.batch_keys(j), cfg.dim) for j in set(steps_idx)}
+    passes = -(-int(cfg.n_keys).bit_length() // 9)
+    out = {}
+    for kid, (bs, name) in sorted(by_kid.items()):
+        alg = float(np.mean([kernel_bytes(stats[j], kid, passes) for j in steps_idx]))
+        out[str(kid)] = {"kernel": name.split("(")[0].replace("(anonymous namespace)::", ""),
+                         "rows": cfg.n_keys, "scale": args.scale, "batch_lookups": cfg.batch,
+                         "launches": len(bs), "bytes_per_launch": float(np.mean(bs)),
+                         "algorithmic_bytes_per_launch": alg, "source": KERNEL_SOURCES[kid],
+                         "source_sha": source_sha(kid)}
+    path = path or TRAFFIC_PATH
+    try:
+        with open(path) as f:
+            allrec = json.load(f)
+    except (OSError, ValueError):
+        allrec = {}
+    allrec[cfg.name] = out
+    with open(path, "w") as f:
+        json.dump(allrec, f, indent=1, sort_keys=True)
+        f.write("\n")
+    return out
 
 
 # --- distributed plumbing (replicas) --------------------------------------------------
@@ -724,7 +794,7 @@ def measure(args, cfg, dist, rank, local, world, dev, headline: bool, steps: int
         achieved = per_launch_bytes / (avg_ms / 1e3) / 1e9
         roofline = {"bound": "hbm", "kernel": KERNEL_NAMES[dominant], "achieved": achieved, "peak": hbm_peak,
                     "unit": "GB/s", "frac": achieved / hbm_peak, "peak_kind": peak_kind,
-                    "traffic": traffic_for(dominant, cfg), "bytes_per_launch": per_launch_bytes,
+                    "traffic": traffic_for(dominant, cfg, per_launch_bytes), "bytes_per_launch": per_launch_bytes,
                     "avg_launch_ms": avg_ms, "launches": dom_n,
                     "share_of_step": dom_ms / roof_region_ms if roof_region_ms else None,
                     "timed_over": "the timed steps run call by call right after the graph-replayed ones"
@@ -912,6 +982,10 @@ def main():
     ap.add_argument("--per-config", default="auto",
                     help="workloads measured after the headline one in the same process, comma-separated "
                          "(auto: kg,gnn,tiered after the default DLRM workload at N=1; none: no others)")
+    ap.add_argument("--traffic-record", metavar="CSV",
+                    help="write the DRAM bytes per launch in this ncu CSV (dram__bytes_read.sum and "
+                         "dram__bytes_write.sum of this command line's timed steps) into profiles/traffic.json "
+                         "and exit (no GPU work)")
     ap.add_argument("--staleness", type=int, default=0,
                     help="HBM-resident training configs: open the table with this staleness bound (>= 1; "
                          "9223372036854775807 = asynchronous) and run Gets and applies on two streams")
@@ -931,6 +1005,9 @@ def main():
         cfg = tier_scaled(cfg, args)
     if args.scale > 1:
         cfg = W.scaled(cfg, args.scale, 1)
+    if args.traffic_record:
+        print(json.dumps(record_traffic(args, cfg, args.traffic_record)))
+        return 0
     if args.impl == "reference":
         return run_reference(args, cfg)
     return run_ours(args, cfg)

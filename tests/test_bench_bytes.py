@@ -66,22 +66,62 @@ def test_every_row_byte_is_counted_once_across_the_reduce_kernels():
 
 def test_traffic_figures_only_for_their_workload_and_source(tmp_path):
     """roofline.traffic comes from a committed ncu figure only when it was taken
-    on the same workload (name, rows, batch) and the kernel's current source."""
-    import hashlib
+    on the same workload and batch size and on the kernel's current source; it
+    is scaled to the launch by the algorithmic bytes."""
     import json
 
     import workloads as W
 
-    src = os.path.join(ROOT, "paper_2504_01506_gb300", "csrc", bench.KERNEL_SOURCES[1])
-    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
     dlrm = W.dlrm()
-    rec = {"workload": "dlrm", "rows": dlrm.n_keys, "batch_lookups": dlrm.batch, "bytes_per_launch": 123.0,
-           "source_sha": sha}
+    rec = {"rows": dlrm.n_keys // 26, "scale": 26, "batch_lookups": dlrm.batch, "bytes_per_launch": 120.0,
+           "algorithmic_bytes_per_launch": 100.0, "source_sha": bench.source_sha(1)}
     path = tmp_path / "traffic.json"
-    path.write_text(json.dumps({"1": rec}))
-    assert bench.traffic_for(1, dlrm, str(path)) == 123.0
-    assert bench.traffic_for(1, W.kg(), str(path)) is None                     # another workload
-    assert bench.traffic_for(1, W.scaled(dlrm, 10, 1), str(path)) is None      # same name, smaller table
-    assert bench.traffic_for(2, dlrm, str(path)) is None                       # no figure for the kernel
-    path.write_text(json.dumps({"1": dict(rec, source_sha="0" * 16)}))
-    assert bench.traffic_for(1, dlrm, str(path)) is None                       # kernel source changed since
+    path.write_text(json.dumps({"dlrm": {"1": rec}}))
+    assert bench.traffic_for(1, dlrm, 200.0, str(path)) == 240.0               # scaled by the algorithmic bytes
+    assert bench.traffic_for(1, W.scaled(dlrm, 26, 1), 100.0, str(path)) == 120.0  # the captured case itself
+    assert bench.traffic_for(1, W.kg(), 200.0, str(path)) is None              # another workload
+    assert bench.traffic_for(1, W.scaled(dlrm, 1, 2), 200.0, str(path)) is None  # another batch size
+    assert bench.traffic_for(2, dlrm, 200.0, str(path)) is None                # no figure for the kernel
+    path.write_text(json.dumps({"dlrm": {"1": dict(rec, source_sha="0" * 16)}}))
+    assert bench.traffic_for(1, dlrm, 200.0, str(path)) is None                # kernel source changed since
+
+
+def test_traffic_record_from_an_ncu_csv(tmp_path):
+    """--traffic-record: per-launch DRAM bytes of each kernel class from ncu's
+    CSV (units converted, launches averaged), beside the algorithmic bytes of
+    the same launches' batch."""
+    import argparse
+    import json
+
+    import workloads as W
+
+    cfg = W.scaled(W.tiny(), 50, 4)
+    hdr = ["ID", "Process ID", "Process Name", "Host Name", "Kernel Name", "Context", "Stream", "Block Size",
+           "Grid Size", "Device", "CC", "Section Name", "Metric Name", "Metric Unit", "Metric Value"]
+
+    def row(i, name, metric, unit, v):
+        return [str(i), "1", "python", "h", name, "1", "7", "(256, 1, 1)", "(1, 1, 1)", "0", "10.3", "Command line",
+                metric, unit, v]
+
+    rows = [hdr,
+            row(0, "void (anonymous namespace)::k_get<4, 1, 1>(IndexArgs)", "dram__bytes_read.sum", "Mbyte", "2.5"),
+            row(0, "void (anonymous namespace)::k_get<4, 1, 1>(IndexArgs)", "dram__bytes_write.sum", "Kbyte", "500"),
+            row(0, "void (anonymous namespace)::k_get<4, 1, 1>(IndexArgs)", "gpu__time_duration.sum", "usecond", "9"),
+            row(1, "(anonymous namespace)::k_sort_scatter(const unsigned int *)", "dram__bytes_read.sum", "byte",
+                "1,000"),
+            row(1, "(anonymous namespace)::k_sort_scatter(const unsigned int *)", "dram__bytes_write.sum", "byte",
+                "0"),
+            row(2, "(anonymous namespace)::k_sort_scatter(const unsigned int *)", "dram__bytes_read.sum", "byte",
+                "3,000"),
+            row(2, "(anonymous namespace)::k_sort_scatter(const unsigned int *)", "dram__bytes_write.sum", "byte",
+                "0")]
+    csv_path = tmp_path / "launches.csv"
+    csv_path.write_text("\n".join(",".join('"%s"' % c for c in r) for r in rows) + "\n")
+    args = argparse.Namespace(pool=2, steps=1, warmup=3, scale=50)
+    out_path = tmp_path / "traffic.json"
+    out = bench.record_traffic(args, cfg, str(csv_path), str(out_path))
+    assert out["1"]["bytes_per_launch"] == 3.0e6 and out["1"]["launches"] == 1
+    assert out["3"]["bytes_per_launch"] == 2000.0 and out["3"]["launches"] == 2
+    s = bench.batch_stats(cfg.batch_keys(1), cfg.dim)  # the timed step replays batch (3 + 0) % 2
+    assert out["1"]["algorithmic_bytes_per_launch"] == bench.kernel_bytes(s, 1, 2)
+    assert json.loads(out_path.read_text())[cfg.name]["3"]["source_sha"] == bench.source_sha(3)
