@@ -367,7 +367,8 @@ def record_traffic(args, cfg, csv_path: str, path=None) -> dict:
     out = {}
     for kid, (bs, name) in sorted(by_kid.items()):
         alg = float(np.mean([kernel_bytes(stats[j], kid, passes) for j in steps_idx]))
-        out[str(kid)] = {"kernel": name.split("(")[0].replace("(anonymous namespace)::", ""),
+        short = name.split("(")[0].replace("void ", "").replace("unnamed>::", "").replace("(anonymous namespace)::", "")
+        out[str(kid)] = {"kernel": short.strip(),
                          "rows": cfg.n_keys, "scale": args.scale, "batch_lookups": cfg.batch,
                          "launches": len(bs), "bytes_per_launch": float(np.mean(bs)),
                          "algorithmic_bytes_per_launch": alg, "source": KERNEL_SOURCES[kid],
