@@ -87,6 +87,10 @@ constexpr uint32_t kBigRunLarge = 32, kBigRunSmall = 4;
 #ifndef MLKV_SINGLE_MIN_BLOCKS
 #define MLKV_SINGLE_MIN_BLOCKS 6
 #endif
+// The apply's reduce kernels on three streams (0: one after the other).
+#ifndef MLKV_REDUCE_BRANCHES
+#define MLKV_REDUCE_BRANCHES 1
+#endif
 // k_small: blocks per SM the register allocation must allow.
 #ifndef MLKV_SMALL_MIN_BLOCKS
 #define MLKV_SMALL_MIN_BLOCKS 4
@@ -905,14 +909,37 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     if (gh > cap) gh = cap;
     if (gh < 1) gh = 1;
     MLKV_LAUNCH(t, MLKV_K_SEGMENTS, k_heads, (unsigned)gh, 256, 0, st, a);
+    // The runs of one lookup, of 2 .. kSmallRun and of up to
+    // MLKV_SEQ_SEGMENT_MAX lookups, and the long runs' chunk sums touch
+    // disjoint rows and scratch: they run on three streams at once, each
+    // filling the others' tails, and join before the combine (the apply's
+    // last kernel, which releases the counters they read).
+    cudaStream_t s1 = st, s2 = st;
+    if (MLKV_REDUCE_BRANCHES) {
+        cudaError_t e;
+        if ((e = cudaEventRecord(t->ev_fork, st)) != cudaSuccess ||
+            (e = cudaStreamWaitEvent(t->branch[0], t->ev_fork, 0)) != cudaSuccess ||
+            (e = cudaStreamWaitEvent(t->branch[1], t->ev_fork, 0)) != cudaSuccess)
+            return e;
+        s1 = t->branch[0];
+        s2 = t->branch[1];
+    }
+    const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, s2, ra, a);
+    const int g2 = persistent_blocks(t, (const void*)k_small<V, KV>, 256);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, s1, ra, a);
+    const int gs = persistent_blocks(t, (const void*)k_short<V, KV>, 256);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, a);
     const int g1 = persistent_blocks(t, (const void*)k_single<V, KV>, 256);
     MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, st, ra, a);
-    const int g2 = persistent_blocks(t, (const void*)k_small<V, KV>, 256);
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, st, ra, a);
-    const int gs = persistent_blocks(t, (const void*)k_short<V, KV>, 256);
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, st, ra, a);
-    const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, st, ra, a);
+    if (MLKV_REDUCE_BRANCHES) {
+        cudaError_t e;
+        if ((e = cudaEventRecord(t->ev_join[0], s1)) != cudaSuccess ||
+            (e = cudaEventRecord(t->ev_join[1], s2)) != cudaSuccess ||
+            (e = cudaStreamWaitEvent(st, t->ev_join[0], 0)) != cudaSuccess ||
+            (e = cudaStreamWaitEvent(st, t->ev_join[1], 0)) != cudaSuccess)
+            return e;
+    }
     int big = 1024;  // the groups' (sum, compensation) pairs must fit the default 48 KB of shared memory
     while (big > 64 && (size_t)(big / t->geom.G) * 2 * t->geom.dpad * sizeof(float) > 48 * 1024) big /= 2;
     const size_t smem = (size_t)(big / t->geom.G) * 2 * t->geom.dpad * sizeof(float);

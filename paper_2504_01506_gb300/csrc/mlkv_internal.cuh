@@ -177,6 +177,12 @@ struct mlkv_table {
     cudaEvent_t* ev_apply;       // [ring]: apply number j records ev_apply[j % ring]
     cudaEvent_t ev_other;        // after the last call other than an apply
     int other_recorded;
+    // The apply's independent reduce kernels run on three streams (the call's
+    // and these two), forked after the run lists are made and joined before
+    // the long runs' combine.
+    cudaStream_t branch[2];
+    cudaEvent_t ev_fork;
+    cudaEvent_t ev_join[2];
     int64_t n_applies;
     int64_t launches;
     mlkv::KernelTimer timer;

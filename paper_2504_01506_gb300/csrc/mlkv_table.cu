@@ -412,6 +412,11 @@ int mlkv_close(mlkv_table* t) {
         delete[] t->ev_apply;
     }
     if (t->ev_other) cudaEventDestroy(t->ev_other);
+    for (int i = 0; i < 2; ++i) {
+        if (t->branch[i]) cudaStreamDestroy(t->branch[i]);
+        if (t->ev_join[i]) cudaEventDestroy(t->ev_join[i]);
+    }
+    if (t->ev_fork) cudaEventDestroy(t->ev_fork);
     if (t->tiered) {
         Tier& tr = t->tier;
         if (tr.la_stream) cudaStreamDestroy(tr.la_stream);
@@ -519,6 +524,11 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
                 return fail(MLKV_ERR_CUDA);
         if (cudaEventCreateWithFlags(&t->ev_other, cudaEventDisableTiming) != cudaSuccess) return fail(MLKV_ERR_CUDA);
     }
+    for (int i = 0; i < 2; ++i)
+        if (cudaStreamCreateWithFlags(&t->branch[i], cudaStreamNonBlocking) != cudaSuccess ||
+            cudaEventCreateWithFlags(&t->ev_join[i], cudaEventDisableTiming) != cudaSuccess)
+            return fail(MLKV_ERR_CUDA);
+    if (cudaEventCreateWithFlags(&t->ev_fork, cudaEventDisableTiming) != cudaSuccess) return fail(MLKV_ERR_CUDA);
     int64_t nslots = 64;
     while (nslots < 2 * c.capacity) nslots <<= 1;
     if (dev_alloc(&t->index, (size_t)nslots * sizeof(Slot)) != cudaSuccess) return fail(MLKV_ERR_NOMEM);
