@@ -91,6 +91,10 @@ constexpr uint32_t kBigRunLarge = 32, kBigRunSmall = 4;
 #ifndef MLKV_REDUCE_BRANCHES
 #define MLKV_REDUCE_BRANCHES 1
 #endif
+// k_single on at most this many blocks per SM (0: as many as fit).
+#ifndef MLKV_SINGLE_PER_SM
+#define MLKV_SINGLE_PER_SM 0
+#endif
 // k_small: blocks per SM the register allocation must allow.
 #ifndef MLKV_SMALL_MIN_BLOCKS
 #define MLKV_SMALL_MIN_BLOCKS 4
@@ -146,6 +150,7 @@ struct RunArgs {
     uint32_t big;          // long runs of more chunks than this are combined by a whole block
     ErrSink err;
     float lr, eps;
+    uint32_t release;      // non-zero in the apply's last kernels: the blocks of all of them (release_counters)
 };
 
 __device__ __forceinline__ unsigned group_mask(int G, int gid) {
@@ -607,6 +612,7 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
         if (glane == 0) c = atomicAdd(&a.cur->short_next, grab);
         base = ngroups * grab + __shfl_sync(gmask, c, 0, G);
     }
+    if (a.release) release_counters(a.cur, a.release);
 }
 
 // One lane group per run of one lookup (most runs of a Zipf batch): its row,
@@ -665,6 +671,7 @@ __global__ void __launch_bounds__(256, MLKV_SINGLE_MIN_BLOCKS) k_single(RowArgs 
             adagrad_store<V, KV>(ra, m[j].x, w[j], Gs[j], acc, glane, a.lr, a.eps);
         }
     }
+    if (a.release) release_counters(a.cur, a.release);
 }
 
 // One lane group per run of 2 .. kSmallRun lookups (most runs of more than one
@@ -884,7 +891,7 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
         for (int k = 0; k < KV; ++k) Vec<V>::add(acc[k], cmp[k]);  // the sum, rounded once
         adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
     }
-    release_counters(a.cur);  // the apply's last kernel
+    if (a.release) release_counters(a.cur, a.release);
 }
 
 template <int V, int KV>
@@ -925,13 +932,29 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
         s2 = t->branch[1];
     }
     const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, s2, ra, a);
     const int g2 = persistent_blocks(t, (const void*)k_small<V, KV>, 256);
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, s1, ra, a);
     const int gs = persistent_blocks(t, (const void*)k_short<V, KV>, 256);
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, a);
-    const int g1 = persistent_blocks(t, (const void*)k_single<V, KV>, 256);
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, st, ra, a);
+    int g1 = persistent_blocks(t, (const void*)k_single<V, KV>, 256);
+    if (MLKV_SINGLE_PER_SM > 0 && g1 > MLKV_SINGLE_PER_SM * t->num_sms) g1 = MLKV_SINGLE_PER_SM * t->num_sms;
+    int big = 1024;  // the groups' (sum, compensation) pairs must fit the default 48 KB of shared memory
+    while (big > 64 && (size_t)(big / t->geom.G) * 2 * t->geom.dpad * sizeof(float) > 48 * 1024) big /= 2;
+    const size_t smem = (size_t)(big / t->geom.G) * 2 * t->geom.dpad * sizeof(float);
+    // one block per SM (a 1024-thread block fills the register file): 4,864
+    // lane groups of 32 for the ordinary long runs, 152 blocks for the big ones
+    const int gc = t->num_sms * (1024 / big);
+    // The counters are released by the apply's last kernels: the last of each
+    // stream (the combine, the runs of 5-32, the runs of one), or the combine
+    // alone when all run in stream order.
+    RunArgs last = a;
+    last.release = (uint32_t)(gc + (MLKV_REDUCE_BRANCHES ? g1 + gs : 0));
+    const RunArgs& tail = MLKV_REDUCE_BRANCHES ? last : a;
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, s2, ra, a);
+    if (MLKV_REDUCE_BRANCHES)
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), gc, big, smem, s2, ra, last,
+                               t->dstate);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, s1, ra, a);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, tail);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, st, ra, tail);
     if (MLKV_REDUCE_BRANCHES) {
         cudaError_t e;
         if ((e = cudaEventRecord(t->ev_join[0], s1)) != cudaSuccess ||
@@ -939,14 +962,10 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
             (e = cudaStreamWaitEvent(st, t->ev_join[0], 0)) != cudaSuccess ||
             (e = cudaStreamWaitEvent(st, t->ev_join[1], 0)) != cudaSuccess)
             return e;
+    } else {
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), gc, big, smem, st, ra, last,
+                               t->dstate);
     }
-    int big = 1024;  // the groups' (sum, compensation) pairs must fit the default 48 KB of shared memory
-    while (big > 64 && (size_t)(big / t->geom.G) * 2 * t->geom.dpad * sizeof(float) > 48 * 1024) big /= 2;
-    const size_t smem = (size_t)(big / t->geom.G) * 2 * t->geom.dpad * sizeof(float);
-    // one block per SM (a 1024-thread block fills the register file): 4,864
-    // lane groups of 32 for the ordinary long runs, 152 blocks for the big ones
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), t->num_sms * (1024 / big), big, smem, st, ra, a,
-                t->dstate);
     return cudaGetLastError();
 }
 

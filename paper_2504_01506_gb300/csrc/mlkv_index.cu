@@ -466,7 +466,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
     asm volatile("griddepcontrol.wait;" ::: "memory");
     const uint32_t m = min(cur->n_miss, n);  // never more misses than lookups
     if (m == 0) {
-        if (release) release_counters(cur);
+        if (release) release_counters(cur, gridDim.x);
         asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
         return;
     }
@@ -566,7 +566,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
             copy_row<V, KV>(ra.slots + (size_t)(r == ROW_ABSENT ? 0 : r) * ra.stride,
                             out + (size_t)p * ra.d, ra.NV, G, glane, r == ROW_ABSENT);
     }
-    if (release) release_counters(cur);
+    if (release) release_counters(cur, gridDim.x);
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 

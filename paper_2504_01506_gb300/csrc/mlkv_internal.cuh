@@ -177,9 +177,9 @@ struct mlkv_table {
     cudaEvent_t* ev_apply;       // [ring]: apply number j records ev_apply[j % ring]
     cudaEvent_t ev_other;        // after the last call other than an apply
     int other_recorded;
-    // The apply's independent reduce kernels run on three streams (the call's
-    // and these two), forked after the run lists are made and joined before
-    // the long runs' combine.
+    // The apply's independent reduce kernels run on the call's stream and
+    // these, forked after the run lists are made and joined before the long
+    // runs' combine.
     cudaStream_t branch[2];
     cudaEvent_t ev_fork;
     cudaEvent_t ev_join[2];
@@ -204,15 +204,16 @@ __device__ __forceinline__ void record_error(const ErrSink& e, uint32_t code) {
     if (atomicCAS(e.dev, 0u, code) == 0u && e.host) *e.host = code;
 }
 
-// Called by every block of a call's last kernel once it has read the call's
-// counters for the last time: the last block to get here zeroes them, so the
-// counters are zero when their next call starts, however that call was
-// launched (a replayed graph passes through no host code).
-__device__ __forceinline__ void release_counters(CallCounters* c) {
+// Called by every block of a call's last kernels (`total` blocks in all: one
+// kernel, or the last kernel of each of the apply's streams) once it has read
+// the call's counters for the last time: the last block to get here zeroes
+// them, so the counters are zero when their next call starts, however that
+// call was launched (a replayed graph passes through no host code).
+__device__ __forceinline__ void release_counters(CallCounters* c, uint32_t total) {
     __syncthreads();
     if (threadIdx.x == 0) {
         __threadfence();
-        if (atomicAdd(&c->done, 1u) == gridDim.x - 1) {
+        if (atomicAdd(&c->done, 1u) == total - 1) {
             uint32_t* w = reinterpret_cast<uint32_t*>(c);
             for (unsigned i = 0; i < sizeof(CallCounters) / 4; ++i) w[i] = 0u;
         }

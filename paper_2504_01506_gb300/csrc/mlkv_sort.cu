@@ -393,7 +393,7 @@ __global__ void k_dedup_out(const int64_t* __restrict__ keys, const uint32_t* __
         uniq[u] = keys[spos[s]];
         counts[u] = (int32_t)(e - s);
     }
-    release_counters(cur);  // the dedup's last kernel
+    release_counters(cur, gridDim.x);  // the dedup's last kernel
 }
 
 inline unsigned tiles(int64_t n) { return (unsigned)((n + kTile - 1) / kTile); }
