@@ -95,6 +95,21 @@ constexpr uint32_t kBigRunLarge = 32, kBigRunSmall = 4;
 #ifndef MLKV_SINGLE_PER_SM
 #define MLKV_SINGLE_PER_SM 0
 #endif
+// Launch order and block priorities of the reduce kernels (measured variants).
+// MLKV_SHORT_FIRST: the runs of 5-32 launched before those of 2-4 (0: never,
+// 1: always, 2: in calls of fewer than kSmallBatch lookups).
+#ifndef MLKV_SHORT_FIRST
+#define MLKV_SHORT_FIRST 2
+#endif
+#ifndef MLKV_PRIO_LONG
+#define MLKV_PRIO_LONG 0
+#endif
+#ifndef MLKV_PRIO_COMBINE
+#define MLKV_PRIO_COMBINE 0
+#endif
+#ifndef MLKV_PRIO_SHORT
+#define MLKV_PRIO_SHORT 0
+#endif
 // k_small: blocks per SM the register allocation must allow.
 #ifndef MLKV_SMALL_MIN_BLOCKS
 #define MLKV_SMALL_MIN_BLOCKS 4
@@ -726,6 +741,7 @@ __global__ void __launch_bounds__(256, KV >= 4 ? 2 : MLKV_SMALL_MIN_BLOCKS) k_sm
         }
         adagrad_store<V, KV>(ra, m.x, w, Gs, acc, glane, a.lr, a.eps);
     }
+    if (a.release) release_counters(a.cur, a.release);  // when it is its stream's last kernel
 }
 
 template <int V, int KV>
@@ -943,17 +959,28 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     // lane groups of 32 for the ordinary long runs, 152 blocks for the big ones
     const int gc = t->num_sms * (1024 / big);
     // The counters are released by the apply's last kernels: the last of each
-    // stream (the combine, the runs of 5-32, the runs of one), or the combine
-    // alone when all run in stream order.
+    // stream (the combine, the last of the runs of 2-4 and of 5-32, the runs
+    // of one), or the combine alone when all run in stream order.
     RunArgs last = a;
-    last.release = (uint32_t)(gc + (MLKV_REDUCE_BRANCHES ? g1 + gs : 0));
+    const bool short_first = MLKV_SHORT_FIRST == 1 || (MLKV_SHORT_FIRST == 2 && n < (int64_t)kSmallBatch);
+    last.release = (uint32_t)(gc + (MLKV_REDUCE_BRANCHES ? g1 + (short_first ? g2 : gs) : 0));
     const RunArgs& tail = MLKV_REDUCE_BRANCHES ? last : a;
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, s2, ra, a);
+    // priorities of the launches' blocks (0: none; lower is placed first)
+    const int pl = MLKV_PRIO_LONG, pc = MLKV_PRIO_COMBINE, ps = MLKV_PRIO_SHORT;
+    MLKV_LAUNCH_PERSISTENT_PRIO(pl, t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, s2, ra, a);
     if (MLKV_REDUCE_BRANCHES)
-        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), gc, big, smem, s2, ra, last,
-                               t->dstate);
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, s1, ra, a);
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, tail);
+        MLKV_LAUNCH_PERSISTENT_PRIO(pc, t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), gc, big, smem, s2, ra,
+                                    last, t->dstate);
+    if (short_first) {
+        // the runs of 5-32 (the longest per run of the three) before those of
+        // 2-4: in a small batch the runs of 5-32 would otherwise be last to
+        // start, after the runs of one had filled the SMs
+        MLKV_LAUNCH_PERSISTENT_PRIO(ps, t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, a);
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, s1, ra, tail);
+    } else {
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, s1, ra, a);
+        MLKV_LAUNCH_PERSISTENT_PRIO(ps, t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, tail);
+    }
     MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, st, ra, tail);
     if (MLKV_REDUCE_BRANCHES) {
         cudaError_t e;

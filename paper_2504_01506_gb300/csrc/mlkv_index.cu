@@ -117,19 +117,22 @@ IndexArgs index_args(mlkv_table* t) {
 // row_of_pos[p] (and the slot) for every position.  Each thread takes
 // kProbeKeys lookups spaced a block apart, so that their loads are in flight
 // together (the probe is latency-bound: a key load, then a random slot load).
-// With COUNT (the gradient apply on an HBM-resident table) a block of 1024
-// threads covers one 4096-lookup tile of the sort and also counts the first
-// sort pass's digits of its rows (see FirstCounts).
+// With CT > 0 (the gradient apply on an HBM-resident table) a block of CT
+// threads covers one tile of the sort (CT * kProbeKeys lookups: 1024 threads
+// for 4096-lookup tiles, 256 for 1024) and also counts the first sort pass's
+// digits of its rows (see FirstCounts).
 constexpr int kProbeKeys = 4;
 
-template <bool INSERT, bool COUNT>
-__global__ void __launch_bounds__(COUNT ? 1024 : 256) k_probe(IndexArgs ia, const int64_t* __restrict__ keys,
+template <bool INSERT, int CT>
+__global__ void __launch_bounds__(CT ? CT : 256) k_probe(IndexArgs ia, const int64_t* __restrict__ keys,
                                                uint32_t n, uint32_t* __restrict__ row_of_pos,
                                                uint32_t* __restrict__ slot_of_pos,
                                                uint32_t* miss_pos, uint32_t* miss_slot,
                                                CallCounters* cur, CallCounters* nxt,
                                                int report_absent, Memo memo, int memo_use, FirstCounts fc) {
-    static_assert(kProbeKeys * 1024 == kSortTile, "a counting block covers one sort tile");
+    constexpr bool COUNT = CT > 0;
+    static_assert(!COUNT || kProbeKeys * CT == kSortTile || kProbeKeys * CT == kSortTileSmall,
+                  "a counting block covers one sort tile");
     pdl_enter();
     zero_counters(nxt);
     __shared__ uint32_t hist[COUNT ? kSortMaxRadix : 1];
@@ -483,7 +486,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
             for (uint32_t i = group; i < m; i += ngroups) {
                 const uint32_t p = miss_pos[i];
                 const uint32_t dig = fc.sent & (uint32_t)(fc.radix - 1);
-                atomicAdd(&fc.counts[(size_t)dig * fc.ntiles + p / kSortTile], 1u);
+                atomicAdd(&fc.counts[(size_t)dig * fc.ntiles + (p >> fc.tile_shift)], 1u);
                 atomicAdd(fc.dtot + dig, 1u);
             }
     };
@@ -558,7 +561,7 @@ __global__ void __launch_bounds__(kMissThreads) k_miss(IndexArgs ia, RowArgs ra,
             ia.index[s].aux = AUX_IDLE;
             if (fc.counts) {  // the first sort pass's count of this lookup's digit in its tile
                 const uint32_t dig = (r >= ROW_ABSENT ? fc.sent : r) & (uint32_t)(fc.radix - 1);
-                atomicAdd(&fc.counts[(size_t)dig * fc.ntiles + p / kSortTile], 1u);
+                atomicAdd(&fc.counts[(size_t)dig * fc.ntiles + (p >> fc.tile_shift)], 1u);
                 atomicAdd(fc.dtot + dig, 1u);
             }
         }
@@ -827,22 +830,35 @@ cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool ins
     const Memo m{t->s.memo_key, t->s.memo_row};
     const int ra = report_absent ? 1 : 0;
     if (fc) {  // one block per sort tile, counting the first pass
-        const unsigned g = grid_for(n, kSortTile);
-        if (insert)
-            MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<true, true>), g, 1024, 0, st, index_args(t), keys, (uint32_t)n,
-                        rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0, m, (int)memo, *fc);
-        else
-            MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<false, true>), g, 1024, 0, st, index_args(t), keys, (uint32_t)n,
-                        rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, ra, m, (int)memo, *fc);
+        const unsigned g = grid_for(n, 1 << fc->tile_shift);
+        if (fc->tile_shift == 12) {
+            if (insert)
+                MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<true, 1024>), g, 1024, 0, st, index_args(t), keys,
+                            (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0, m,
+                            (int)memo, *fc);
+            else
+                MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<false, 1024>), g, 1024, 0, st, index_args(t), keys,
+                            (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, ra, m,
+                            (int)memo, *fc);
+        } else {
+            if (insert)
+                MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<true, 256>), g, 256, 0, st, index_args(t), keys,
+                            (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0, m,
+                            (int)memo, *fc);
+            else
+                MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<false, 256>), g, 256, 0, st, index_args(t), keys,
+                            (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, ra, m,
+                            (int)memo, *fc);
+        }
         return cudaGetLastError();
     }
     const FirstCounts none{};
     const unsigned g = grid_for(n, 256 * kProbeKeys);
     if (insert)
-        MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<true, false>), g, 256, 0, st, index_args(t), keys,
+        MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<true, 0>), g, 256, 0, st, index_args(t), keys,
                     (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0, m, (int)memo, none);
     else
-        MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<false, false>), g, 256, 0, st, index_args(t), keys,
+        MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<false, 0>), g, 256, 0, st, index_args(t), keys,
                     (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, ra, m, (int)memo, none);
     return cudaGetLastError();
 }

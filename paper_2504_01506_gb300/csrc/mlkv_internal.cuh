@@ -29,7 +29,16 @@ constexpr int PROBE_LIMIT = MLKV_PROBE_LIMIT;
 constexpr int kSortMaxPasses = 4;      // row ids have at most 31 bits
 constexpr int kSortMaxDigitBits = 9;   // radix <= 512
 constexpr int kSortMaxRadix = 1 << kSortMaxDigitBits;
-constexpr int kSortTile = 4096;        // lookups per tile of a sort pass
+constexpr int kSortTile = 4096;        // lookups per tile of a sort pass ...
+constexpr int kSortTileSmall = 1024;   // ... and in batches of fewer than kSortSmallBatch lookups
+#ifndef MLKV_SORT_SMALL_BATCH
+#define MLKV_SORT_SMALL_BATCH (1u << 19)
+#endif
+constexpr uint32_t kSortSmallBatch = MLKV_SORT_SMALL_BATCH;
+// log2 of the sort's tile for a batch of n lookups: small batches take small
+// tiles, so that a pass still spreads over the SMs (200k lookups are 49 tiles
+// of 4096 but 196 of 1024)
+inline int sort_tile_shift(int64_t n) { return n < (int64_t)kSortSmallBatch ? 10 : 12; }
 constexpr int kSmallRun = 4;           // runs of 2 .. kSmallRun lookups carry their positions in their record
 constexpr int64_t kMaxStaleness = MLKV_MAX_STALENESS;  // largest bound kept below no bound
 
@@ -87,7 +96,8 @@ struct Scratch {
     uint32_t* rank;         // [max_batch]
     uint32_t* sk[2];        // sort keys (row ids), ping-pong [max_batch]
     uint32_t* sv[2];        // sort values (positions), ping-pong [max_batch]
-    uint32_t* sort_counts;  // [512][tiles] digit counts of a sort pass
+    uint32_t* sort_counts;  // [512][tiles] digit counts of the sort's even passes ...
+    uint32_t* sort_counts2; // ... and of its odd passes (zero between sorts)
     uint32_t* sort_offsets; // [tiles][512] output position of each tile's first element of each digit
     uint32_t* sort_dtot;    // [kSortMaxPasses][512] digit totals of each pass, zero between sorts
     uint32_t* tile_sums;    // [max(scan tiles, SMs)]: per-tile sums of the dedup's scan, per-block of the miss kernel
@@ -109,6 +119,7 @@ struct Scratch {
     int64_t max_long;
     int64_t max_items;
     int64_t tile_sums_len;
+    int64_t sort_counts_bytes;
 };
 
 // Tiered store (hbm_cache_rows > 0): see mlkv_tier.cu.
@@ -450,6 +461,7 @@ struct FirstCounts {
     uint32_t ntiles;
     int radix;       // digits of the first pass
     uint32_t sent;   // sort key of a lookup without a row
+    int tile_shift;  // log2 of the sort's tile (sort_tile_shift)
 };
 
 // ---------------------------------------------------------------------------
@@ -520,31 +532,43 @@ int persistent_blocks(mlkv_table* t, const void* kernel, int threads);
 #endif
 
 namespace mlkv {
+// prio: 0, or a scheduling priority for the launch's blocks (lower is
+// placed first, as for stream priorities; kept by graph capture)
 template <typename... Params, typename... Args>
-inline void launch_kernel(bool pdl, void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+inline void launch_kernel(bool pdl, int prio, void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
                           cudaStream_t st, Args&&... args) {
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchAttribute attr[2];
+    int na = 0;
+    if (MLKV_PDL && pdl) {
+        attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[na].val.programmaticStreamSerializationAllowed = 1;
+        ++na;
+    }
+    if (prio) {
+        attr[na].id = cudaLaunchAttributePriority;
+        attr[na].val.priority = prio;
+        ++na;
+    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = block;
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
     cfg.attrs = attr;
-    cfg.numAttrs = MLKV_PDL && pdl ? 1 : 0;
+    cfg.numAttrs = na;
     cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);  // an error stays in cudaGetLastError()
 }
 }  // namespace mlkv
 
 // Launch helper: counts the launch and records timing events when asked.
-#define MLKV_LAUNCH_PDL(pdl, t, kid, kernel, grid, block, smem, stream, ...)                      \
-    do {                                                                                          \
-        mlkv::timer_before((t), (kid), (stream));                                                 \
-        mlkv::launch_kernel((pdl), kernel, dim3(grid), dim3(block), (smem), (stream), __VA_ARGS__); \
-        mlkv::timer_after((t), (kid), (stream));                                                  \
-        (t)->launches++;                                                                          \
+#define MLKV_LAUNCH_PDL_PRIO(pdl, prio, t, kid, kernel, grid, block, smem, stream, ...)                      \
+    do {                                                                                                     \
+        mlkv::timer_before((t), (kid), (stream));                                                            \
+        mlkv::launch_kernel((pdl), (prio), kernel, dim3(grid), dim3(block), (smem), (stream), __VA_ARGS__);   \
+        mlkv::timer_after((t), (kid), (stream));                                                             \
+        (t)->launches++;                                                                                     \
     } while (0)
+#define MLKV_LAUNCH_PDL(pdl, ...) MLKV_LAUNCH_PDL_PRIO(pdl, 0, __VA_ARGS__)
 #define MLKV_LAUNCH(...) MLKV_LAUNCH_PDL(true, __VA_ARGS__)
 // The persistent grids (one wave, each block a fixed share of the work) may
 // start as the kernel before them drains too; -DMLKV_PDL_PERSISTENT=0 makes
@@ -553,3 +577,4 @@ inline void launch_kernel(bool pdl, void (*kernel)(Params...), dim3 grid, dim3 b
 #define MLKV_PDL_PERSISTENT 1
 #endif
 #define MLKV_LAUNCH_PERSISTENT(...) MLKV_LAUNCH_PDL(MLKV_PDL_PERSISTENT != 0, __VA_ARGS__)
+#define MLKV_LAUNCH_PERSISTENT_PRIO(prio, ...) MLKV_LAUNCH_PDL_PRIO(MLKV_PDL_PERSISTENT != 0, prio, __VA_ARGS__)

@@ -6,27 +6,33 @@
 // 40-bit keys), and the sorted order visits rows in memory order.  An absent
 // lookup is given the all-ones digit pattern and sorts last.
 //
-// Each pass is a reduce-then-scan pass over 4096-element tiles: one kernel
-// counts the digits of every tile (and the pass's digit totals; in a gradient
-// apply the probe and the miss kernel count the first pass, see FirstCounts);
-// one kernel
-// gives every (tile, digit) the output position of its first element (the
-// elements of lower digits plus those of the digit in earlier tiles); a third
-// ranks each tile's elements stably (over rounds of 32, in order) and
-// scatters them.  No block waits on another, so a pass costs the same when
-// the sort shares the GPU with other kernels.  (A single-pass decoupled
-// look-back sort was slower here: a batch is about one wave of tiles, and
-// the chain of tiles that know their prefix grows one window per round trip.)
+// Each pass is a reduce-then-scan pass over tiles of 4096 elements (1024 in
+// batches of fewer than kSortSmallBatch lookups, which would otherwise cover a
+// fraction of the SMs): the digit counts of every tile and the pass's digit
+// totals come first; one kernel gives every (tile, digit) the output position
+// of its first element (the elements of lower digits plus those of the digit
+// in earlier tiles); a second ranks each tile's elements stably (over rounds
+// of 32, in order) and scatters them.  The counts of the first pass are made
+// by a histogram kernel, or in a gradient apply by the probe and the miss
+// kernel (FirstCounts); those of every later pass by the scatter before it,
+// which knows the tile each element lands in and adds the element's next digit
+// to that tile's count (one add per run of equal targets in a warp), so no
+// pass after the first reads its input twice.  No block waits on another, so
+// a pass costs the same when the sort shares the GPU with other kernels.  (A
+// single-pass decoupled look-back sort was slower here: a batch is about one
+// wave of tiles, and the chain of tiles that know their prefix grows one
+// window per round trip.)
 #include "mlkv_internal.cuh"
 
 namespace mlkv {
 
 namespace {
 
+// the tiles of the segment scan (k_seg_*), and the block of the histogram and
+// offsets kernels
 constexpr int kThreads = 256;
 constexpr int kItems = 16;
 constexpr int kTile = kThreads * kItems;  // 4096
-static_assert(kTile == kSortTile, "the probe counts tiles of the sort's size");
 constexpr int kWarps = kThreads / 32;
 
 // Exclusive scan of one value per thread over a block of THREADS threads.
@@ -104,22 +110,23 @@ __device__ __forceinline__ uint32_t digit_peers(uint32_t dig, bool valid, int bi
 }
 
 // Digit counts of one tile, written to column `tile` of counts[d][tile], and
-// added to the pass's digit totals dtot[d].  A thread counts 16 consecutive
-// elements and adds a run of equal digits with one atomic: after the first
-// pass a hot key's lookups are consecutive, and 32 lanes adding to one counter
-// would queue.  (In a gradient apply the first pass is counted by the probe
-// and the miss kernel instead, see FirstCounts.)
+// added to the pass's digit totals dtot[d]: the first pass of a sort whose
+// counts the probe did not make.  A thread counts consecutive elements and
+// adds a run of equal digits with one atomic.
+template <int TILE>
 __global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restrict__ kin, uint32_t n,
                                                         uint32_t* __restrict__ counts, uint32_t* __restrict__ dtot,
                                                         uint32_t ntiles, int shift, int radix, uint32_t sent,
                                                         int first) {
+    constexpr int kItems = TILE / kThreads;
+    static_assert(kItems % 4 == 0, "whole 16-byte loads");
     pdl_enter();
     __shared__ uint32_t hist[kMaxRadix];
     for (int d = threadIdx.x; d < radix; d += kThreads) hist[d] = 0;
     __syncthreads();
-    const uint32_t i0 = blockIdx.x * kTile + threadIdx.x * kItems;
+    const uint32_t i0 = blockIdx.x * TILE + threadIdx.x * kItems;
     uint32_t key[kItems];
-    if (i0 + kItems <= n) {  // 16 consecutive keys, 16-byte aligned
+    if (i0 + kItems <= n) {  // consecutive keys, 16-byte aligned
         const uint4* src = reinterpret_cast<const uint4*>(kin + i0);
 #pragma unroll
         for (int q = 0; q < kItems / 4; ++q) {
@@ -156,31 +163,45 @@ __global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restri
 
 // Output position of the first element of every (tile, digit): the elements
 // of all lower digits, plus those of digit d in earlier tiles; written to
-// offsets[tile][d].  Each block first scans the pass's digit totals (all of
-// them, two per thread) for the elements of the lower digits; then a warp per
-// digit scans the digit's counts over the tiles, 32 tiles a round, with the
-// loads of 16 rounds issued together (every tile of a batch of up to 2M
-// lookups in one round trip).
-__global__ void __launch_bounds__(kThreads) k_sort_offsets(const uint32_t* __restrict__ counts,
-                                                           const uint32_t* __restrict__ dtot,
-                                                           uint32_t* __restrict__ offsets, uint32_t ntiles,
-                                                           int radix) {
+// offsets[tile][d].  Each block of OT
+// threads first scans the pass's digit totals (all of them) for the elements
+// of the lower digits; then a warp per digit scans the digit's counts over the
+// tiles, 32 tiles a round, with the loads of 16 rounds issued together (every
+// tile of a batch of up to 2M lookups in one round trip).
+#ifndef MLKV_OFFSETS_THREADS
+#define MLKV_OFFSETS_THREADS 256
+#endif
+constexpr int kOThreads = MLKV_OFFSETS_THREADS;
+#ifndef MLKV_OFFSETS_PDL
+#define MLKV_OFFSETS_PDL 0
+#endif
+__global__ void __launch_bounds__(kOThreads) k_sort_offsets(const uint32_t* __restrict__ counts,
+                                                            const uint32_t* __restrict__ dtot,
+                                                            uint32_t* __restrict__ offsets, uint32_t ntiles,
+                                                            int radix) {
     pdl_enter();
-    static_assert(2 * kThreads == kMaxRadix, "two digit totals per thread");
+    constexpr int kPer = kMaxRadix / kOThreads;  // digit totals per thread
     constexpr int kRounds = 16;
     __shared__ uint32_t lower[kMaxRadix];  // elements of the digits below each digit
     {
-        const int i = 2 * threadIdx.x;
-        const uint32_t a = i < radix ? __ldg(dtot + i) : 0u;
-        const uint32_t b = i + 1 < radix ? __ldg(dtot + i + 1) : 0u;
+        const int i0 = kPer * threadIdx.x;
+        uint32_t v[kPer], sum = 0;
+#pragma unroll
+        for (int k = 0; k < kPer; ++k) {
+            v[k] = i0 + k < radix ? __ldg(dtot + i0 + k) : 0u;
+            sum += v[k];
+        }
         uint32_t total;
-        const uint32_t ex = block_exclusive_scan(a + b, total);
-        lower[i] = ex;
-        lower[i + 1] = ex + a;
+        uint32_t ex = block_exclusive_scan_n<kOThreads>(sum, total);
+#pragma unroll
+        for (int k = 0; k < kPer; ++k) {
+            lower[i0 + k] = ex;
+            ex += v[k];
+        }
     }
     __syncthreads();
     const int lane = threadIdx.x & 31;
-    const int d = blockIdx.x * kWarps + (threadIdx.x >> 5);
+    const int d = blockIdx.x * (kOThreads / 32) + (threadIdx.x >> 5);
     if (d >= radix) return;  // warp-uniform
     const uint32_t* row = counts + (size_t)d * ntiles;
     uint32_t run = lower[d];
@@ -211,43 +232,57 @@ __global__ void __launch_bounds__(kThreads) k_sort_offsets(const uint32_t* __res
 // then laid out in shared memory in sorted order and written out so that
 // consecutive threads write consecutive addresses of a digit's run (a direct
 // scatter from registers costs one L2 sector per element).  The block has
-// kSThreads threads; warp w owns elements w*kSItems*32 .. of the tile, in
-// rounds of 32 consecutive elements (more warps a tile: fewer rounds each).  An element of digit d goes to offsets[tile][d] plus its rank
-// among the tile's elements of digit d.
-#ifndef MLKV_SCATTER_THREADS
-#define MLKV_SCATTER_THREADS 512
+// THREADS threads; warp w owns elements w*kSItems*32 .. of the tile, in
+// rounds of 32 consecutive elements (more warps a tile: fewer rounds each).
+// An element of digit d goes to offsets[tile][d] plus its rank among the
+// tile's elements of digit d.  With nshift >= 0 the element's digit of the
+// next pass (bits nshift ..) is added to the count of the tile of the next
+// pass that holds its output position, ncounts[digit][dst / TILE] (zero on
+// entry), and to the next pass's digit totals ndtot.  The counts this pass's
+// offsets came from (`counts`, read by the offsets kernel, which has
+// finished) are zeroed, for the pass after next to count into.
+// threads of the scatter's block for tiles of 1024 (4 elements a thread)
+#ifndef MLKV_SCATTER_SMALL_THREADS
+#define MLKV_SCATTER_SMALL_THREADS 256
 #endif
 #ifndef MLKV_SCATTER_MIN_BLOCKS
 #define MLKV_SCATTER_MIN_BLOCKS 3
 #endif
-constexpr int kSThreads = MLKV_SCATTER_THREADS;
-constexpr int kSWarps = kSThreads / 32;
-constexpr int kSItems = kTile / kSThreads;
-__global__ void __launch_bounds__(kSThreads, kSThreads == 256 ? 3 : MLKV_SCATTER_MIN_BLOCKS) k_sort_scatter(const uint32_t* __restrict__ kin,
-                                                              const uint32_t* __restrict__ vin,
-                                                              uint32_t* __restrict__ kout,
-                                                              uint32_t* __restrict__ vout, uint32_t n,
-                                                              const uint32_t* __restrict__ offsets,
-                                                              uint32_t ntiles, int shift, int radix, uint32_t sent,
-                                                              int first, uint32_t* __restrict__ dtot) {
+template <int TILE, int THREADS>
+__global__ void __launch_bounds__(THREADS, THREADS == 512 ? MLKV_SCATTER_MIN_BLOCKS : 4) k_sort_scatter(
+    const uint32_t* __restrict__ kin, const uint32_t* __restrict__ vin, uint32_t* __restrict__ kout,
+    uint32_t* __restrict__ vout, uint32_t n, const uint32_t* __restrict__ offsets, uint32_t ntiles, int shift,
+    int radix, uint32_t sent, int first, uint32_t* __restrict__ dtot, int nshift, uint32_t* __restrict__ ncounts,
+    uint32_t* __restrict__ ndtot, uint32_t* __restrict__ counts) {
+    constexpr int kSWarps = THREADS / 32;
+    constexpr int kSItems = TILE / THREADS;
+    constexpr int kTileShift = TILE == 4096 ? 12 : 10;
+    static_assert(TILE == (1 << kTileShift), "tiles of 4096 or 1024");
     pdl_enter();
     // the pass's digit totals were read by the offsets kernel, which has
     // finished: zero them for the next sort (the totals are zero between sorts)
     if (blockIdx.x == 0)
-        for (int d = threadIdx.x; d < radix; d += kSThreads) dtot[d] = 0u;
+        for (int d = threadIdx.x; d < radix; d += THREADS) dtot[d] = 0u;
+    // ... and this tile's column of the counts (radix x ntiles, a column a block)
+    for (int d = threadIdx.x; d < radix; d += THREADS) counts[(size_t)d * ntiles + blockIdx.x] = 0u;
     // the per-warp digit counts, then (once every position is known) the sorted tile
-    __shared__ uint32_t pool[2 * kTile];
-    static_assert(kSWarps * kMaxRadix <= 2 * kTile, "counts fit the tile buffer");
-    uint32_t (*wcnt)[kMaxRadix] = reinterpret_cast<uint32_t (*)[kMaxRadix]>(pool);
+    __shared__ uint32_t pool[2 * TILE];
+    constexpr bool kShare = kSWarps * kMaxRadix <= 2 * TILE;  // the counts fit the tile buffer
+    __shared__ uint32_t wpool[kShare ? 1 : kSWarps * kMaxRadix];
+    uint32_t (*wcnt)[kMaxRadix] = reinterpret_cast<uint32_t (*)[kMaxRadix]>(kShare ? pool : wpool);
     uint32_t* skey = pool;
-    uint32_t* sval = pool + kTile;
+    uint32_t* sval = pool + TILE;
     __shared__ uint32_t gbase[kMaxRadix];   // output position of the tile's first element of each digit
     __shared__ uint32_t lbase[kMaxRadix];   // position in the sorted tile of its first element of each digit
+    __shared__ uint32_t ntot[kMaxRadix];    // the tile's elements of each digit of the next pass
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    for (int i = threadIdx.x; i < kSWarps * kMaxRadix; i += kSThreads) (&wcnt[0][0])[i] = 0;
-    for (int d = threadIdx.x; d < radix; d += kSThreads) gbase[d] = offsets[(size_t)blockIdx.x * radix + d];
+    for (int i = threadIdx.x; i < kSWarps * kMaxRadix; i += THREADS) (&wcnt[0][0])[i] = 0;
+    for (int d = threadIdx.x; d < radix; d += THREADS) {
+        gbase[d] = offsets[(size_t)blockIdx.x * radix + d];
+        ntot[d] = 0u;
+    }
     __syncthreads();
-    const uint32_t tile0 = blockIdx.x * kTile;
+    const uint32_t tile0 = blockIdx.x * TILE;
     const uint32_t base = tile0 + w * (kSItems * 32);
     const int digit_bits = __ffs(radix) - 1;
     const uint32_t lt = lanemask_lt();
@@ -274,10 +309,11 @@ __global__ void __launch_bounds__(kSThreads, kSThreads == 256 ? 3 : MLKV_SCATTER
     __syncthreads();
     // per digit: exclusive prefix over the warps; per tile: exclusive prefix
     // over the digits (thread t owns digits t*dpt .. t*dpt+dpt-1, in order)
-    const int dpt = radix > kSThreads ? radix / kSThreads : 1;
-    uint32_t tot[kMaxRadix / kSThreads], mine = 0;
+    constexpr int kDpt = kMaxRadix > THREADS ? kMaxRadix / THREADS : 1;
+    const int dpt = radix > THREADS ? radix / THREADS : 1;
+    uint32_t tot[kDpt], mine = 0;
 #pragma unroll
-    for (int j = 0; j < kMaxRadix / kSThreads; ++j) {
+    for (int j = 0; j < kDpt; ++j) {
         const int d = threadIdx.x * dpt + j;
         tot[j] = 0;
         if (j >= dpt || d >= radix) continue;
@@ -290,9 +326,9 @@ __global__ void __launch_bounds__(kSThreads, kSThreads == 256 ? 3 : MLKV_SCATTER
         mine += tot[j];
     }
     uint32_t all;
-    uint32_t run = block_exclusive_scan_n<kSThreads>(mine, all);
+    uint32_t run = block_exclusive_scan_n<THREADS>(mine, all);
 #pragma unroll
-    for (int j = 0; j < kMaxRadix / kSThreads; ++j) {
+    for (int j = 0; j < kDpt; ++j) {
         const int d = threadIdx.x * dpt + j;
         if (j >= dpt || d >= radix) continue;
         lbase[d] = run;
@@ -313,13 +349,48 @@ __global__ void __launch_bounds__(kSThreads, kSThreads == 256 ? 3 : MLKV_SCATTER
         sval[rnk[r]] = val[r];
     }
     __syncthreads();
-    const uint32_t cnt = n - tile0 < (uint32_t)kTile ? n - tile0 : (uint32_t)kTile;
-    for (uint32_t l = threadIdx.x; l < cnt; l += kSThreads) {
-        const uint32_t k = skey[l];
-        const uint32_t dig = (k >> shift) & (radix - 1);
-        const uint32_t dst = gbase[dig] + (l - lbase[dig]);
-        kout[dst] = k;
-        vout[dst] = sval[l];
+    const uint32_t cnt = n - tile0 < (uint32_t)TILE ? n - tile0 : (uint32_t)TILE;
+    if (nshift < 0) {
+        for (uint32_t l = threadIdx.x; l < cnt; l += THREADS) {
+            const uint32_t k = skey[l];
+            const uint32_t dig = (k >> shift) & (radix - 1);
+            const uint32_t dst = gbase[dig] + (l - lbase[dig]);
+            kout[dst] = k;
+            vout[dst] = sval[l];
+        }
+        return;
+    }
+    // every lane of the warp takes part in each round (the last may be partial)
+    for (uint32_t l0 = threadIdx.x - lane; l0 < cnt; l0 += THREADS) {
+        const uint32_t l = l0 + lane;
+        const bool valid = l < cnt;
+        uint32_t target = 0xFFFFFFFFu, e = 0;
+        if (valid) {
+            const uint32_t k = skey[l];
+            const uint32_t dig = (k >> shift) & (radix - 1);
+            const uint32_t dst = gbase[dig] + (l - lbase[dig]);
+            kout[dst] = k;
+            vout[dst] = sval[l];
+            e = (k >> nshift) & (radix - 1);
+            target = e * ntiles + (dst >> kTileShift);
+        }
+        // consecutive lanes with one target (a hot row's lookups, a digit's
+        // run within one tile) add their count once, from the run's first lane
+        const uint32_t prev = __shfl_up_sync(0xffffffffu, target, 1);
+        const bool head = valid && (lane == 0 || prev != target);
+        const uint32_t heads = __ballot_sync(0xffffffffu, head);
+        const uint32_t nvalid = __popc(__ballot_sync(0xffffffffu, valid));
+        if (head) {
+            const uint32_t later = heads & ~((2u << lane) - 1u);
+            const uint32_t len = (later ? (uint32_t)(__ffs(later) - 1) : nvalid) - (uint32_t)lane;
+            atomicAdd(ncounts + target, len);
+            atomicAdd(&ntot[e], len);
+        }
+    }
+    __syncthreads();
+    for (int d = threadIdx.x; d < radix; d += THREADS) {
+        const uint32_t c = ntot[d];
+        if (c) atomicAdd(ndtot + d, c);
     }
 }
 
@@ -409,44 +480,71 @@ void sort_geometry(int bits, int& passes, int& D) {
 }
 }  // namespace
 
+inline unsigned sort_tiles(int64_t n) {
+    const int sh = sort_tile_shift(n);
+    return (unsigned)((n + (1 << sh) - 1) >> sh);
+}
+
 FirstCounts first_counts(mlkv_table* t, int64_t n) {
     int passes, D;
     sort_geometry(t->sort_bits, passes, D);
-    return FirstCounts{t->s.sort_counts, t->s.sort_dtot, tiles(n), 1 << D,
-                       (uint32_t)((1ull << t->sort_bits) - 1)};
+    return FirstCounts{t->s.sort_counts, t->s.sort_dtot, sort_tiles(n), 1 << D,
+                       (uint32_t)((1ull << t->sort_bits) - 1), sort_tile_shift(n)};
 }
 
-cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow,
-                             const uint32_t** spos, bool first_counted) {
-    const int bits = t->sort_bits;
-    int passes, D;
-    sort_geometry(bits, passes, D);
+namespace {
+template <int TILE, int THREADS>
+void sort_passes(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow, const uint32_t** spos,
+                 bool first_counted, int passes, int D) {
     const int radix = 1 << D;
-    const uint32_t sent = (uint32_t)((1ull << bits) - 1);
-    const unsigned nt = tiles(n);
-    uint32_t* counts = t->s.sort_counts;
+    const uint32_t sent = (uint32_t)((1ull << t->sort_bits) - 1);
+    const unsigned nt = sort_tiles(n);
+    // two count buffers in turn: pass p's counts are in counts[p & 1], and its
+    // scatter counts pass p + 1 into counts[(p + 1) & 1]
+    uint32_t* counts[2] = {t->s.sort_counts, t->s.sort_counts2};
     uint32_t* offsets = t->s.sort_offsets;
-    // the digit totals of every pass are zero (the arena starts zeroed; each
-    // pass's scatter zeroes its pass's totals once they are read)
+    // the digit totals of every pass, and the second count buffer, are zero
+    // between sorts (the arena starts zeroed; each pass's scatter zeroes its
+    // pass's totals and the counts its offsets came from; the first pass's
+    // counts are written whole by the probe or the histogram kernel)
     const uint32_t* kin = t->s.row_of_pos;
     const uint32_t* vin = nullptr;
     int out = 0;
     for (int p = 0; p < passes; ++p) {
         const int first = p == 0;
         uint32_t* dtot = t->s.sort_dtot + p * kMaxRadix;
-        if (!(first && first_counted))
-            MLKV_LAUNCH(t, 0, k_sort_hist, nt, kThreads, 0, st, kin, (uint32_t)n, counts, dtot, nt, p * D, radix,
-                        sent, first);
-        MLKV_LAUNCH(t, 0, k_sort_offsets, (unsigned)((radix + kWarps - 1) / kWarps), kThreads, 0, st, counts, dtot,
-                    offsets, nt, radix);
-        MLKV_LAUNCH(t, MLKV_K_SORT_SCATTER, k_sort_scatter, nt, kSThreads, 0, st, kin, vin, t->s.sk[out],
-                    t->s.sv[out], (uint32_t)n, offsets, nt, p * D, radix, sent, first, dtot);
+        if (first && !first_counted)
+            MLKV_LAUNCH(t, 0, k_sort_hist<TILE>, nt, kThreads, 0, st, kin, (uint32_t)n, counts[0], dtot, nt, 0,
+                        radix, sent, first);
+        // launched after the kernel before it has finished, not beside its
+        // drain: placed early, its few blocks landed on the SMs the scatter
+        // left room on (a tenth of them) and took twice as long
+        MLKV_LAUNCH_PDL(MLKV_OFFSETS_PDL != 0, t, 0, k_sort_offsets,
+                        (unsigned)((radix + kOThreads / 32 - 1) / (kOThreads / 32)), kOThreads, 0, st,
+                        counts[p & 1], dtot, offsets, nt, radix);
+        // every pass but the last counts the next one
+        const int nshift = p + 1 < passes ? (p + 1) * D : -1;
+        MLKV_LAUNCH(t, MLKV_K_SORT_SCATTER, (k_sort_scatter<TILE, THREADS>), nt, THREADS, 0, st, kin, vin,
+                    t->s.sk[out], t->s.sv[out], (uint32_t)n, offsets, nt, p * D, radix, sent, first, dtot, nshift,
+                    counts[(p + 1) & 1], nshift < 0 ? nullptr : t->s.sort_dtot + (p + 1) * kMaxRadix,
+                    counts[p & 1]);
         kin = t->s.sk[out];
         vin = t->s.sv[out];
         out ^= 1;
     }
     *srow = kin;
     *spos = vin;
+}
+}  // namespace
+
+cudaError_t launch_sort_rows(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** srow,
+                             const uint32_t** spos, bool first_counted) {
+    int passes, D;
+    sort_geometry(t->sort_bits, passes, D);
+    if (sort_tile_shift(n) == 12)
+        sort_passes<kSortTile, 512>(t, n, st, srow, spos, first_counted, passes, D);
+    else
+        sort_passes<kSortTileSmall, MLKV_SCATTER_SMALL_THREADS>(t, n, st, srow, spos, first_counted, passes, D);
     return cudaGetLastError();
 }
 

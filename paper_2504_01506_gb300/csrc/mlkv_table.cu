@@ -552,6 +552,9 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
     s.max_long = long_runs_bound(B);
     s.max_items = long_items_bound(B);
     s.tile_sums_len = std::max<int64_t>(tiles_of(B) + 1, t->num_sms);
+    // the sort's tiles: 4096 lookups, 1024 in batches under kSortSmallBatch
+    const int64_t sort_tiles = std::max<int64_t>(
+        tiles_of(B), (std::min<int64_t>(B, (int64_t)kSortSmallBatch - 1) + kSortTileSmall - 1) / kSortTileSmall);
     struct Piece {
         void** ptr;
         int64_t bytes;
@@ -564,8 +567,9 @@ int mlkv_open(const mlkv_config* cfg, mlkv_table** out) {
         {(void**)&s.sk[0], B * 4},          {(void**)&s.sk[1], B * 4},
         {(void**)&s.sv[0], B * 4},          {(void**)&s.sv[1], B * 4},
         {(void**)&s.tile_sums, s.tile_sums_len * 4},
-        {(void**)&s.sort_counts, 512 * tiles_of(B) * 4},
-        {(void**)&s.sort_offsets, 512 * tiles_of(B) * 4},
+        {(void**)&s.sort_counts, s.sort_counts_bytes = 512 * sort_tiles * 4},
+        {(void**)&s.sort_counts2, 512 * sort_tiles * 4},
+        {(void**)&s.sort_offsets, 512 * sort_tiles * 4},
         {(void**)&s.sort_dtot, kSortMaxPasses * 512 * 4},
         {(void**)&s.seg_start, (B + 1) * 4},  {(void**)&s.long_s, s.max_long * 4},
         {(void**)&s.long_e, s.max_long * 4},   {(void**)&s.long_row, s.max_long * 4},
@@ -868,6 +872,10 @@ int mlkv_clear_status(mlkv_table* t) {
     // ... and its counters, which its last kernel did not release
     CK(t, cudaMemset(t->dstate->cc, 0, sizeof(t->dstate->cc)));
     CK(t, cudaMemset(t->dstate->cca, 0, sizeof(t->dstate->cca)));
+    // ... and the sort's counts and digit totals, zero between sorts
+    CK(t, cudaMemset(t->s.sort_counts, 0, t->s.sort_counts_bytes));
+    CK(t, cudaMemset(t->s.sort_counts2, 0, t->s.sort_counts_bytes));
+    CK(t, cudaMemset(t->s.sort_dtot, 0, kSortMaxPasses * 512 * 4));
     CK(t, cudaDeviceSynchronize());
     *(volatile uint32_t*)t->status_host = 0;
     t->last_error[0] = 0;
