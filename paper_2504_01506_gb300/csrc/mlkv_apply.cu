@@ -110,6 +110,13 @@ constexpr uint32_t kBigRunLarge = 32, kBigRunSmall = 4;
 #ifndef MLKV_PRIO_SHORT
 #define MLKV_PRIO_SHORT 0
 #endif
+// k_long_combine's block (a big run's chunks are split over its lane groups):
+// 256 threads fit the slots that retiring blocks of the other reduce kernels
+// free, where a 1024-thread block waited for a whole SM to drain (DLRM: the
+// combine started 70 us after its chunk sums were done).
+#ifndef MLKV_COMBINE_THREADS
+#define MLKV_COMBINE_THREADS 256
+#endif
 // k_small: blocks per SM the register allocation must allow.
 #ifndef MLKV_SMALL_MIN_BLOCKS
 #define MLKV_SMALL_MIN_BLOCKS 4
@@ -952,11 +959,12 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     const int gs = persistent_blocks(t, (const void*)k_short<V, KV>, 256);
     int g1 = persistent_blocks(t, (const void*)k_single<V, KV>, 256);
     if (MLKV_SINGLE_PER_SM > 0 && g1 > MLKV_SINGLE_PER_SM * t->num_sms) g1 = MLKV_SINGLE_PER_SM * t->num_sms;
-    int big = 1024;  // the groups' (sum, compensation) pairs must fit the default 48 KB of shared memory
+    // the combine's block (MLKV_COMBINE_THREADS): the groups' (sum,
+    // compensation) pairs must fit the default 48 KB of shared memory
+    int big = MLKV_COMBINE_THREADS;
     while (big > 64 && (size_t)(big / t->geom.G) * 2 * t->geom.dpad * sizeof(float) > 48 * 1024) big /= 2;
     const size_t smem = (size_t)(big / t->geom.G) * 2 * t->geom.dpad * sizeof(float);
-    // one block per SM (a 1024-thread block fills the register file): 4,864
-    // lane groups of 32 for the ordinary long runs, 152 blocks for the big ones
+    // 1024 threads per SM: 4,864 lane groups of 32 for the ordinary long runs
     const int gc = t->num_sms * (1024 / big);
     // The counters are released by the apply's last kernels: the last of each
     // stream (the combine, the last of the runs of 2-4 and of 5-32, the runs
