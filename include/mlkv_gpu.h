@@ -300,7 +300,10 @@ int mlkv_tier_stats(mlkv_table* t, int64_t* rows_fetched, int64_t* rows_written_
 /* Per-kernel timing with CUDA events recorded on the launching stream around
  * every launch of kernel `kernel_id` (MLKV_K_*); 0 turns it off.  Read it with
  * mlkv_kernel_time, which synchronises and returns the summed milliseconds and
- * the number of timed launches since the last reset. */
+ * the number of timed launches since the last reset.  While it is on, a
+ * gradient apply launches its reduce kernels one after another on the call's
+ * stream (otherwise they run on three streams at once), so that each timed
+ * launch's events bracket that kernel alone. */
 #define MLKV_K_GET_GATHER 1
 #define MLKV_K_PROBE 2
 #define MLKV_K_SORT_SCATTER 3

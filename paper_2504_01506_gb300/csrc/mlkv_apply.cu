@@ -945,7 +945,11 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     // filling the others' tails, and join before the combine (the apply's
     // last kernel, which releases the counters they read).
     cudaStream_t s1 = st, s2 = st;
-    if (MLKV_REDUCE_BRANCHES) {
+    // While a kernel class is being timed (mlkv_time_kernel) the reduce kernels
+    // run one after another: on three streams a kernel's events would also
+    // span the time it waits for the SMs the others hold.
+    const bool branches = MLKV_REDUCE_BRANCHES && t->timer.kernel_id == 0;
+    if (branches) {
         cudaError_t e;
         if ((e = cudaEventRecord(t->ev_fork, st)) != cudaSuccess ||
             (e = cudaStreamWaitEvent(t->branch[0], t->ev_fork, 0)) != cudaSuccess ||
@@ -971,12 +975,12 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     // of one), or the combine alone when all run in stream order.
     RunArgs last = a;
     const bool short_first = MLKV_SHORT_FIRST == 1 || (MLKV_SHORT_FIRST == 2 && n < (int64_t)kSmallBatch);
-    last.release = (uint32_t)(gc + (MLKV_REDUCE_BRANCHES ? g1 + (short_first ? g2 : gs) : 0));
-    const RunArgs& tail = MLKV_REDUCE_BRANCHES ? last : a;
+    last.release = (uint32_t)(gc + (branches ? g1 + (short_first ? g2 : gs) : 0));
+    const RunArgs& tail = branches ? last : a;
     // priorities of the launches' blocks (0: none; lower is placed first)
     const int pl = MLKV_PRIO_LONG, pc = MLKV_PRIO_COMBINE, ps = MLKV_PRIO_SHORT;
     MLKV_LAUNCH_PERSISTENT_PRIO(pl, t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, s2, ra, a);
-    if (MLKV_REDUCE_BRANCHES)
+    if (branches)
         MLKV_LAUNCH_PERSISTENT_PRIO(pc, t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), gc, big, smem, s2, ra,
                                     last, t->dstate);
     if (short_first) {
@@ -990,7 +994,7 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
         MLKV_LAUNCH_PERSISTENT_PRIO(ps, t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, tail);
     }
     MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, st, ra, tail);
-    if (MLKV_REDUCE_BRANCHES) {
+    if (branches) {
         cudaError_t e;
         if ((e = cudaEventRecord(t->ev_join[0], s1)) != cudaSuccess ||
             (e = cudaEventRecord(t->ev_join[1], s2)) != cudaSuccess ||
