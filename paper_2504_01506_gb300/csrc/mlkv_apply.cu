@@ -95,20 +95,10 @@ constexpr uint32_t kBigRunLarge = 32, kBigRunSmall = 4;
 #ifndef MLKV_SINGLE_PER_SM
 #define MLKV_SINGLE_PER_SM 0
 #endif
-// Launch order and block priorities of the reduce kernels (measured variants).
-// MLKV_SHORT_FIRST: the runs of 5-32 launched before those of 2-4 (0: never,
+// Launch order of the reduce kernels.  MLKV_SHORT_FIRST: the runs of 5-32 launched before those of 2-4 (0: never,
 // 1: always, 2: in calls of fewer than kSmallBatch lookups).
 #ifndef MLKV_SHORT_FIRST
 #define MLKV_SHORT_FIRST 2
-#endif
-#ifndef MLKV_PRIO_LONG
-#define MLKV_PRIO_LONG 0
-#endif
-#ifndef MLKV_PRIO_COMBINE
-#define MLKV_PRIO_COMBINE 0
-#endif
-#ifndef MLKV_PRIO_SHORT
-#define MLKV_PRIO_SHORT 0
 #endif
 // k_long_combine's block (a big run's chunks are split over its lane groups):
 // 256 threads fit the slots that retiring blocks of the other reduce kernels
@@ -940,10 +930,10 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     if (gh < 1) gh = 1;
     MLKV_LAUNCH(t, MLKV_K_SEGMENTS, k_heads, (unsigned)gh, 256, 0, st, a);
     // The runs of one lookup, of 2 .. kSmallRun and of up to
-    // MLKV_SEQ_SEGMENT_MAX lookups, and the long runs' chunk sums touch
-    // disjoint rows and scratch: they run on three streams at once, each
-    // filling the others' tails, and join before the combine (the apply's
-    // last kernel, which releases the counters they read).
+    // MLKV_SEQ_SEGMENT_MAX lookups, and the long runs (chunk sums, then their
+    // combine) touch disjoint rows and scratch: they run on three streams at
+    // once, each filling the others' tails, and join at the end of the call;
+    // the last kernel of each stream releases the counters they read.
     cudaStream_t s1 = st, s2 = st;
     // While a kernel class is being timed (mlkv_time_kernel) the reduce kernels
     // run one after another: on three streams a kernel's events would also
@@ -977,23 +967,22 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     const bool short_first = MLKV_SHORT_FIRST == 1 || (MLKV_SHORT_FIRST == 2 && n < (int64_t)kSmallBatch);
     last.release = (uint32_t)(gc + (branches ? g1 + (short_first ? g2 : gs) : 0));
     const RunArgs& tail = branches ? last : a;
-    // priorities of the launches' blocks (0: none; lower is placed first)
-    const int pl = MLKV_PRIO_LONG, pc = MLKV_PRIO_COMBINE, ps = MLKV_PRIO_SHORT;
-    MLKV_LAUNCH_PERSISTENT_PRIO(pl, t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, s2, ra, a);
+    const cudaStream_t s_long = s2, s_single = st;
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_LONG, (k_long_sum<V, KV>), gl, 256, 0, s_long, ra, a);
     if (branches)
-        MLKV_LAUNCH_PERSISTENT_PRIO(pc, t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), gc, big, smem, s2, ra,
-                                    last, t->dstate);
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_LONG_COMBINE, (k_long_combine<V, KV>), gc, big, smem, s_long, ra, last,
+                               t->dstate);
     if (short_first) {
         // the runs of 5-32 (the longest per run of the three) before those of
         // 2-4: in a small batch the runs of 5-32 would otherwise be last to
         // start, after the runs of one had filled the SMs
-        MLKV_LAUNCH_PERSISTENT_PRIO(ps, t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, a);
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, a);
         MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, s1, ra, tail);
     } else {
         MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, s1, ra, a);
-        MLKV_LAUNCH_PERSISTENT_PRIO(ps, t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, tail);
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, tail);
     }
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, st, ra, tail);
+    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, s_single, ra, tail);
     if (branches) {
         cudaError_t e;
         if ((e = cudaEventRecord(t->ev_join[0], s1)) != cudaSuccess ||

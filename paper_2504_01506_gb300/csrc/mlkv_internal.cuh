@@ -532,43 +532,31 @@ int persistent_blocks(mlkv_table* t, const void* kernel, int threads);
 #endif
 
 namespace mlkv {
-// prio: 0, or a scheduling priority for the launch's blocks (lower is
-// placed first, as for stream priorities; kept by graph capture)
 template <typename... Params, typename... Args>
-inline void launch_kernel(bool pdl, int prio, void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+inline void launch_kernel(bool pdl, void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
                           cudaStream_t st, Args&&... args) {
-    cudaLaunchAttribute attr[2];
-    int na = 0;
-    if (MLKV_PDL && pdl) {
-        attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr[na].val.programmaticStreamSerializationAllowed = 1;
-        ++na;
-    }
-    if (prio) {
-        attr[na].id = cudaLaunchAttributePriority;
-        attr[na].val.priority = prio;
-        ++na;
-    }
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = block;
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
     cfg.attrs = attr;
-    cfg.numAttrs = na;
+    cfg.numAttrs = MLKV_PDL && pdl ? 1 : 0;
     cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);  // an error stays in cudaGetLastError()
 }
 }  // namespace mlkv
 
 // Launch helper: counts the launch and records timing events when asked.
-#define MLKV_LAUNCH_PDL_PRIO(pdl, prio, t, kid, kernel, grid, block, smem, stream, ...)                      \
-    do {                                                                                                     \
-        mlkv::timer_before((t), (kid), (stream));                                                            \
-        mlkv::launch_kernel((pdl), (prio), kernel, dim3(grid), dim3(block), (smem), (stream), __VA_ARGS__);   \
-        mlkv::timer_after((t), (kid), (stream));                                                             \
-        (t)->launches++;                                                                                     \
+#define MLKV_LAUNCH_PDL(pdl, t, kid, kernel, grid, block, smem, stream, ...)                      \
+    do {                                                                                          \
+        mlkv::timer_before((t), (kid), (stream));                                                 \
+        mlkv::launch_kernel((pdl), kernel, dim3(grid), dim3(block), (smem), (stream), __VA_ARGS__); \
+        mlkv::timer_after((t), (kid), (stream));                                                  \
+        (t)->launches++;                                                                          \
     } while (0)
-#define MLKV_LAUNCH_PDL(pdl, ...) MLKV_LAUNCH_PDL_PRIO(pdl, 0, __VA_ARGS__)
 #define MLKV_LAUNCH(...) MLKV_LAUNCH_PDL(true, __VA_ARGS__)
 // The persistent grids (one wave, each block a fixed share of the work) may
 // start as the kernel before them drains too; -DMLKV_PDL_PERSISTENT=0 makes
@@ -577,4 +565,3 @@ inline void launch_kernel(bool pdl, int prio, void (*kernel)(Params...), dim3 gr
 #define MLKV_PDL_PERSISTENT 1
 #endif
 #define MLKV_LAUNCH_PERSISTENT(...) MLKV_LAUNCH_PDL(MLKV_PDL_PERSISTENT != 0, __VA_ARGS__)
-#define MLKV_LAUNCH_PERSISTENT_PRIO(prio, ...) MLKV_LAUNCH_PDL_PRIO(MLKV_PDL_PERSISTENT != 0, prio, __VA_ARGS__)
