@@ -31,9 +31,10 @@
 //                 fewer than 2^19 lookups) of a long run
 //                 (Zipf-hot keys reach 10^4-10^5 lookups): the chunk's sum,
 //                 compensated, to scratch as a (sum, compensation) pair.
-//  k_long_combine one block per long run: the chunk pairs are split over the
-//                 block's lane groups in a fixed way, added in that order with
-//                 compensation, the sum rounded once, and the row updated.
+//  k_long_combine per long run: the chunk pairs added in a fixed order with
+//                 compensation (split over a whole block's lane groups for the
+//                 runs of many chunks, one lane group for the others), the sum
+//                 rounded once, and the row updated.
 // Long runs are summed with compensation because the Adagrad step is
 // ill-conditioned where a summed gradient element lands near eps (with zero
 // state, u = lr * g / (|g| + eps) changes fast in g there): a plain fp32 sum
@@ -62,7 +63,8 @@ namespace {
 #endif
 constexpr uint32_t kChunkLarge = 64, kChunkSmall = MLKV_CHUNK_SMALL, kSmallBatch = MLKV_SMALL_BATCH;
 // Long runs of more than `big` chunk sums (the hottest rows) are combined by a
-// whole 1024-thread block of k_long_combine; the rest by one lane group each.
+// whole block of k_long_combine (MLKV_COMBINE_THREADS); the rest by one lane
+// group each.
 // In calls of at least kSmallBatch lookups, big = kBigRunLarge (many long
 // runs: lane groups keep the SMs busy); below, kBigRunSmall (few long runs:
 // blocks sum their chunks in parallel).
