@@ -840,13 +840,14 @@ cudaError_t launch_probe(mlkv_table* t, const int64_t* keys, int64_t n, bool ins
                 MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<false, 1024>), g, 1024, 0, st, index_args(t), keys,
                             (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, ra, m,
                             (int)memo, *fc);
-        } else {
+        } else {  // the small tiles: kSortTileSmall / kProbeKeys threads
+            constexpr int CT = kSortTileSmall / kProbeKeys;
             if (insert)
-                MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<true, 256>), g, 256, 0, st, index_args(t), keys,
+                MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<true, CT>), g, CT, 0, st, index_args(t), keys,
                             (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, 0, m,
                             (int)memo, *fc);
             else
-                MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<false, 256>), g, 256, 0, st, index_args(t), keys,
+                MLKV_LAUNCH(t, MLKV_K_PROBE, (k_probe<false, CT>), g, CT, 0, st, index_args(t), keys,
                             (uint32_t)n, rows, slot_of_pos, t->s.miss_pos, t->s.miss_slot, cur, nxt, ra, m,
                             (int)memo, *fc);
         }

@@ -30,7 +30,12 @@ constexpr int kSortMaxPasses = 4;      // row ids have at most 31 bits
 constexpr int kSortMaxDigitBits = 9;   // radix <= 512
 constexpr int kSortMaxRadix = 1 << kSortMaxDigitBits;
 constexpr int kSortTile = 4096;        // lookups per tile of a sort pass ...
-constexpr int kSortTileSmall = 1024;   // ... and in batches of fewer than kSortSmallBatch lookups
+#ifndef MLKV_SORT_SMALL_TILE_SHIFT
+#define MLKV_SORT_SMALL_TILE_SHIFT 10
+#endif
+constexpr int kSortTileSmallShift = MLKV_SORT_SMALL_TILE_SHIFT;
+constexpr int kSortTileSmall = 1 << kSortTileSmallShift;  // ... and in batches of fewer than kSortSmallBatch lookups
+static_assert(kSortTileSmallShift >= 9 && kSortTileSmallShift <= 11, "small tiles of 512 .. 2048 lookups");
 #ifndef MLKV_SORT_SMALL_BATCH
 #define MLKV_SORT_SMALL_BATCH (1u << 19)
 #endif
@@ -38,7 +43,7 @@ constexpr uint32_t kSortSmallBatch = MLKV_SORT_SMALL_BATCH;
 // log2 of the sort's tile for a batch of n lookups: small batches take small
 // tiles, so that a pass still spreads over the SMs (200k lookups are 49 tiles
 // of 4096 but 196 of 1024)
-inline int sort_tile_shift(int64_t n) { return n < (int64_t)kSortSmallBatch ? 10 : 12; }
+inline int sort_tile_shift(int64_t n) { return n < (int64_t)kSortSmallBatch ? kSortTileSmallShift : 12; }
 constexpr int kSmallRun = 4;           // runs of 2 .. kSmallRun lookups carry their positions in their record
 constexpr int64_t kMaxStaleness = MLKV_MAX_STALENESS;  // largest bound kept below no bound
 

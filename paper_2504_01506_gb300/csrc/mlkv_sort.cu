@@ -114,15 +114,16 @@ __device__ __forceinline__ uint32_t digit_peers(uint32_t dig, bool valid, int bi
 // counts the probe did not make.  A thread counts consecutive elements and
 // adds a run of equal digits with one atomic.
 template <int TILE>
-__global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restrict__ kin, uint32_t n,
+__global__ void __launch_bounds__(TILE >= 1024 ? kThreads : TILE / 4) k_sort_hist(const uint32_t* __restrict__ kin, uint32_t n,
                                                         uint32_t* __restrict__ counts, uint32_t* __restrict__ dtot,
                                                         uint32_t ntiles, int shift, int radix, uint32_t sent,
                                                         int first) {
-    constexpr int kItems = TILE / kThreads;
+    constexpr int kHThreads = TILE >= 1024 ? kThreads : TILE / 4;
+    constexpr int kItems = TILE / kHThreads;
     static_assert(kItems % 4 == 0, "whole 16-byte loads");
     pdl_enter();
     __shared__ uint32_t hist[kMaxRadix];
-    for (int d = threadIdx.x; d < radix; d += kThreads) hist[d] = 0;
+    for (int d = threadIdx.x; d < radix; d += kHThreads) hist[d] = 0;
     __syncthreads();
     const uint32_t i0 = blockIdx.x * TILE + threadIdx.x * kItems;
     uint32_t key[kItems];
@@ -154,7 +155,7 @@ __global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* __restri
     }
     if (cnt) atomicAdd(&hist[cur], cnt);
     __syncthreads();
-    for (int d = threadIdx.x; d < radix; d += kThreads) {
+    for (int d = threadIdx.x; d < radix; d += kHThreads) {
         const uint32_t c = hist[d];
         counts[(size_t)d * ntiles + blockIdx.x] = c;
         if (c) atomicAdd(dtot + d, c);
@@ -241,9 +242,9 @@ __global__ void __launch_bounds__(kOThreads) k_sort_offsets(const uint32_t* __re
 // entry), and to the next pass's digit totals ndtot.  The counts this pass's
 // offsets came from (`counts`, read by the offsets kernel, which has
 // finished) are zeroed, for the pass after next to count into.
-// threads of the scatter's block for tiles of 1024 (4 elements a thread)
+// threads of the scatter's block for the small tiles (4 elements a thread)
 #ifndef MLKV_SCATTER_SMALL_THREADS
-#define MLKV_SCATTER_SMALL_THREADS 256
+#define MLKV_SCATTER_SMALL_THREADS (kSortTileSmall / 4)
 #endif
 #ifndef MLKV_SCATTER_MIN_BLOCKS
 #define MLKV_SCATTER_MIN_BLOCKS 3
@@ -256,8 +257,8 @@ __global__ void __launch_bounds__(THREADS, THREADS == 512 ? MLKV_SCATTER_MIN_BLO
     uint32_t* __restrict__ ndtot, uint32_t* __restrict__ counts) {
     constexpr int kSWarps = THREADS / 32;
     constexpr int kSItems = TILE / THREADS;
-    constexpr int kTileShift = TILE == 4096 ? 12 : 10;
-    static_assert(TILE == (1 << kTileShift), "tiles of 4096 or 1024");
+    constexpr int kTileShift = TILE == 4096 ? 12 : TILE == 2048 ? 11 : TILE == 1024 ? 10 : 9;
+    static_assert(TILE == (1 << kTileShift), "tiles of 512 .. 4096");
     pdl_enter();
     // the pass's digit totals were read by the offsets kernel, which has
     // finished: zero them for the next sort (the totals are zero between sorts)
@@ -514,7 +515,8 @@ void sort_passes(mlkv_table* t, int64_t n, cudaStream_t st, const uint32_t** sro
         const int first = p == 0;
         uint32_t* dtot = t->s.sort_dtot + p * kMaxRadix;
         if (first && !first_counted)
-            MLKV_LAUNCH(t, 0, k_sort_hist<TILE>, nt, kThreads, 0, st, kin, (uint32_t)n, counts[0], dtot, nt, 0,
+            MLKV_LAUNCH(t, 0, k_sort_hist<TILE>, nt, TILE >= 1024 ? kThreads : TILE / 4, 0, st, kin, (uint32_t)n,
+                        counts[0], dtot, nt, 0,
                         radix, sent, first);
         // launched after the kernel before it has finished, not beside its
         // drain: placed early, its few blocks landed on the SMs the scatter
