@@ -42,6 +42,10 @@
  *     the kernel that gives new keys their rows, between the blocks of that
  *     one grid (one block per SM; the next kernel may launch only after them),
  *     bounded: one that runs out records MLKV_ERR_TIMEOUT.
+ *   - Each call that enqueues work, and mlkv_open / close / sync /
+ *     clear_status, is an NVTX range named after the call ("mlkv_get",
+ *     "mlkv_apply_grad", ...), for timeline tools; the kernels it launches
+ *     fall inside it.
  */
 #ifndef MLKV_GPU_H
 #define MLKV_GPU_H
