@@ -93,6 +93,13 @@ constexpr uint32_t kBigRunLarge = 32, kBigRunSmall = 4;
 #ifndef MLKV_REDUCE_BRANCHES
 #define MLKV_REDUCE_BRANCHES 1
 #endif
+// Narrow rows (a row on at most 16 lanes: dim <= 64): runs of one lookup two
+// at a time per lane group on at most 3 blocks per SM, runs of 5-32 lookups
+// with 4 gradient rows in flight at 3 blocks per SM (more warps); 0: the
+// wide rows' kernels for every dim.
+#ifndef MLKV_NARROW_ROWS
+#define MLKV_NARROW_ROWS 1
+#endif
 // k_single on at most this many blocks per SM (0: as many as fit).
 #ifndef MLKV_SINGLE_PER_SM
 #define MLKV_SINGLE_PER_SM 0
@@ -353,7 +360,7 @@ __device__ __forceinline__ void write_long_runs(const RunArgs& a, const uint32_t
 // One short run [s, s + len) of `row`, first lookup p0, by one lane group: the
 // row, the state and the first gradient row are loaded together, the rest of
 // the gradient rows are added in occurrence order, then the Adagrad step.
-template <int V, int KV>
+template <int V, int KV, int ROWS = MLKV_REDUCE_ROWS_IN_FLIGHT>
 __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, uint32_t s, uint32_t len,
                                           uint32_t row, uint32_t p0, int glane, unsigned gmask) {
     using VT = typename Vec<V>::T;
@@ -375,7 +382,7 @@ __device__ __forceinline__ void short_run(const RowArgs& ra, const RunArgs& a, u
         if (j < ra.NV) Vec<V>::add(acc[k], __ldcs(g0 + j));  // 0 + g: first term, in order
     }
     if (len > 1)
-        sum_rows<V, KV, MLKV_REDUCE_ROWS_IN_FLIGHT, true>(acc, acc, a.grads, a.spos, s + 1, rest, ra.d, ra.NV,
+        sum_rows<V, KV, ROWS, true>(acc, acc, a.grads, a.spos, s + 1, rest, ra.d, ra.NV,
                                                           ra.G, glane, gmask, a.err, kChkShortPos, a.n, pl0);
     adagrad_store<V, KV>(ra, row, w, Gs, acc, glane, a.lr, a.eps);
 }
@@ -598,8 +605,8 @@ __device__ __forceinline__ uint4 run_meta(const RunArgs& a, uint32_t u, uint32_t
     return u < U ? __ldg(a.runs + u) : make_uint4(0u, 0u, 0u, 0u);
 }
 
-template <int V, int KV>
-__global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra, RunArgs a) {
+template <int V, int KV, int ROWS = MLKV_REDUCE_ROWS_IN_FLIGHT>
+__global__ void __launch_bounds__(256, ROWS >= 8 ? MLKV_SHORT_MIN_BLOCKS : 3) k_short(RowArgs ra, RunArgs a) {
     pdl_enter();
     if (MLKV_CHECK && !in_bounds(a.err, kChkListEntry, a.cur->n_short, (unsigned long long)a.n + 1)) return;
     const uint32_t U = min(a.cur->n_short, a.n);  // a list never holds more runs than lookups
@@ -620,7 +627,7 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
         for (uint32_t u = base; u < end; ++u) {
             const uint4 m = next;  // (start, end, row, first lookup)
             next = run_meta(a, u + 1, end);
-            short_run<V, KV>(ra, a, m.x, m.y - m.x, m.z, m.w, glane, gmask);
+            short_run<V, KV, ROWS>(ra, a, m.x, m.y - m.x, m.z, m.w, glane, gmask);
         }
         uint32_t c = 0;
         if (glane == 0) c = atomicAdd(&a.cur->short_next, grab);
@@ -634,11 +641,10 @@ __global__ void __launch_bounds__(256, MLKV_SHORT_MIN_BLOCKS) k_short(RowArgs ra
 // ahead; the sum is the gradient row itself (0 + g), then the Adagrad step.
 // With no loop over positions it needs few registers, so more warps (and
 // rows) are in flight than in k_short.
-template <int V, int KV>
-__global__ void __launch_bounds__(256, MLKV_SINGLE_MIN_BLOCKS) k_single(RowArgs ra, RunArgs a) {
+template <int V, int KV, int SG = MLKV_SINGLES>
+__global__ void __launch_bounds__(256, SG == 1 ? MLKV_SINGLE_MIN_BLOCKS : 4) k_single(RowArgs ra, RunArgs a) {
     pdl_enter();
     using VT = typename Vec<V>::T;
-    constexpr int SG = MLKV_SINGLES;
     if (MLKV_CHECK && !in_bounds(a.err, kChkListEntry, a.cur->n_single, (unsigned long long)a.n + 1)) return;
     const uint32_t U = min(a.cur->n_single, a.n);  // a list never holds more runs than lookups
     const int lane = threadIdx.x & 31, G = ra.G, glane = lane & (G - 1);
@@ -910,6 +916,14 @@ __global__ void __launch_bounds__(1024) k_long_combine(RowArgs ra, RunArgs a, De
 }
 
 template <int V, int KV>
+void launch_short(mlkv_table* t, bool narrow, int grid, cudaStream_t st, const RowArgs& ra, const RunArgs& a) {
+    if (narrow)
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV, 4>), grid, 256, 0, st, ra, a);
+    else
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), grid, 256, 0, st, ra, a);
+}
+
+template <int V, int KV>
 cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, const uint32_t* spos,
                        int64_t n, uint32_t sent, cudaStream_t st, CallCounters* cur) {
     RowArgs ra{t->slots, t->geom.stride, t->geom.dpad, t->geom.NV, t->geom.G, t->geom.d,
@@ -952,9 +966,13 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
     }
     const int gl = persistent_blocks(t, (const void*)k_long_sum<V, KV>, 256);
     const int g2 = persistent_blocks(t, (const void*)k_small<V, KV>, 256);
-    const int gs = persistent_blocks(t, (const void*)k_short<V, KV>, 256);
-    int g1 = persistent_blocks(t, (const void*)k_single<V, KV>, 256);
+    const bool narrow = MLKV_NARROW_ROWS && t->geom.G <= 16;
+    const void* short_k = narrow ? (const void*)k_short<V, KV, 4> : (const void*)k_short<V, KV>;
+    const void* single_k = narrow ? (const void*)k_single<V, KV, 2> : (const void*)k_single<V, KV>;
+    const int gs = persistent_blocks(t, short_k, 256);
+    int g1 = persistent_blocks(t, single_k, 256);
     if (MLKV_SINGLE_PER_SM > 0 && g1 > MLKV_SINGLE_PER_SM * t->num_sms) g1 = MLKV_SINGLE_PER_SM * t->num_sms;
+    if (narrow && g1 > 3 * t->num_sms) g1 = 3 * t->num_sms;
     // the combine's block (MLKV_COMBINE_THREADS): the groups' (sum,
     // compensation) pairs must fit the default 48 KB of shared memory
     int big = MLKV_COMBINE_THREADS;
@@ -978,13 +996,16 @@ cudaError_t run_reduce(mlkv_table* t, const float* grads, const uint32_t* srow, 
         // the runs of 5-32 (the longest per run of the three) before those of
         // 2-4: in a small batch the runs of 5-32 would otherwise be last to
         // start, after the runs of one had filled the SMs
-        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, a);
+        launch_short<V, KV>(t, narrow, gs, s1, ra, a);
         MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, s1, ra, tail);
     } else {
         MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SMALL, (k_small<V, KV>), g2, 256, 0, s1, ra, a);
-        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SHORT, (k_short<V, KV>), gs, 256, 0, s1, ra, tail);
+        launch_short<V, KV>(t, narrow, gs, s1, ra, tail);
     }
-    MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, s_single, ra, tail);
+    if (narrow)
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV, 2>), g1, 256, 0, s_single, ra, tail);
+    else
+        MLKV_LAUNCH_PERSISTENT(t, MLKV_K_REDUCE_SINGLE, (k_single<V, KV>), g1, 256, 0, s_single, ra, tail);
     if (branches) {
         cudaError_t e;
         if ((e = cudaEventRecord(t->ev_join[0], s1)) != cudaSuccess ||
