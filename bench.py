@@ -15,9 +15,10 @@ per launch over its CUDA-event duration against the measured HBM copy peak;
 `cpu_baseline` is the oracle (single thread, host cores) on a bounded sample.
 
 With the default DLRM workload at N=1 the same process then measures the
-knowledge-graph, GNN and tiered workloads one after another (each store closed
-before the next opens) and reports them under `per_config`, each with its own
-roofline, clocks and oracle baseline.
+knowledge-graph, GNN and tiered workloads and the YCSB-shaped Get/Put batches
+(Zipf and uniform keys) one after another (each store closed before the next
+opens) and reports them under `per_config`, each with its own metric, roofline,
+clocks and oracle baseline.
 
 `--gpus N` without a launcher's environment starts N replica ranks itself
 (torch.distributed.run on this host, one process per GPU).
@@ -905,7 +906,9 @@ def per_config_names(args, world) -> list:
     if args.per_config == "none" or world > 1:
         return []
     if args.per_config == "auto":
-        return ["kg", "gnn", "tiered"] if args.config == "dlrm" and args.scale == 1 and not args.staleness else []
+        if args.config != "dlrm" or args.scale != 1 or args.staleness:
+            return []
+        return ["kg", "gnn", "tiered", "ycsb", "ycsb-uniform"]
     return [c for c in args.per_config.split(",") if c]
 
 
@@ -934,8 +937,9 @@ def run_ours(args, cfg):
         # each workload's own step count (the timed region stays short), at most --steps
         r = measure(args, c, dist, rank, local, world, dev, headline=False, steps=min(args.steps, c.steps))
         r.pop("e2e", None)
-        r["metric"] = METRIC
-        r["unit"] = UNIT
+        kvc = isinstance(c, W.YcsbConfig)
+        r["metric"] = METRIC_YCSB if kvc else METRIC
+        r["unit"] = UNIT_YCSB if kvc else UNIT
         extra[name] = r
     if rank == 0:
         line = {
@@ -982,7 +986,8 @@ def main():
                     help="also event-time every kernel class over the timed steps (run call by call)")
     ap.add_argument("--per-config", default="auto",
                     help="workloads measured after the headline one in the same process, comma-separated "
-                         "(auto: kg,gnn,tiered after the default DLRM workload at N=1; none: no others)")
+                         "(auto: kg,gnn,tiered,ycsb,ycsb-uniform after the default DLRM workload at N=1; "
+                         "none: no others)")
     ap.add_argument("--traffic-record", metavar="CSV",
                     help="write the DRAM bytes per launch in this ncu CSV (dram__bytes_read.sum and "
                          "dram__bytes_write.sum of this command line's timed steps) into profiles/traffic.json "
