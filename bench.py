@@ -363,7 +363,10 @@ def record_traffic(args, cfg, csv_path: str, path=None) -> dict:
             by_kid.setdefault(kid, ([], name))[0].append(b)
     pool = max(1, min(args.pool, args.steps + args.warmup))
     steps_idx = [(args.warmup + i) % pool for i in range(args.steps)]
-    stats = {j: batch_stats(cfg.batch_keys(j), cfg.dim) for j in set(steps_idx)}
+    if isinstance(cfg, W.YcsbConfig):  # a batch of Gets, then Puts (the bytes measure() uses)
+        stats = {j: ycsb_stats(*cfg.ops(j)[:2], cfg.dim) for j in set(steps_idx)}
+    else:
+        stats = {j: batch_stats(cfg.batch_keys(j), cfg.dim) for j in set(steps_idx)}
     passes = -(-int(cfg.n_keys).bit_length() // 9)
     out = {}
     for kid, (bs, name) in sorted(by_kid.items()):

@@ -125,3 +125,27 @@ def test_traffic_record_from_an_ncu_csv(tmp_path):
     s = bench.batch_stats(cfg.batch_keys(1), cfg.dim)  # the timed step replays batch (3 + 0) % 2
     assert out["1"]["algorithmic_bytes_per_launch"] == bench.kernel_bytes(s, 1, 2)
     assert json.loads(out_path.read_text())[cfg.name]["3"]["source_sha"] == bench.source_sha(3)
+
+
+def test_traffic_record_of_get_put_batches_uses_their_gets(tmp_path):
+    """For the YCSB-shaped batches the Get reads only the batch's Get keys: the
+    record's algorithmic bytes are those of ycsb_stats (what the bench's own
+    roofline uses), not of every key of the batch."""
+    import argparse
+
+    import workloads as W
+
+    cfg = W.scaled(W.ycsb(), 50_000, 64)  # 1,000 records, batches of 16,384 operations
+    hdr = ["ID", "Process ID", "Process Name", "Host Name", "Kernel Name", "Context", "Stream", "Block Size",
+           "Grid Size", "Device", "CC", "Section Name", "Metric Name", "Metric Unit", "Metric Value"]
+    name = "void (anonymous namespace)::k_get<4, 2, 1>(IndexArgs)"
+    rows = [hdr] + [[ "0", "1", "python", "h", name, "1", "7", "(256, 1, 1)", "(1, 1, 1)", "0", "10.3",
+                      "Command line", m, "byte", "100"] for m in ("dram__bytes_read.sum", "dram__bytes_write.sum")]
+    csv_path = tmp_path / "launches.csv"
+    csv_path.write_text("\n".join(",".join('"%s"' % c for c in r) for r in rows) + "\n")
+    args = argparse.Namespace(pool=2, steps=1, warmup=3, scale=50_000)
+    out = bench.record_traffic(args, cfg, str(csv_path), str(tmp_path / "traffic.json"))
+    read, write, _ = cfg.ops(1)  # the timed step replays batch (3 + 0) % 2
+    want = bench.kernel_bytes(bench.ycsb_stats(read, write, cfg.dim), 1, 1)
+    assert out["1"]["algorithmic_bytes_per_launch"] == want
+    assert want < bench.kernel_bytes(bench.batch_stats(cfg.batch_keys(1), cfg.dim), 1, 1)
